@@ -1,0 +1,36 @@
+"""Write the oracle's tiny fp32 tree (seed 0) to tiny_f32_seed0.json.
+
+Calls only oracle/ and synth/. Run from the repository root:
+    python tests/golden/make_golden.py
+"""
+import json
+import os
+import sys
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, os.path.dirname(os.path.dirname(HERE)))
+
+import synth  # noqa: E402
+from oracle import treeflash_oracle as O  # noqa: E402
+
+
+def main():
+    out = {}
+    for name in ("tiny_f32", "tiny_peaked"):
+        cfg = synth.get_config(name)
+        inp = synth.make_inputs(cfg)
+        W = O.weights_f64(inp, synth.to_f64)
+        H = synth.to_f64(inp["hidden"])[0]
+        res = O.draft_sequence(H, int(inp["root_tok"][0]), int(inp["root_pos"][0]), W,
+                               M=cfg.M, K2=cfg.K2, B=cfg.B, temperature=cfg.temperature,
+                               eps=cfg.rms_eps, mode=cfg.mode)
+        out[name] = dict(tok=res.tree.tok.tolist(), parent=res.tree.parent.tolist(),
+                         depth=res.tree.depth.tolist(),
+                         score=[float(x) for x in res.tree.score],
+                         top_ids=res.top_ids.tolist())
+    with open(os.path.join(HERE, "tiny_f32_seed0.json"), "w") as f:
+        json.dump(out, f, indent=1)
+
+
+if __name__ == "__main__":
+    main()
