@@ -1,0 +1,225 @@
+/*
+ * treeflash.h - C ABI of the TreeFlash drafting hot path on one GB300 (sm_103a).
+ *
+ * TreeFlash ("Parallel AR-Approximation for Faster Speculative Decoding") drafts a tree of
+ * B candidate tokens from the gamma hidden states h_{t+1..t+gamma} that a one-shot block
+ * drafter produces in a single forward pass. Algorithm 1 (App. B, "AR-approximated OPT-Tree
+ * construction") has two parts, and this library runs both on the GPU:
+ *
+ *   Part 1, stage 1  (tf_stage1_marginals)  q_{t+i} = LMHead(h_{t+i}); TopM per depth.
+ *   Part 1, stage 2  (tf_stage2_ar_approx)  h' = h + SwiGLU(h~ :: e) (Eq. 1) on 1 + M(gamma-1)
+ *                                           rows, each through the LM head, log-softmax, top-K2.
+ *   Part 2           (tf_build_tree)        OPT-Tree best-first selection of B nodes (Sec. 3,
+ *                                           "Inference"), the M-ary rule for non-leaves.
+ *   verification     (tf_tree_mask)         ancestor mask and position ids for the verifier's
+ *                                           single parallel pass over the tree (Sec. 1, Sec. 3).
+ *
+ * Conventions shared by every call:
+ *  - Pointers are DEVICE pointers owned by the caller unless a parameter says "host". The
+ *    library allocates no memory and keeps no state between calls; scratch lives in the
+ *    caller's workspace (tf_workspace_size). Calls are asynchronous on `stream` (NULL = the
+ *    legacy default stream) and return once the work is queued.
+ *  - Shapes are row-major. b = batch (independent sequences), d = hidden size, V = vocabulary,
+ *    I = approximator width, gamma = block size, M = stage-1 candidates per depth, K2 =
+ *    children kept per stage-2 row, B = draft budget (non-root nodes),
+ *    R = 1 + M (gamma - 1) stage-2 rows per sequence, K1 = max(M, K2).
+ *  - Float tensors have the element type of dims->dtype (TF_BF16: __nv_bfloat16, TF_F32:
+ *    float); log-probabilities are always float32, token ids int32.
+ *  - Errors: a call that finds an invalid argument returns TF_ERR_INVALID_ARG,
+ *    TF_ERR_UNSUPPORTED or TF_ERR_WORKSPACE before queueing anything; a failed launch returns
+ *    TF_ERR_CUDA. Conditions only the GPU can see (an out-of-range token id, an underfull
+ *    candidate universe, a bounded wait that gave up) are OR-ed into device status words
+ *    (TF_DEV_* bits) that the caller reads after synchronising. No call aborts the process.
+ *  - Ties (the paper is silent): inside a distribution the larger value comes first, then the
+ *    smaller token id; in the queue the larger path score, then the smaller depth, then the
+ *    smaller parent index, then the smaller token id.
+ */
+#ifndef TREEFLASH_H
+#define TREEFLASH_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A cudaStream_t; declared here so the header needs no CUDA include. */
+typedef struct CUstream_st* tf_stream_t;
+
+typedef enum {
+    TF_OK = 0,
+    TF_ERR_INVALID_ARG = 1,   /* null pointer, inconsistent or out-of-range dimension */
+    TF_ERR_UNSUPPORTED = 2,   /* valid but outside what the kernels implement (see limits) */
+    TF_ERR_WORKSPACE = 3,     /* workspace null, too small or not 256-byte aligned */
+    TF_ERR_CUDA = 4,          /* a CUDA runtime/driver call or a kernel launch failed */
+    TF_ERR_DEVICE_STATUS = 5, /* tf_status_read found TF_DEV_* flags set */
+    TF_ERR_TIMEOUT = 6        /* tf_status_read found TF_DEV_TIMEOUT set */
+} tf_status;
+
+typedef enum { TF_BF16 = 0, TF_F32 = 1 } tf_dtype;
+
+typedef enum {
+    TF_MODE_AR = 0,            /* TreeFlash: stage-2 conditional rows, M-ary rule (Alg. 1) */
+    TF_MODE_MARGINAL = 1,      /* DDTree baseline: OPT-Tree on the stage-1 marginals, every
+                                  node expandable (Sec. 4 "Baselines") */
+    TF_MODE_MARGINAL_MARY = 2  /* stage-1 marginals under the M-ary rule: what TF_MODE_AR
+                                  computes when the approximator is zero (Sec. 3 "Training") */
+} tf_mode;
+
+/* Device status bits (int32 words written with atomic OR). */
+enum {
+    TF_DEV_BAD_TOKEN = 1,      /* a token id outside [0, V) was read; the row/node is skipped */
+    TF_DEV_UNDERFULL = 2,      /* fewer than B candidates exist; missing nodes are marked */
+    TF_DEV_NONFINITE = 4,      /* a non-finite logit or score was seen */
+    TF_DEV_TIMEOUT = 8,        /* a bounded wait inside a kernel gave up; outputs invalid */
+    TF_DEV_RECOMPUTED = 16     /* informational: a top-k list was recomputed exactly */
+};
+
+typedef struct {
+    int32_t batch;        /* b >= 1 */
+    int32_t d;            /* hidden size; TF_BF16 needs d % 64 == 0, TF_F32 d % 4 == 0 */
+    int32_t V;            /* vocabulary size, K1 <= V < 2^31 */
+    int32_t I;            /* approximator intermediate width; TF_BF16 needs I % 64 == 0 */
+    int32_t gamma;        /* block size (max depth), 1..64 */
+    int32_t M;            /* stage-1 candidates per depth (M-ary branching), 1..32 */
+    int32_t K2;           /* children kept per distribution, 1..64; K2 >= B is exact */
+    int32_t B;            /* draft budget (nodes besides the root), 1..1023 */
+    float temperature;    /* logits are W_lm x / temperature, temperature > 0 */
+    float rms_eps;        /* RMSNorm epsilon of Eq. 1's normalisations */
+    int32_t dtype;        /* tf_dtype */
+    int32_t mode;         /* tf_mode */
+} tf_dims;
+
+/* Model parameters (device, dims->dtype, row-major, read only, never copied). */
+typedef struct {
+    const void* lm_head;  /* [V, d]  verifier output embedding W_lm */
+    const void* embed;    /* [V, d]  verifier input embedding Embd */
+    const void* norm_h;   /* [d]     RMSNorm weight of the hidden-state half of Eq. 1 */
+    const void* norm_e;   /* [d]     RMSNorm weight of the embedding half of Eq. 1 */
+    const void* w_gate;   /* [I, 2d] SwiGLU gate projection, input [h~ ; e] */
+    const void* w_up;     /* [I, 2d] SwiGLU up projection, input [h~ ; e] */
+    const void* w_down;   /* [d, I]  SwiGLU down projection */
+} tf_weights;
+
+/* Human-readable name of a status code (static storage). */
+const char* tf_status_string(tf_status status);
+
+/* Library version as major*10000 + minor*100 + patch. */
+int32_t tf_version(void);
+
+/* Validate `dims` and return the workspace bytes every call below needs for these dims
+ * (the maximum over all calls, so one buffer serves the whole step). Host only; no GPU
+ * work. The workspace must be device memory, 256-byte aligned, and must not be used by two
+ * calls that overlap on the GPU. */
+tf_status tf_workspace_size(const tf_dims* dims, size_t* bytes);
+
+/* Zero the workspace's status word (asynchronous). tf_stage1_marginals does this itself. */
+tf_status tf_status_reset(void* ws, size_t ws_bytes, tf_stream_t stream);
+
+/* Synchronise `stream`, copy the workspace's status word to *flags (host) and return
+ * TF_ERR_TIMEOUT if TF_DEV_TIMEOUT is set, TF_ERR_DEVICE_STATUS if any other error bit is
+ * set (TF_DEV_RECOMPUTED alone is not an error), TF_OK otherwise. */
+tf_status tf_status_read(const void* ws, size_t ws_bytes, int32_t* flags, tf_stream_t stream);
+
+/* Stage 1 of Algorithm 1 Part 1: for every sequence s and depth i,
+ *   q_{t+i} = softmax(W_lm h_{t+i} / T) and its K1 largest entries.
+ *  hidden   [b, gamma, d] dtype: the drafter's hidden states h_{t+1..t+gamma}.
+ *  top_ids  [b, gamma, K1] int32 out: token ids in the tie order above; the first M are the
+ *           candidates x^(1..M)_{t+i} of the M-ary tree.
+ *  top_logp [b, gamma, K1] float out: log q_{t+i}(top_ids), exact log-softmax over all V.
+ * Resets the workspace status word. */
+tf_status tf_stage1_marginals(const tf_dims* dims, const tf_weights* w, const void* hidden,
+                              int32_t* top_ids, float* top_logp,
+                              void* ws, size_t ws_bytes, tf_stream_t stream);
+
+/* Stage 2 of Algorithm 1 Part 1 (Eq. 1): for every sequence, R rows
+ *   row 0:                 h' = h_{t+1} + SwiGLU(RMSNorm(h_{t+1}) :: RMSNorm(Embd(x_t)))
+ *   row 1 + (i-2) M + m:   h' = h_{t+i} + SwiGLU(RMSNorm(h_{t+i}) :: RMSNorm(Embd(x^(m)_{t+i-1})))
+ * for i = 2..gamma, m = 0..M-1, then q' = softmax(W_lm h' / T) and its K2 largest entries.
+ *  hidden     [b, gamma, d] dtype (as in stage 1)
+ *  root_tok   [b] int32: the last accepted token x_t of each sequence
+ *  top_ids    [b, gamma, K1] int32: stage-1 output (the first M per depth are used)
+ *  child_ids  [b, R, K2] int32 out, child_logp [b, R, K2] float out (exact log-softmax).
+ * h' is kept in the workspace (bf16 path: rounded to bf16, as the MLP's output type).
+ * Requires dims->mode == TF_MODE_AR. */
+tf_status tf_stage2_ar_approx(const tf_dims* dims, const tf_weights* w, const void* hidden,
+                              const int32_t* root_tok, const int32_t* top_ids,
+                              int32_t* child_ids, float* child_logp,
+                              void* ws, size_t ws_bytes, tf_stream_t stream);
+
+/* Algorithm 1 Part 2 (OPT-Tree selection, Sec. 3): one warp per sequence grows the tree by
+ * popping the candidate of highest cumulative log-probability B times. The root's children
+ * are row 0 of child_ids (TF_MODE_AR) or depth 1 of top_ids (marginal modes). A popped node
+ * at depth i < gamma whose token is x^(m)_{t+i} (m < M) makes row 1 + (i-1) M + m available
+ * (TF_MODE_AR); in TF_MODE_MARGINAL every node at depth i < gamma makes stage-1 depth i+1
+ * available, in TF_MODE_MARGINAL_MARY only the M-ary ones do. Each distribution contributes
+ * at most K2 children (exact when K2 >= B). child_ids/child_logp may be NULL in the marginal
+ * modes. Outputs [b, B+1]: node 0 is the root (token root_tok, parent -1, depth 0, score 0);
+ * nodes follow in pop order, so parent < child. Missing nodes (underfull universe) have
+ * token/parent/depth -1 and score -inf, and set TF_DEV_UNDERFULL.
+ *  dev_status [b] int32 out: TF_DEV_* bits per sequence (overwritten, not OR-ed). */
+tf_status tf_build_tree(const tf_dims* dims, const int32_t* root_tok,
+                        const int32_t* top_ids, const float* top_logp,
+                        const int32_t* child_ids, const float* child_logp,
+                        int32_t* node_tok, int32_t* node_parent, int32_t* node_depth,
+                        float* node_score, int32_t* dev_status, tf_stream_t stream);
+
+/* Tree-attention mask and position ids for verifying the tree in one forward pass:
+ *  mask [b, B+1, B+1] uint8 out: mask[s][i][j] = 1 iff node j is node i or an ancestor.
+ *  pos_ids [b, B+1] int32 out: root_pos[s] + depth; -1 for missing nodes (all-zero rows and
+ *  columns in the mask).  root_pos [b] int32. */
+tf_status tf_tree_mask(const tf_dims* dims, const int32_t* node_parent, const int32_t* node_depth,
+                       const int32_t* root_pos, uint8_t* mask, int32_t* pos_ids,
+                       tf_stream_t stream);
+
+/* The whole drafting step for callers holding the step's inputs in HOST memory (pinned memory
+ * makes the copies asynchronous): copies hidden/root_tok/root_pos to the device, runs the four
+ * calls above, copies the tree, mask and status back, and synchronises `stream`.
+ * Host inputs: hidden [b, gamma, d] dtype, root_tok [b], root_pos [b]. Host outputs:
+ * node_tok, node_parent, node_depth [b, B+1] int32, node_score [b, B+1] float,
+ * mask [b, B+1, B+1] uint8, pos_ids [b, B+1] int32, dev_status [b] int32 (per-sequence bits
+ * OR-ed with the workspace status word). Weights stay on the device. The workspace size is
+ * the same tf_workspace_size. Returns TF_ERR_TIMEOUT / TF_ERR_DEVICE_STATUS like
+ * tf_status_read when an error bit is set. */
+tf_status tf_draft_tree_host(const tf_dims* dims, const tf_weights* w, const void* hidden,
+                             const int32_t* root_tok, const int32_t* root_pos,
+                             int32_t* node_tok, int32_t* node_parent, int32_t* node_depth,
+                             float* node_score, uint8_t* mask, int32_t* pos_ids,
+                             int32_t* dev_status, void* ws, size_t ws_bytes, tf_stream_t stream);
+
+/* ------------------------------------------------------------------------------------------
+ * The pieces the stage calls are made of. tf_stage1_marginals is tf_lmhead_partials +
+ * tf_lmhead_merge on the hidden states; tf_stage2_ar_approx is tf_ar_approx followed by the
+ * same two on h'. They are exported so a caller (or a profiler) can run or time one kernel.
+ * ---------------------------------------------------------------------------------------- */
+
+/* The LM-head pass fused with log-softmax bookkeeping (Alg. 1 "LMHead" and "TopM"):
+ * streams W_lm once and, for every row r of x [n_rows, d] (dtype) and every block of 256
+ * vocabulary entries, leaves in the workspace the block's max logit, its sum of
+ * exp(logit - max) and its 8 largest (logit, id). Logits never reach memory.
+ * n_rows <= the larger of b*gamma and b*R. */
+tf_status tf_lmhead_partials(const tf_dims* dims, const void* lm_head, const void* x,
+                             int32_t n_rows, void* ws, size_t ws_bytes, tf_stream_t stream);
+
+/* Merge the per-block partials of tf_lmhead_partials into each row's log-sum-exp and exact
+ * top-k (k <= 64): out_ids [n_rows, k] int32, out_logp [n_rows, k] float = logit - LSE. A
+ * block whose 8 kept entries could hide a member of the top-k has its logits recomputed
+ * exactly from lm_head and x (sets TF_DEV_RECOMPUTED), so the result never depends on the
+ * 8-entry truncation. */
+tf_status tf_lmhead_merge(const tf_dims* dims, const void* lm_head, const void* x,
+                          int32_t n_rows, int32_t k, int32_t* out_ids, float* out_logp,
+                          void* ws, size_t ws_bytes, tf_stream_t stream);
+
+/* Eq. 1 on the R rows of every sequence (stage 2 before the LM head): gathers Embd rows,
+ * normalises both halves, runs the SwiGLU MLP and adds the residual.
+ * h_prime [b, R, d] dtype out (may be NULL: then only the workspace copy is written). */
+tf_status tf_ar_approx(const tf_dims* dims, const tf_weights* w, const void* hidden,
+                       const int32_t* root_tok, const int32_t* top_ids, void* h_prime,
+                       void* ws, size_t ws_bytes, tf_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TREEFLASH_H */

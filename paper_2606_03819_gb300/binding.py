@@ -1,0 +1,235 @@
+"""ctypes binding of the TreeFlash C ABI (include/treeflash.h).
+
+Argument marshalling only: every function here passes raw device pointers of torch tensors,
+the current CUDA stream and the dims/weights structs to the function of the same name in
+lib/libtreeflash.so and raises TreeFlashError if it returns a status other than TF_OK. All
+computation happens in the library's CUDA kernels; nothing here computes any part of the
+path, and there is no fallback: without the built library every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "lib", "libtreeflash.so")
+
+TF_OK, TF_ERR_INVALID_ARG, TF_ERR_UNSUPPORTED, TF_ERR_WORKSPACE, TF_ERR_CUDA, TF_ERR_DEVICE_STATUS, \
+    TF_ERR_TIMEOUT = range(7)
+TF_BF16, TF_F32 = 0, 1
+MODES = {"ar": 0, "marginal": 1, "marginal_mary": 2}
+TF_DEV_BAD_TOKEN, TF_DEV_UNDERFULL, TF_DEV_NONFINITE, TF_DEV_TIMEOUT, TF_DEV_RECOMPUTED = 1, 2, 4, 8, 16
+
+
+class TreeFlashError(RuntimeError):
+    def __init__(self, fn: str, status: int, msg: str):
+        super().__init__(f"{fn}: {msg} (status {status})")
+        self.status = status
+
+
+class TfDims(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("d", ctypes.c_int32), ("V", ctypes.c_int32),
+                ("I", ctypes.c_int32), ("gamma", ctypes.c_int32), ("M", ctypes.c_int32),
+                ("K2", ctypes.c_int32), ("B", ctypes.c_int32), ("temperature", ctypes.c_float),
+                ("rms_eps", ctypes.c_float), ("dtype", ctypes.c_int32), ("mode", ctypes.c_int32)]
+
+
+class TfWeights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in
+                ("lm_head", "embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down")]
+
+
+EXPORTS = ("tf_status_string", "tf_version", "tf_workspace_size", "tf_status_reset", "tf_status_read",
+           "tf_stage1_marginals", "tf_stage2_ar_approx", "tf_build_tree", "tf_tree_mask",
+           "tf_draft_tree_host", "tf_lmhead_partials", "tf_lmhead_merge", "tf_ar_approx")
+
+_lib = None
+
+
+def load_library(path: Optional[str] = None) -> ctypes.CDLL:
+    """Load lib/libtreeflash.so (built by __graft_entry__.build()). Raises if it is missing."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise RuntimeError(f"TreeFlash CUDA library not found at {p}; build it with "
+                           "`python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(p)
+    P, I32, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t
+    D, W = ctypes.POINTER(TfDims), ctypes.POINTER(TfWeights)
+    sig = {
+        "tf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+        "tf_version": (I32, []),
+        "tf_workspace_size": (ctypes.c_int, [D, ctypes.POINTER(SZ)]),
+        "tf_status_reset": (ctypes.c_int, [P, SZ, P]),
+        "tf_status_read": (ctypes.c_int, [P, SZ, ctypes.POINTER(I32), P]),
+        "tf_stage1_marginals": (ctypes.c_int, [D, W, P, P, P, P, SZ, P]),
+        "tf_stage2_ar_approx": (ctypes.c_int, [D, W, P, P, P, P, P, P, SZ, P]),
+        "tf_build_tree": (ctypes.c_int, [D, P, P, P, P, P, P, P, P, P, P, P]),
+        "tf_tree_mask": (ctypes.c_int, [D, P, P, P, P, P, P]),
+        "tf_draft_tree_host": (ctypes.c_int, [D, W, P, P, P, P, P, P, P, P, P, P, P, SZ, P]),
+        "tf_lmhead_partials": (ctypes.c_int, [D, P, P, I32, P, SZ, P]),
+        "tf_lmhead_merge": (ctypes.c_int, [D, P, P, I32, I32, P, P, P, SZ, P]),
+        "tf_ar_approx": (ctypes.c_int, [D, W, P, P, P, P, P, P, SZ, P]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype, f.argtypes = res, args
+    if path is None:
+        _lib = lib
+    return lib
+
+
+def _check(fn: str, status: int):
+    if status != TF_OK:
+        msg = load_library().tf_status_string(status).decode()
+        raise TreeFlashError(fn, status, msg)
+
+
+@dataclass(frozen=True)
+class Dims:
+    batch: int
+    d: int
+    V: int
+    I: int
+    gamma: int
+    M: int
+    K2: int
+    B: int
+    temperature: float = 1.0
+    rms_eps: float = 1e-6
+    dtype: str = "bf16"
+    mode: str = "ar"
+
+    @property
+    def R(self) -> int:
+        return 1 + self.M * (self.gamma - 1)
+
+    @property
+    def K1(self) -> int:
+        return max(self.M, self.K2)
+
+    @property
+    def torch_dtype(self):
+        return torch.bfloat16 if self.dtype == "bf16" else torch.float32
+
+    def c(self) -> TfDims:
+        return TfDims(self.batch, self.d, self.V, self.I, self.gamma, self.M, self.K2, self.B,
+                      self.temperature, self.rms_eps, TF_BF16 if self.dtype == "bf16" else TF_F32,
+                      MODES[self.mode])
+
+    @classmethod
+    def from_config(cls, cfg) -> "Dims":
+        return cls(cfg.batch, cfg.d, cfg.V, cfg.I, cfg.gamma, cfg.M, cfg.K2, cfg.B, cfg.temperature,
+                   cfg.rms_eps, cfg.dtype, cfg.mode)
+
+
+WEIGHT_KEYS = ("lm_head", "embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down")
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_contiguous():
+        raise ValueError("tensors passed to the TreeFlash ABI must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def weights_struct(w: dict) -> TfWeights:
+    return TfWeights(*[w[k].data_ptr() if w.get(k) is not None else None for k in WEIGHT_KEYS])
+
+
+def tf_version() -> int:
+    return load_library().tf_version()
+
+
+def tf_workspace_size(dims: Dims) -> int:
+    n = ctypes.c_size_t(0)
+    _check("tf_workspace_size", load_library().tf_workspace_size(ctypes.byref(dims.c()), ctypes.byref(n)))
+    return n.value
+
+
+def alloc_workspace(dims: Dims, device="cuda") -> torch.Tensor:
+    """A torch-owned workspace (256-byte aligned) of tf_workspace_size bytes."""
+    n = tf_workspace_size(dims)
+    buf = torch.empty(n + 256, dtype=torch.uint8, device=device)
+    off = (-buf.data_ptr()) % 256
+    return buf[off:off + n]
+
+
+def tf_status_reset(ws: torch.Tensor, stream=None):
+    _check("tf_status_reset", load_library().tf_status_reset(_ptr(ws), ws.numel(), _stream(stream)))
+
+
+def tf_status_read(ws: torch.Tensor, stream=None, raise_on_error: bool = False) -> int:
+    flags = ctypes.c_int32(0)
+    st = load_library().tf_status_read(_ptr(ws), ws.numel(), ctypes.byref(flags), _stream(stream))
+    if st == TF_ERR_CUDA or raise_on_error:
+        _check("tf_status_read", st)
+    return flags.value
+
+
+def tf_stage1_marginals(dims: Dims, w: dict, hidden, top_ids, top_logp, ws, stream=None):
+    _check("tf_stage1_marginals", load_library().tf_stage1_marginals(
+        ctypes.byref(dims.c()), ctypes.byref(weights_struct(w)), _ptr(hidden), _ptr(top_ids),
+        _ptr(top_logp), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def tf_stage2_ar_approx(dims: Dims, w: dict, hidden, root_tok, top_ids, child_ids, child_logp, ws,
+                        stream=None):
+    _check("tf_stage2_ar_approx", load_library().tf_stage2_ar_approx(
+        ctypes.byref(dims.c()), ctypes.byref(weights_struct(w)), _ptr(hidden), _ptr(root_tok),
+        _ptr(top_ids), _ptr(child_ids), _ptr(child_logp), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def tf_build_tree(dims: Dims, root_tok, top_ids, top_logp, child_ids, child_logp, node_tok, node_parent,
+                  node_depth, node_score, dev_status, stream=None):
+    _check("tf_build_tree", load_library().tf_build_tree(
+        ctypes.byref(dims.c()), _ptr(root_tok), _ptr(top_ids), _ptr(top_logp), _ptr(child_ids),
+        _ptr(child_logp), _ptr(node_tok), _ptr(node_parent), _ptr(node_depth), _ptr(node_score),
+        _ptr(dev_status), _stream(stream)))
+
+
+def tf_tree_mask(dims: Dims, node_parent, node_depth, root_pos, mask, pos_ids, stream=None):
+    _check("tf_tree_mask", load_library().tf_tree_mask(
+        ctypes.byref(dims.c()), _ptr(node_parent), _ptr(node_depth), _ptr(root_pos), _ptr(mask),
+        _ptr(pos_ids), _stream(stream)))
+
+
+def tf_draft_tree_host(dims: Dims, w: dict, hidden, root_tok, root_pos, node_tok, node_parent, node_depth,
+                       node_score, mask, pos_ids, dev_status, ws, stream=None):
+    """Host tensors in and out (pinned memory recommended); weights and workspace on the device."""
+    st = load_library().tf_draft_tree_host(
+        ctypes.byref(dims.c()), ctypes.byref(weights_struct(w)), _ptr(hidden), _ptr(root_tok),
+        _ptr(root_pos), _ptr(node_tok), _ptr(node_parent), _ptr(node_depth), _ptr(node_score), _ptr(mask),
+        _ptr(pos_ids), _ptr(dev_status), _ptr(ws), ws.numel(), _stream(stream))
+    if st not in (TF_OK, TF_ERR_DEVICE_STATUS):
+        _check("tf_draft_tree_host", st)
+    return st
+
+
+def tf_lmhead_partials(dims: Dims, lm_head, x, n_rows: int, ws, stream=None):
+    _check("tf_lmhead_partials", load_library().tf_lmhead_partials(
+        ctypes.byref(dims.c()), _ptr(lm_head), _ptr(x), n_rows, _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def tf_lmhead_merge(dims: Dims, lm_head, x, n_rows: int, k: int, out_ids, out_logp, ws, stream=None):
+    _check("tf_lmhead_merge", load_library().tf_lmhead_merge(
+        ctypes.byref(dims.c()), _ptr(lm_head), _ptr(x), n_rows, k, _ptr(out_ids), _ptr(out_logp), _ptr(ws),
+        ws.numel(), _stream(stream)))
+
+
+def tf_ar_approx(dims: Dims, w: dict, hidden, root_tok, top_ids, h_prime, ws, stream=None):
+    _check("tf_ar_approx", load_library().tf_ar_approx(
+        ctypes.byref(dims.c()), ctypes.byref(weights_struct(w)), _ptr(hidden), _ptr(root_tok), _ptr(top_ids),
+        _ptr(h_prime), _ptr(ws), ws.numel(), _stream(stream)))

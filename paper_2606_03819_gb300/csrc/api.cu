@@ -1,0 +1,381 @@
+// C ABI of the TreeFlash drafting path (declared in include/treeflash.h): argument checks,
+// workspace layout and the kernel sequence of every call. No allocation, no global state
+// besides the cached driver entry point used to build TMA descriptors.
+#include <math.h>
+#include <string.h>
+
+#include <algorithm>
+
+#include "common.cuh"
+
+namespace tf {
+size_t merge_smem_bytes(int n_tiles);
+}
+
+namespace {
+
+using namespace tf;
+
+constexpr size_t kAlign = 256;
+constexpr size_t kMaxMergeSmem = 220 * 1024;
+
+size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+struct Dims {
+    int b, d, V, I, gamma, M, K2, B, K1, R, dtype, mode, n_tiles;
+    size_t esize;
+    float inv_temp, eps;
+};
+
+struct Layout {
+    size_t status, partials, X, A, hp;
+    size_t h_hidden, h_root, h_pos, top_ids, top_logp, child_ids, child_logp;
+    size_t n_tok, n_par, n_dep, n_score, n_mask, n_pos, n_stat;
+    size_t total;
+};
+
+tf_status check_dims(const tf_dims* dims, Dims* o) {
+    if (!dims) return TF_ERR_INVALID_ARG;
+    const tf_dims& d = *dims;
+    if (d.batch < 1 || d.d < 1 || d.V < 1 || d.gamma < 1 || d.M < 1 || d.K2 < 1 || d.B < 1)
+        return TF_ERR_INVALID_ARG;
+    if (d.dtype != TF_BF16 && d.dtype != TF_F32) return TF_ERR_INVALID_ARG;
+    if (d.mode != TF_MODE_AR && d.mode != TF_MODE_MARGINAL && d.mode != TF_MODE_MARGINAL_MARY)
+        return TF_ERR_INVALID_ARG;
+    if (!(d.temperature > 0.0f) || !isfinite(d.temperature)) return TF_ERR_INVALID_ARG;
+    if (!(d.rms_eps >= 0.0f) || !isfinite(d.rms_eps)) return TF_ERR_INVALID_ARG;
+    const int K1 = d.M > d.K2 ? d.M : d.K2;
+    if (K1 > d.V) return TF_ERR_INVALID_ARG;
+    if (d.mode == TF_MODE_AR && d.I < 1) return TF_ERR_INVALID_ARG;
+    if (d.gamma > kMaxGamma || d.M > kMaxM || d.K2 > kMaxK || d.B > kMaxB) return TF_ERR_UNSUPPORTED;
+    if (d.dtype == TF_BF16 && (d.d % 64 != 0 || (d.mode == TF_MODE_AR && d.I % 64 != 0)))
+        return TF_ERR_UNSUPPORTED;
+    const int n_tiles = (d.V + kBlockV - 1) / kBlockV;
+    if (merge_smem_bytes(n_tiles) > kMaxMergeSmem) return TF_ERR_UNSUPPORTED;
+    const long long R = 1 + static_cast<long long>(d.M) * (d.gamma - 1);
+    if (static_cast<long long>(d.batch) * R > (1ll << 30) || static_cast<long long>(d.batch) * d.gamma > (1ll << 30))
+        return TF_ERR_UNSUPPORTED;
+    o->b = d.batch;
+    o->d = d.d;
+    o->V = d.V;
+    o->I = d.mode == TF_MODE_AR ? d.I : 0;
+    o->gamma = d.gamma;
+    o->M = d.M;
+    o->K2 = d.K2;
+    o->B = d.B;
+    o->K1 = K1;
+    o->R = static_cast<int>(R);
+    o->dtype = d.dtype;
+    o->mode = d.mode;
+    o->n_tiles = n_tiles;
+    o->esize = d.dtype == TF_BF16 ? 2 : 4;
+    o->inv_temp = 1.0f / d.temperature;
+    o->eps = d.rms_eps;
+    return TF_OK;
+}
+
+Layout layout(const Dims& D) {
+    Layout L{};
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = off;
+        off += up(bytes);
+        return at;
+    };
+    const size_t rows1 = static_cast<size_t>(D.b) * D.gamma;
+    const size_t rows2 = D.mode == TF_MODE_AR ? static_cast<size_t>(D.b) * D.R : 0;
+    const size_t rows = rows1 > rows2 ? rows1 : rows2;
+    const size_t nn = static_cast<size_t>(D.b) * (D.B + 1);
+    L.status = take(sizeof(int32_t));
+    L.partials = take(rows * D.n_tiles * sizeof(Partial));
+    L.X = take(rows2 * 2 * D.d * D.esize);
+    L.A = take(rows2 * D.I * D.esize);
+    L.hp = take(rows2 * D.d * D.esize);
+    L.h_hidden = take(rows1 * D.d * D.esize);
+    L.h_root = take(D.b * sizeof(int32_t));
+    L.h_pos = take(D.b * sizeof(int32_t));
+    L.top_ids = take(rows1 * D.K1 * sizeof(int32_t));
+    L.top_logp = take(rows1 * D.K1 * sizeof(float));
+    L.child_ids = take(rows2 * D.K2 * sizeof(int32_t));
+    L.child_logp = take(rows2 * D.K2 * sizeof(float));
+    L.n_tok = take(nn * sizeof(int32_t));
+    L.n_par = take(nn * sizeof(int32_t));
+    L.n_dep = take(nn * sizeof(int32_t));
+    L.n_score = take(nn * sizeof(float));
+    L.n_mask = take(static_cast<size_t>(D.b) * (D.B + 1) * (D.B + 1));
+    L.n_pos = take(nn * sizeof(int32_t));
+    L.n_stat = take(D.b * sizeof(int32_t));
+    L.total = off;
+    return L;
+}
+
+tf_status check_ws(const Layout& L, const void* ws, size_t ws_bytes) {
+    if (!ws) return TF_ERR_WORKSPACE;
+    if (reinterpret_cast<uintptr_t>(ws) % kAlign != 0) return TF_ERR_WORKSPACE;
+    if (ws_bytes < L.total) return TF_ERR_WORKSPACE;
+    return TF_OK;
+}
+
+bool aligned16(const void* p) { return p && reinterpret_cast<uintptr_t>(p) % 16 == 0; }
+
+template <typename P>
+P* at(void* ws, size_t off) {
+    return reinterpret_cast<P*>(static_cast<uint8_t*>(ws) + off);
+}
+
+tf_status make_ctx(void* ws, const Layout& L, tf_stream_t stream, Ctx* ctx) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return TF_ERR_CUDA;
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+        return TF_ERR_CUDA;
+    ctx->stream = reinterpret_cast<cudaStream_t>(stream);
+    ctx->num_sms = sms;
+    ctx->status = at<int>(ws, L.status);
+    return TF_OK;
+}
+
+tf_status cuda_status(cudaError_t e) { return e == cudaSuccess ? TF_OK : TF_ERR_CUDA; }
+
+#define TF_TRY(expr)                    \
+    do {                                \
+        const tf_status _s = (expr);    \
+        if (_s != TF_OK) return _s;     \
+    } while (0)
+
+// ---- the pieces -----------------------------------------------------------------------------
+tf_status do_partials(const Ctx& ctx, const Dims& D, const Layout& L, void* ws, const void* lm_head, const void* x,
+                      int n_rows) {
+    Partial* partials = at<Partial>(ws, L.partials);
+    if (D.dtype == TF_BF16)
+        return cuda_status(launch_lmhead_tc(ctx, lm_head, x, n_rows, D.d, D.V, D.inv_temp, partials));
+    return cuda_status(launch_lmhead_simt(ctx, D.dtype, lm_head, x, n_rows, D.d, D.V, D.inv_temp, partials));
+}
+
+tf_status do_merge(const Ctx& ctx, const Dims& D, const Layout& L, void* ws, const void* lm_head, const void* x,
+                   int n_rows, int k, int32_t* ids, float* logp) {
+    return cuda_status(launch_lmhead_merge(ctx, D.dtype, at<Partial>(ws, L.partials), n_rows, D.V, D.d, k,
+                                           D.inv_temp, lm_head, x, ids, logp));
+}
+
+tf_status do_ar_approx(const Ctx& ctx, const Dims& D, const Layout& L, void* ws, const tf_weights* w,
+                       const void* hidden, const int32_t* root_tok, const int32_t* top_ids) {
+    void* X = at<void>(ws, L.X);
+    void* A = at<void>(ws, L.A);
+    void* hp = at<void>(ws, L.hp);
+    TF_TRY(cuda_status(launch_gather_norm(ctx, D.dtype, hidden, w->embed, w->norm_h, w->norm_e, root_tok, top_ids,
+                                          D.b, D.gamma, D.M, D.K1, D.d, D.V, D.eps, X)));
+    const int rows = D.b * D.R;
+    if (D.dtype == TF_BF16)
+        return cuda_status(launch_swiglu_tc(ctx, X, w->w_gate, w->w_up, w->w_down, hidden, rows, D.d, D.I, D.R, D.M,
+                                            D.gamma, A, hp));
+    return cuda_status(launch_swiglu_simt(ctx, X, w->w_gate, w->w_up, w->w_down, hidden, rows, D.d, D.I, D.R, D.M,
+                                          D.gamma, A, hp));
+}
+
+tf_status check_weights(const Dims& D, const tf_weights* w, bool need_mlp) {
+    if (!w || !aligned16(w->lm_head)) return TF_ERR_INVALID_ARG;
+    if (need_mlp && (!aligned16(w->embed) || !aligned16(w->norm_h) || !aligned16(w->norm_e) ||
+                     !aligned16(w->w_gate) || !aligned16(w->w_up) || !aligned16(w->w_down)))
+        return TF_ERR_INVALID_ARG;
+    (void)D;
+    return TF_OK;
+}
+
+struct Prepared {
+    Dims D;
+    Layout L;
+    Ctx ctx;
+};
+
+tf_status prepare(const tf_dims* dims, void* ws, size_t ws_bytes, tf_stream_t stream, Prepared* p) {
+    TF_TRY(check_dims(dims, &p->D));
+    p->L = layout(p->D);
+    TF_TRY(check_ws(p->L, ws, ws_bytes));
+    return make_ctx(ws, p->L, stream, &p->ctx);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* tf_status_string(tf_status s) {
+    switch (s) {
+        case TF_OK: return "ok";
+        case TF_ERR_INVALID_ARG: return "invalid argument";
+        case TF_ERR_UNSUPPORTED: return "unsupported dimensions";
+        case TF_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+        case TF_ERR_CUDA: return "CUDA error";
+        case TF_ERR_DEVICE_STATUS: return "device reported a condition (TF_DEV_* flags)";
+        case TF_ERR_TIMEOUT: return "a bounded device wait gave up";
+    }
+    return "unknown status";
+}
+
+int32_t tf_version(void) { return 100; }
+
+tf_status tf_workspace_size(const tf_dims* dims, size_t* bytes) {
+    if (!bytes) return TF_ERR_INVALID_ARG;
+    Dims D;
+    TF_TRY(check_dims(dims, &D));
+    *bytes = layout(D).total;
+    return TF_OK;
+}
+
+tf_status tf_status_reset(void* ws, size_t ws_bytes, tf_stream_t stream) {
+    if (!ws || ws_bytes < sizeof(int32_t) || reinterpret_cast<uintptr_t>(ws) % kAlign) return TF_ERR_WORKSPACE;
+    return cuda_status(cudaMemsetAsync(ws, 0, sizeof(int32_t), reinterpret_cast<cudaStream_t>(stream)));
+}
+
+tf_status tf_status_read(const void* ws, size_t ws_bytes, int32_t* flags, tf_stream_t stream) {
+    if (!flags) return TF_ERR_INVALID_ARG;
+    if (!ws || ws_bytes < sizeof(int32_t) || reinterpret_cast<uintptr_t>(ws) % kAlign) return TF_ERR_WORKSPACE;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int32_t v = 0;
+    if (cudaMemcpyAsync(&v, ws, sizeof(int32_t), cudaMemcpyDeviceToHost, st) != cudaSuccess) return TF_ERR_CUDA;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return TF_ERR_CUDA;
+    *flags = v;
+    if (v & TF_DEV_TIMEOUT) return TF_ERR_TIMEOUT;
+    if (v & ~TF_DEV_RECOMPUTED) return TF_ERR_DEVICE_STATUS;
+    return TF_OK;
+}
+
+tf_status tf_lmhead_partials(const tf_dims* dims, const void* lm_head, const void* x, int32_t n_rows, void* ws,
+                             size_t ws_bytes, tf_stream_t stream) {
+    Prepared p;
+    TF_TRY(prepare(dims, ws, ws_bytes, stream, &p));
+    const long long max_rows = std::max(static_cast<long long>(p.D.b) * p.D.gamma,
+                                        p.D.mode == TF_MODE_AR ? static_cast<long long>(p.D.b) * p.D.R : 0ll);
+    if (!aligned16(lm_head) || !aligned16(x) || n_rows < 0 || n_rows > max_rows) return TF_ERR_INVALID_ARG;
+    return do_partials(p.ctx, p.D, p.L, ws, lm_head, x, n_rows);
+}
+
+tf_status tf_lmhead_merge(const tf_dims* dims, const void* lm_head, const void* x, int32_t n_rows, int32_t k,
+                          int32_t* out_ids, float* out_logp, void* ws, size_t ws_bytes, tf_stream_t stream) {
+    Prepared p;
+    TF_TRY(prepare(dims, ws, ws_bytes, stream, &p));
+    const long long max_rows = std::max(static_cast<long long>(p.D.b) * p.D.gamma,
+                                        p.D.mode == TF_MODE_AR ? static_cast<long long>(p.D.b) * p.D.R : 0ll);
+    if (!lm_head || !x || !out_ids || !out_logp || n_rows < 0 || n_rows > max_rows) return TF_ERR_INVALID_ARG;
+    if (k < 1 || k > kMaxK || k > p.D.V) return TF_ERR_INVALID_ARG;
+    return do_merge(p.ctx, p.D, p.L, ws, lm_head, x, n_rows, k, out_ids, out_logp);
+}
+
+tf_status tf_stage1_marginals(const tf_dims* dims, const tf_weights* w, const void* hidden, int32_t* top_ids,
+                              float* top_logp, void* ws, size_t ws_bytes, tf_stream_t stream) {
+    Prepared p;
+    TF_TRY(prepare(dims, ws, ws_bytes, stream, &p));
+    TF_TRY(check_weights(p.D, w, false));
+    if (!aligned16(hidden) || !top_ids || !top_logp) return TF_ERR_INVALID_ARG;
+    TF_TRY(cuda_status(cudaMemsetAsync(p.ctx.status, 0, sizeof(int32_t), p.ctx.stream)));
+    const int rows = p.D.b * p.D.gamma;
+    TF_TRY(do_partials(p.ctx, p.D, p.L, ws, w->lm_head, hidden, rows));
+    return do_merge(p.ctx, p.D, p.L, ws, w->lm_head, hidden, rows, p.D.K1, top_ids, top_logp);
+}
+
+tf_status tf_ar_approx(const tf_dims* dims, const tf_weights* w, const void* hidden, const int32_t* root_tok,
+                       const int32_t* top_ids, void* h_prime, void* ws, size_t ws_bytes, tf_stream_t stream) {
+    Prepared p;
+    TF_TRY(prepare(dims, ws, ws_bytes, stream, &p));
+    if (p.D.mode != TF_MODE_AR) return TF_ERR_INVALID_ARG;
+    TF_TRY(check_weights(p.D, w, true));
+    if (!aligned16(hidden) || !root_tok || !top_ids) return TF_ERR_INVALID_ARG;
+    TF_TRY(do_ar_approx(p.ctx, p.D, p.L, ws, w, hidden, root_tok, top_ids));
+    if (h_prime) {
+        const size_t bytes = static_cast<size_t>(p.D.b) * p.D.R * p.D.d * p.D.esize;
+        TF_TRY(cuda_status(cudaMemcpyAsync(h_prime, at<void>(ws, p.L.hp), bytes, cudaMemcpyDeviceToDevice,
+                                           p.ctx.stream)));
+    }
+    return TF_OK;
+}
+
+tf_status tf_stage2_ar_approx(const tf_dims* dims, const tf_weights* w, const void* hidden, const int32_t* root_tok,
+                              const int32_t* top_ids, int32_t* child_ids, float* child_logp, void* ws,
+                              size_t ws_bytes, tf_stream_t stream) {
+    Prepared p;
+    TF_TRY(prepare(dims, ws, ws_bytes, stream, &p));
+    if (p.D.mode != TF_MODE_AR) return TF_ERR_INVALID_ARG;
+    TF_TRY(check_weights(p.D, w, true));
+    if (!aligned16(hidden) || !root_tok || !top_ids || !child_ids || !child_logp) return TF_ERR_INVALID_ARG;
+    TF_TRY(do_ar_approx(p.ctx, p.D, p.L, ws, w, hidden, root_tok, top_ids));
+    const int rows = p.D.b * p.D.R;
+    const void* hp = at<void>(ws, p.L.hp);
+    TF_TRY(do_partials(p.ctx, p.D, p.L, ws, w->lm_head, hp, rows));
+    return do_merge(p.ctx, p.D, p.L, ws, w->lm_head, hp, rows, p.D.K2, child_ids, child_logp);
+}
+
+tf_status tf_build_tree(const tf_dims* dims, const int32_t* root_tok, const int32_t* top_ids, const float* top_logp,
+                        const int32_t* child_ids, const float* child_logp, int32_t* node_tok, int32_t* node_parent,
+                        int32_t* node_depth, float* node_score, int32_t* dev_status, tf_stream_t stream) {
+    Dims D;
+    TF_TRY(check_dims(dims, &D));
+    if (!root_tok || !top_ids || !top_logp || !node_tok || !node_parent || !node_depth || !node_score || !dev_status)
+        return TF_ERR_INVALID_ARG;
+    if (D.mode == TF_MODE_AR && (!child_ids || !child_logp)) return TF_ERR_INVALID_ARG;
+    Ctx ctx{reinterpret_cast<cudaStream_t>(stream), 0, nullptr};
+    return cuda_status(launch_build_tree(ctx, D.b, D.gamma, D.M, D.K1, D.K2, D.B, D.V, D.mode, D.R, root_tok,
+                                         top_ids, top_logp, child_ids, child_logp, node_tok, node_parent,
+                                         node_depth, node_score, dev_status));
+}
+
+tf_status tf_tree_mask(const tf_dims* dims, const int32_t* node_parent, const int32_t* node_depth,
+                       const int32_t* root_pos, uint8_t* mask, int32_t* pos_ids, tf_stream_t stream) {
+    Dims D;
+    TF_TRY(check_dims(dims, &D));
+    if (!node_parent || !node_depth || !root_pos || !mask || !pos_ids) return TF_ERR_INVALID_ARG;
+    Ctx ctx{reinterpret_cast<cudaStream_t>(stream), 0, nullptr};
+    return cuda_status(launch_tree_mask(ctx, D.b, D.B, node_parent, node_depth, root_pos, mask, pos_ids));
+}
+
+tf_status tf_draft_tree_host(const tf_dims* dims, const tf_weights* w, const void* hidden, const int32_t* root_tok,
+                             const int32_t* root_pos, int32_t* node_tok, int32_t* node_parent, int32_t* node_depth,
+                             float* node_score, uint8_t* mask, int32_t* pos_ids, int32_t* dev_status, void* ws,
+                             size_t ws_bytes, tf_stream_t stream) {
+    Prepared p;
+    TF_TRY(prepare(dims, ws, ws_bytes, stream, &p));
+    if (!hidden || !root_tok || !root_pos || !node_tok || !node_parent || !node_depth || !node_score || !mask ||
+        !pos_ids || !dev_status)
+        return TF_ERR_INVALID_ARG;
+    const Dims& D = p.D;
+    const Layout& L = p.L;
+    cudaStream_t st = p.ctx.stream;
+    const size_t nn = static_cast<size_t>(D.b) * (D.B + 1);
+    void* d_hidden = at<void>(ws, L.h_hidden);
+    int32_t* d_root = at<int32_t>(ws, L.h_root);
+    int32_t* d_pos = at<int32_t>(ws, L.h_pos);
+    TF_TRY(cuda_status(cudaMemcpyAsync(d_hidden, hidden, static_cast<size_t>(D.b) * D.gamma * D.d * D.esize,
+                                       cudaMemcpyHostToDevice, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(d_root, root_tok, D.b * sizeof(int32_t), cudaMemcpyHostToDevice, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(d_pos, root_pos, D.b * sizeof(int32_t), cudaMemcpyHostToDevice, st)));
+    int32_t* top_ids = at<int32_t>(ws, L.top_ids);
+    float* top_logp = at<float>(ws, L.top_logp);
+    int32_t* child_ids = at<int32_t>(ws, L.child_ids);
+    float* child_logp = at<float>(ws, L.child_logp);
+    TF_TRY(tf_stage1_marginals(dims, w, d_hidden, top_ids, top_logp, ws, ws_bytes, stream));
+    if (D.mode == TF_MODE_AR)
+        TF_TRY(tf_stage2_ar_approx(dims, w, d_hidden, d_root, top_ids, child_ids, child_logp, ws, ws_bytes, stream));
+    int32_t* d_tok = at<int32_t>(ws, L.n_tok);
+    int32_t* d_par = at<int32_t>(ws, L.n_par);
+    int32_t* d_dep = at<int32_t>(ws, L.n_dep);
+    float* d_score = at<float>(ws, L.n_score);
+    uint8_t* d_mask = at<uint8_t>(ws, L.n_mask);
+    int32_t* d_posid = at<int32_t>(ws, L.n_pos);
+    int32_t* d_stat = at<int32_t>(ws, L.n_stat);
+    TF_TRY(tf_build_tree(dims, d_root, top_ids, top_logp, D.mode == TF_MODE_AR ? child_ids : nullptr,
+                         D.mode == TF_MODE_AR ? child_logp : nullptr, d_tok, d_par, d_dep, d_score, d_stat, stream));
+    TF_TRY(tf_tree_mask(dims, d_par, d_dep, d_pos, d_mask, d_posid, stream));
+    TF_TRY(cuda_status(cudaMemcpyAsync(node_tok, d_tok, nn * 4, cudaMemcpyDeviceToHost, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(node_parent, d_par, nn * 4, cudaMemcpyDeviceToHost, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(node_depth, d_dep, nn * 4, cudaMemcpyDeviceToHost, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(node_score, d_score, nn * 4, cudaMemcpyDeviceToHost, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(mask, d_mask, nn * (D.B + 1), cudaMemcpyDeviceToHost, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(pos_ids, d_posid, nn * 4, cudaMemcpyDeviceToHost, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(dev_status, d_stat, D.b * 4, cudaMemcpyDeviceToHost, st)));
+    int32_t flags = 0;
+    const tf_status rs = tf_status_read(ws, ws_bytes, &flags, stream);  // synchronises the stream
+    if (rs == TF_ERR_CUDA) return rs;
+    for (int s = 0; s < D.b; ++s) dev_status[s] |= flags;
+    return rs;
+}
+
+}  // extern "C"

@@ -1,0 +1,112 @@
+// Shared definitions of the TreeFlash CUDA library (device side and launcher side).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "treeflash.h"
+
+namespace tf {
+
+// ---- sizes fixed by the kernels --------------------------------------------------------------
+constexpr int kBlockV = 256;        // vocabulary entries per LM-head block (one MMA N-tile)
+constexpr int kListLen = 8;         // (logit, id) pairs kept per (row, block) by the LM-head pass
+constexpr int kMaxK = 64;           // largest top-k a merge can return
+constexpr int kMaxM = 32;           // largest M (the builder tests membership with one warp)
+constexpr int kMaxB = 1023;         // largest draft budget
+constexpr int kMaxGamma = 64;
+constexpr int kMergeExpandLists = 8;  // lists a merge may recompute exactly (>= (kMaxK-1)/8 + 1)
+
+// Per (row, vocabulary block) summary written by the LM-head pass: the block's max logit m,
+// sum_v exp(z_v - m), and its kListLen largest logits in (value desc, id asc) order; unused
+// slots have id -1 and value -inf.
+struct __align__(8) Partial {
+    float m;
+    float s;
+    float v[kListLen];
+    int id[kListLen];
+};
+static_assert(sizeof(Partial) == 72, "Partial layout");
+
+// ---- bf16 / f32 element access ----------------------------------------------------------------
+__device__ __forceinline__ float to_f32(float x) { return x; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 x) { return __bfloat162float(x); }
+template <typename T> __device__ __forceinline__ T from_f32(float x);
+template <> __device__ __forceinline__ float from_f32<float>(float x) { return x; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float x) {
+    return __float2bfloat16_rn(x);
+}
+
+// Order-preserving map of a float to uint32 (larger float -> larger key; -0 < +0; NaN ends up
+// above +inf or below -inf depending on its sign bit, it never appears in practice).
+__device__ __forceinline__ uint32_t float_key(float f) {
+    uint32_t u = __float_as_uint(f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float key_float(uint32_t k) {
+    uint32_t u = (k & 0x80000000u) ? (k & 0x7fffffffu) : ~k;
+    return __uint_as_float(u);
+}
+// 64-bit candidate key: larger value first, then smaller token id.
+__device__ __forceinline__ unsigned long long cand_key(float v, int id) {
+    return ((unsigned long long)float_key(v) << 32) | (unsigned long long)(0xffffffffu - (uint32_t)id);
+}
+__device__ __forceinline__ int key_id(unsigned long long k) {
+    return (int)(0xffffffffu - (uint32_t)(k & 0xffffffffull));
+}
+__device__ __forceinline__ float key_value(unsigned long long k) { return key_float((uint32_t)(k >> 32)); }
+
+__device__ __forceinline__ void set_status(int* status, int bits) {
+    if (status) atomicOr(status, bits);
+}
+
+// Stage-2 row -> (index of the hidden state it refines within its sequence, previous-token
+// source). Row 0 of a sequence refines h_{t+1} with the root token; row 1 + (i-2) M + m
+// refines h_{t+i} with stage-1 candidate m of depth i-1 (Algorithm 1 Part 1, 1 + M(gamma-1)
+// rows per sequence).
+__host__ __device__ __forceinline__ int stage2_hidden_index(int r, int M) {
+    return r == 0 ? 0 : (r - 1) / M + 1;
+}
+
+}  // namespace tf
+
+// ---- launchers (one per kernel family); implemented in the .cu files -------------------------
+namespace tf {
+
+struct Ctx {
+    cudaStream_t stream;
+    int num_sms;
+    int* status;  // device status word in the workspace
+};
+
+// LM-head pass (tensor-core path for bf16, CUDA-core path for f32)
+cudaError_t launch_lmhead_tc(const Ctx&, const void* lm_head, const void* x, int n_rows, int d,
+                             int V, float inv_temp, Partial* partials);
+cudaError_t launch_lmhead_simt(const Ctx&, int dtype, const void* lm_head, const void* x,
+                               int n_rows, int d, int V, float inv_temp, Partial* partials);
+cudaError_t launch_lmhead_merge(const Ctx&, int dtype, const Partial* partials, int n_rows, int V,
+                                int d, int k, float inv_temp, const void* lm_head, const void* x,
+                                int32_t* out_ids, float* out_logp);
+// Eq. 1 pieces
+cudaError_t launch_gather_norm(const Ctx&, int dtype, const void* hidden, const void* embed,
+                               const void* norm_h, const void* norm_e, const int32_t* root_tok,
+                               const int32_t* top_ids, int b, int gamma, int M, int K1, int d,
+                               int V, float eps, void* X);
+cudaError_t launch_swiglu_tc(const Ctx&, const void* X, const void* w_gate, const void* w_up,
+                             const void* w_down, const void* hidden, int n_rows, int d, int I,
+                             int R, int M, int gamma, void* A, void* h_prime);
+cudaError_t launch_swiglu_simt(const Ctx&, const void* X, const void* w_gate, const void* w_up,
+                               const void* w_down, const void* hidden, int n_rows, int d, int I,
+                               int R, int M, int gamma, void* A, void* h_prime);
+// Part 2 and the mask
+cudaError_t launch_build_tree(const Ctx&, int b, int gamma, int M, int K1, int K2, int B, int V,
+                              int mode, int R, const int32_t* root_tok, const int32_t* top_ids,
+                              const float* top_logp, const int32_t* child_ids,
+                              const float* child_logp, int32_t* node_tok, int32_t* node_parent,
+                              int32_t* node_depth, float* node_score, int32_t* dev_status);
+cudaError_t launch_tree_mask(const Ctx&, int b, int B, const int32_t* node_parent,
+                             const int32_t* node_depth, const int32_t* root_pos, uint8_t* mask,
+                             int32_t* pos_ids);
+
+}  // namespace tf

@@ -1,0 +1,222 @@
+// CUDA-core (fp32 FMA) kernels of the TF_F32 path: the same LM-head pass and SwiGLU of Eq. 1
+// as the tensor-core path, for fp32 inputs whose 1e-4 accuracy target rules out TF32 / bf16
+// tensor-core arithmetic. Same partial format, same merge.
+#include <math.h>
+
+#include "common.cuh"
+
+namespace tf {
+namespace {
+
+constexpr int kRowsPerCta = 32;
+constexpr int kKChunk = 32;
+
+// One CTA: rows [r0, r0 + 32) x vocabulary block [v0, v0 + 256). Thread t owns vocabulary column
+// v0 + t and accumulates its 32 logits; the block is then staged in shared memory and one warp
+// per row computes the block max, sum of exp and top-8 with warp shuffles.
+__global__ void __launch_bounds__(256) lmhead_simt_kernel(const float* __restrict__ W, const float* __restrict__ X,
+                                                          int n_rows, int d, int V, float inv_temp,
+                                                          Partial* __restrict__ partials, int n_tiles) {
+    __shared__ float xs[kRowsPerCta][kKChunk + 1];
+    __shared__ float ws[kBlockV][kKChunk + 1];
+    const int vt = blockIdx.x;
+    const int r0 = blockIdx.y * kRowsPerCta;
+    const int t = threadIdx.x;
+    float acc[kRowsPerCta];
+#pragma unroll
+    for (int r = 0; r < kRowsPerCta; ++r) acc[r] = 0.0f;
+
+    for (int k0 = 0; k0 < d; k0 += kKChunk) {
+        for (int i = t; i < kRowsPerCta * kKChunk; i += 256) {
+            const int r = i / kKChunk, k = i % kKChunk;
+            xs[r][k] = (r0 + r < n_rows && k0 + k < d) ? X[static_cast<size_t>(r0 + r) * d + k0 + k] : 0.0f;
+        }
+        for (int i = t; i < kBlockV * kKChunk; i += 256) {
+            const int v = i / kKChunk, k = i % kKChunk;
+            const int gv = vt * kBlockV + v;
+            ws[v][k] = (gv < V && k0 + k < d) ? W[static_cast<size_t>(gv) * d + k0 + k] : 0.0f;
+        }
+        __syncthreads();
+#pragma unroll 4
+        for (int k = 0; k < kKChunk; ++k) {
+            const float w = ws[t][k];
+#pragma unroll
+            for (int r = 0; r < kRowsPerCta; ++r) acc[r] = fmaf(xs[r][k], w, acc[r]);
+        }
+        __syncthreads();
+    }
+    // stage the logits of the block: zt[r][t]
+    float* zt = &ws[0][0];
+    const bool valid = vt * kBlockV + t < V;
+#pragma unroll
+    for (int r = 0; r < kRowsPerCta; ++r) zt[r * kBlockV + t] = valid ? acc[r] * inv_temp : -INFINITY;
+    __syncthreads();
+
+    const int warp = t >> 5, lane = t & 31;
+    for (int r = warp; r < kRowsPerCta; r += 8) {
+        if (r0 + r >= n_rows) break;
+        float z[8];
+        float m = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            z[j] = zt[r * kBlockV + lane + 32 * j];
+            m = fmaxf(m, z[j]);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+        float s = 0.0f;
+        if (m > -INFINITY) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) s += expf(z[j] - m);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        // top-8: eight rounds of a warp-wide (value desc, id asc) arg-max
+        float tv[kListLen];
+        int ti[kListLen];
+        for (int k = 0; k < kListLen; ++k) {
+            float bv = -INFINITY;
+            int bid = 0x7fffffff;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int id = vt * kBlockV + lane + 32 * j;
+                if (z[j] > bv || (z[j] == bv && z[j] > -INFINITY && id < bid)) {
+                    bv = z[j];
+                    bid = id;
+                }
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+                const int oid = __shfl_xor_sync(0xffffffffu, bid, o);
+                if (ov > bv || (ov == bv && oid < bid)) {
+                    bv = ov;
+                    bid = oid;
+                }
+            }
+            if (bv == -INFINITY) {
+                tv[k] = -INFINITY;
+                ti[k] = -1;
+                continue;
+            }
+            tv[k] = bv;
+            ti[k] = bid;
+            const int owner = (bid - vt * kBlockV) & 31;
+            const int slot = (bid - vt * kBlockV) >> 5;
+            if (lane == owner) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j)
+                    if (j == slot) z[j] = -INFINITY;
+            }
+        }
+        if (lane == 0) {
+            Partial* p = partials + static_cast<size_t>(r0 + r) * n_tiles + vt;
+            p->m = m;
+            p->s = s;
+#pragma unroll
+            for (int j = 0; j < kListLen; ++j) {
+                p->v[j] = tv[j];
+                p->id[j] = ti[j];
+            }
+        }
+    }
+}
+
+// C[n_rows, N] = X[n_rows, K] W[N, K]^T on 64 x 64 tiles (16 x 16 threads, 4 x 4 outputs each).
+// GATEUP: out = SiLU(X Wg^T) * (X Wu^T); DOWN: out = hidden[stage-2 row's depth] + X Wd^T.
+template <bool GATEUP>
+__global__ void __launch_bounds__(256) swiglu_simt_kernel(const float* __restrict__ X, const float* __restrict__ W0,
+                                                          const float* __restrict__ W1, int n_rows, int K, int N,
+                                                          float* __restrict__ out, const float* __restrict__ hidden,
+                                                          int R, int M, int gamma) {
+    constexpr int T = 64, KC = 16;
+    __shared__ float xs[KC][T + 4];
+    __shared__ float w0s[KC][T + 4];
+    __shared__ float w1s[GATEUP ? KC : 1][T + 4];
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const int row0 = blockIdx.y * T, col0 = blockIdx.x * T;
+    float a0[4][4] = {}, a1[4][4] = {};
+    for (int k0 = 0; k0 < K; k0 += KC) {
+        for (int i = threadIdx.x; i < T * KC; i += 256) {
+            const int r = i / KC, k = i % KC;
+            const bool kin = k0 + k < K;
+            xs[k][r] = (row0 + r < n_rows && kin) ? X[static_cast<size_t>(row0 + r) * K + k0 + k] : 0.0f;
+            w0s[k][r] = (col0 + r < N && kin) ? W0[static_cast<size_t>(col0 + r) * K + k0 + k] : 0.0f;
+            if (GATEUP) w1s[k][r] = (col0 + r < N && kin) ? W1[static_cast<size_t>(col0 + r) * K + k0 + k] : 0.0f;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int k = 0; k < KC; ++k) {
+            float xv[4], wv0[4], wv1[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                xv[i] = xs[k][ty * 4 + i];
+                wv0[i] = w0s[k][tx * 4 + i];
+                if (GATEUP) wv1[i] = w1s[k][tx * 4 + i];
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    a0[i][j] = fmaf(xv[i], wv0[j], a0[i][j]);
+                    if (GATEUP) a1[i][j] = fmaf(xv[i], wv1[j], a1[i][j]);
+                }
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int r = row0 + ty * 4 + i;
+        if (r >= n_rows) continue;
+        int hid = 0;
+        if (!GATEUP) {
+            const int sq = r / R, rr = r - sq * R;
+            hid = sq * gamma + stage2_hidden_index(rr, M);
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int c = col0 + tx * 4 + j;
+            if (c >= N) continue;
+            float v;
+            if (GATEUP) {
+                const float g = a0[i][j];
+                v = g / (1.0f + expf(-g)) * a1[i][j];
+            } else {
+                v = hidden[static_cast<size_t>(hid) * N + c] + a0[i][j];
+            }
+            out[static_cast<size_t>(r) * N + c] = v;
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_lmhead_simt(const Ctx& ctx, int dtype, const void* lm_head, const void* x, int n_rows, int d,
+                               int V, float inv_temp, Partial* partials) {
+    if (dtype != TF_F32) return cudaErrorNotSupported;
+    if (n_rows <= 0) return cudaSuccess;
+    const int n_tiles = (V + kBlockV - 1) / kBlockV;
+    dim3 grid(n_tiles, (n_rows + kRowsPerCta - 1) / kRowsPerCta);
+    lmhead_simt_kernel<<<grid, 256, 0, ctx.stream>>>(static_cast<const float*>(lm_head), static_cast<const float*>(x),
+                                                     n_rows, d, V, inv_temp, partials, n_tiles);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_swiglu_simt(const Ctx& ctx, const void* X, const void* w_gate, const void* w_up,
+                               const void* w_down, const void* hidden, int n_rows, int d, int I, int R, int M,
+                               int gamma, void* A, void* h_prime) {
+    if (n_rows <= 0) return cudaSuccess;
+    dim3 g1((I + 63) / 64, (n_rows + 63) / 64);
+    swiglu_simt_kernel<true><<<g1, 256, 0, ctx.stream>>>(
+        static_cast<const float*>(X), static_cast<const float*>(w_gate), static_cast<const float*>(w_up), n_rows,
+        2 * d, I, static_cast<float*>(A), nullptr, R, M, gamma);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    dim3 g2((d + 63) / 64, (n_rows + 63) / 64);
+    swiglu_simt_kernel<false><<<g2, 256, 0, ctx.stream>>>(
+        static_cast<const float*>(A), static_cast<const float*>(w_down), nullptr, n_rows, I, d,
+        static_cast<float*>(h_prime), static_cast<const float*>(hidden), R, M, gamma);
+    return cudaGetLastError();
+}
+
+}  // namespace tf

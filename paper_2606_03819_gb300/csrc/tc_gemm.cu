@@ -1,0 +1,461 @@
+// Tensor-core (tcgen05 + TMA) GEMM kernels of the bf16 path.
+//
+//   D[r, n] = sum_k X[r, k] * W[n, k]          X: activations [rows, K], W: weights [N, K]
+//
+// X rows sit in the 128 TMEM lanes (M = 128 per tile), weight rows in the MMA N dimension, so
+// every epilogue thread owns one activation row and walks its logits / outputs serially.
+// Three fused epilogues:
+//   LMHEAD  the LM-head pass of Algorithm 1 (stage 1 and stage 2): for each (row, block of 256
+//           vocabulary entries) it keeps the block max, the sum of exp(z - max) and the 8 largest
+//           (z, id). Logits never leave the SM.
+//   GATEUP  SwiGLU of Eq. 1, first half: A = SiLU(X W_gate^T) * (X W_up^T), bf16 out.
+//   DOWN    SwiGLU of Eq. 1, second half plus the residual: h' = h + A W_down^T, bf16 out.
+//
+// Warp roles (320 threads, one CTA per SM, persistent over work units):
+//   warp 0      TMA producer: one elected lane streams X and W tiles into a ring of stages.
+//   warp 1      TMEM allocator and MMA issuer (one lane issues tcgen05.mma and commits).
+//   warps 2..9  epilogue, two groups of four; group g drains accumulator slot g (TMEM columns
+//               [256 g, 256 g + 256)); warp w may only touch TMEM lanes 32 (w % 4) .. + 31.
+// A work unit is (N tile, group of MT M-tiles). With MT = 2 both slots hold one unit (M-tile j
+// in slot j); with MT = 1 consecutive units alternate slots so the epilogue of one overlaps the
+// MMAs of the next. Every wait is bounded: after a time limit the kernel raises TF_DEV_TIMEOUT,
+// drains its in-flight copies and MMAs, frees TMEM and returns.
+#include <cuda.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "tc_ptx.cuh"
+
+namespace tf {
+namespace {
+
+constexpr int kBK = 64;       // K elements per stage: one 128-byte swizzle row of bf16
+constexpr int kBM = 128;      // activation rows per M-tile (TMEM lanes)
+constexpr int kThreads = 320;
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
+enum { EPI_LMHEAD = 0, EPI_GATEUP = 1, EPI_DOWN = 2 };
+
+struct EpiParams {
+    Partial* partials;           // LMHEAD: [n_rows, n_tiles]
+    int V;
+    float inv_temp;
+    __nv_bfloat16* out;          // GATEUP: A [n_rows, ld_out]; DOWN: h' [n_rows, ld_out]
+    int ld_out;
+    const __nv_bfloat16* hidden; // DOWN: residual rows, [b * gamma, ld_out]
+    int R, M, gamma;
+};
+
+template <int MT, int NB, int BN, int STAGES>
+struct TileCfg {
+    static constexpr int kABytes = kBM * kBK * 2;
+    static constexpr int kBBytes = BN * kBK * 2;
+    static constexpr int kStageBytes = MT * kABytes + NB * kBBytes;
+    static constexpr int kBarrierBytes = 256;
+    static constexpr int kSmemBytes = STAGES * kStageBytes + kBarrierBytes + 1024;
+    static_assert(NB * BN <= 256, "one accumulator slot is 256 TMEM columns");
+    static_assert(BN % 32 == 0 && BN >= 32 && BN <= 256, "N tile");
+    static_assert(kStageBytes % 1024 == 0, "stages must stay 1024-byte aligned for 128B swizzle");
+};
+
+__device__ __forceinline__ float silu_f(float g) { return g / (1.0f + __expf(-g)); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+
+template <int EPI, int MT, int NB, int BN, int STAGES>
+__global__ void __launch_bounds__(kThreads, 1)
+tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_w0,
+               const __grid_constant__ CUtensorMap tmap_w1, int n_rows, int K, int n_ntiles,
+               int n_mgroups, int w_stream_once, EpiParams ep, int* status) {
+    using C = TileCfg<MT, NB, BN, STAGES>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * C::kStageBytes);
+    uint64_t* empty = full + STAGES;
+    uint64_t* tfull = empty + STAGES;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* drain = tempty + 2;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int n_units = n_ntiles * n_mgroups;
+    const int nk = K / kBK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            ptx::mbar_init(&full[s], 1);
+            ptx::mbar_init(&empty[s], 1);
+        }
+        for (int g = 0; g < 2; ++g) {
+            ptx::mbar_init(&tfull[g], 1);
+            ptx::mbar_init(&tempty[g], 128);
+        }
+        ptx::mbar_init(drain, 1);
+        *abort_flag = 0;
+        ptx::fence_barrier_init();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(tmem_slot, 512);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            ptx::prefetch_tmap(&tmap_x);
+            ptx::prefetch_tmap(&tmap_w0);
+            if (NB == 2) ptx::prefetch_tmap(&tmap_w1);
+            const uint64_t pol_x = ptx::policy_evict_last();
+            const uint64_t pol_w = w_stream_once ? ptx::policy_evict_first() : ptx::policy_evict_last();
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t issued_mask = 0;                 // stages that ever received a load
+            uint32_t last_parity[STAGES > 0 ? STAGES : 1];
+            bool ok = true;
+            for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+                const int nt = u / n_mgroups, mg = u % n_mgroups;
+                for (int kb = 0; kb < nk; ++kb) {
+                    if (!ptx::mbar_wait(&empty[stage], phase ^ 1u, abort_flag, kWaitLimitNs)) {
+                        ok = false;
+                        break;
+                    }
+                    ptx::mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
+                    uint8_t* sp = smem + stage * C::kStageBytes;
+#pragma unroll
+                    for (int j = 0; j < MT; ++j)
+                        ptx::tma_load_2d(sp + j * C::kABytes, &tmap_x, &full[stage], kb * kBK,
+                                         (mg * MT + j) * kBM, pol_x);
+                    ptx::tma_load_2d(sp + MT * C::kABytes, &tmap_w0, &full[stage], kb * kBK, nt * BN, pol_w);
+                    if (NB == 2)
+                        ptx::tma_load_2d(sp + MT * C::kABytes + C::kBBytes, &tmap_w1, &full[stage],
+                                         kb * kBK, nt * BN, pol_w);
+                    issued_mask |= 1u << stage;
+                    last_parity[stage] = phase;
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            if (!ok) {
+                *abort_flag = 1;
+                set_status(status, TF_DEV_TIMEOUT);
+            }
+            // No copy may still be writing this CTA's shared memory when it exits: wait for the
+            // last load of every stage (already complete unless another role gave up early).
+            for (int s = 0; s < STAGES; ++s)
+                if (issued_mask & (1u << s)) ptx::mbar_wait(&full[s], last_parity[s], nullptr, kWaitLimitNs);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kBM, BN);
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t use[2] = {0u, 0u};
+            bool ok = true;
+            int kl = 0;
+            for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++kl) {
+                const int g0 = (MT == 2) ? 0 : (kl & 1);
+                for (int j = 0; j < MT && ok; ++j)
+                    ok = ptx::mbar_wait(&tempty[g0 + j], (use[g0 + j] & 1u) ^ 1u, abort_flag, kWaitLimitNs);
+                if (!ok) break;
+                ptx::tc_fence_after();
+                for (int kb = 0; kb < nk; ++kb) {
+                    if (!ptx::mbar_wait(&full[stage], phase, abort_flag, kWaitLimitNs)) {
+                        ok = false;
+                        break;
+                    }
+                    ptx::tc_fence_after();
+                    const uint32_t a0 = ptx::smem_u32(smem + stage * C::kStageBytes);
+                    const uint32_t b0 = a0 + MT * C::kABytes;
+#pragma unroll
+                    for (int kk = 0; kk < kBK / 16; ++kk) {
+#pragma unroll
+                        for (int j = 0; j < MT; ++j) {
+                            const uint64_t ad = ptx::sw128_kmajor_desc(a0 + j * C::kABytes + kk * 32);
+#pragma unroll
+                            for (int nb = 0; nb < NB; ++nb) {
+                                const uint64_t bd = ptx::sw128_kmajor_desc(b0 + nb * C::kBBytes + kk * 32);
+                                ptx::mma_bf16(tmem_base + 256u * (g0 + j) + nb * BN, ad, bd, kIdesc,
+                                              (kb | kk) != 0 ? 1u : 0u);
+                            }
+                        }
+                    }
+                    ptx::mma_commit(&empty[stage]);   // frees the stage once these MMAs finish
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+                if (!ok) break;
+                for (int j = 0; j < MT; ++j) {
+                    ptx::mma_commit(&tfull[g0 + j]);
+                    ++use[g0 + j];
+                }
+            }
+            if (!ok) {
+                *abort_flag = 1;
+                set_status(status, TF_DEV_TIMEOUT);
+            }
+            // every MMA issued so far must finish before TMEM is released
+            ptx::mma_commit(drain);
+            ptx::mbar_wait(drain, 0, nullptr, kWaitLimitNs);
+        }
+    } else {
+        // ------------------------------------------------------------------ epilogue
+        const int e = warp - 2;
+        const int g = e >> 2;            // accumulator slot of this group
+        const int q = warp & 3;          // TMEM lane quarter of this warp
+        uint32_t use = 0;
+        int kl = 0;
+        for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++kl) {
+            if (MT == 1 && (kl & 1) != g) continue;
+            if (!ptx::mbar_wait(&tfull[g], use & 1u, abort_flag, kWaitLimitNs)) {
+                *abort_flag = 1;
+                set_status(status, TF_DEV_TIMEOUT);
+                break;
+            }
+            ++use;
+            ptx::tc_fence_after();
+            const int nt = u / n_mgroups, mg = u % n_mgroups;
+            const int row = (mg * MT + (MT == 2 ? g : 0)) * kBM + q * 32 + lane;
+            const uint32_t tb = tmem_base + 256u * g + (static_cast<uint32_t>(q * 32) << 16);
+
+            if constexpr (EPI == EPI_LMHEAD) {
+                float m = -INFINITY, s = 0.0f;
+                float tv[kListLen];
+                int ti[kListLen];
+#pragma unroll
+                for (int j = 0; j < kListLen; ++j) {
+                    tv[j] = -INFINITY;
+                    ti[j] = -1;
+                }
+#pragma unroll 1
+                for (int c = 0; c < BN; c += 32) {
+                    uint32_t r[32];
+                    ptx::tmem_ld_32cols(tb + c, r);
+                    const int v0 = nt * BN + c;
+                    float z[32];
+                    float cmax = -INFINITY;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        z[j] = (v0 + j < ep.V) ? __uint_as_float(r[j]) * ep.inv_temp : -INFINITY;
+                        cmax = fmaxf(cmax, z[j]);
+                    }
+                    if (cmax > m) {
+                        s *= __expf(m - cmax);
+                        m = cmax;
+                    }
+                    if (cmax > -INFINITY) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) s += __expf(z[j] - m);
+                    }
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        // ids arrive in increasing order, so a strict > keeps the smaller id first
+                        if (z[j] > tv[kListLen - 1]) {
+                            tv[kListLen - 1] = z[j];
+                            ti[kListLen - 1] = v0 + j;
+#pragma unroll
+                            for (int t = kListLen - 1; t > 0; --t) {
+                                if (tv[t] > tv[t - 1]) {
+                                    const float fv = tv[t]; tv[t] = tv[t - 1]; tv[t - 1] = fv;
+                                    const int iv = ti[t]; ti[t] = ti[t - 1]; ti[t - 1] = iv;
+                                }
+                            }
+                        }
+                    }
+                }
+                ptx::tc_fence_before();
+                ptx::mbar_arrive(&tempty[g]);
+                if (row < n_rows) {
+                    Partial* p = ep.partials + static_cast<size_t>(row) * n_ntiles + nt;
+                    float2* pf = reinterpret_cast<float2*>(p);
+                    pf[0] = make_float2(m, s);
+#pragma unroll
+                    for (int j = 0; j < kListLen; j += 2) pf[1 + j / 2] = make_float2(tv[j], tv[j + 1]);
+                    int2* pi = reinterpret_cast<int2*>(p->id);
+#pragma unroll
+                    for (int j = 0; j < kListLen; j += 2) pi[j / 2] = make_int2(ti[j], ti[j + 1]);
+                }
+            } else if constexpr (EPI == EPI_GATEUP) {
+#pragma unroll 1
+                for (int c = 0; c < BN; c += 32) {
+                    uint32_t rg[32], ru[32];
+                    ptx::tmem_ld_32cols(tb + c, rg);
+                    ptx::tmem_ld_32cols(tb + BN + c, ru);
+                    uint32_t packed[16];
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        const float a0 = silu_f(__uint_as_float(rg[2 * j])) * __uint_as_float(ru[2 * j]);
+                        const float a1 = silu_f(__uint_as_float(rg[2 * j + 1])) * __uint_as_float(ru[2 * j + 1]);
+                        packed[j] = pack_bf16x2(a0, a1);
+                    }
+                    if (row < n_rows) {
+                        uint4* dst = reinterpret_cast<uint4*>(ep.out + static_cast<size_t>(row) * ep.ld_out + nt * BN + c);
+#pragma unroll
+                        for (int j = 0; j < 4; ++j)
+                            dst[j] = make_uint4(packed[4 * j], packed[4 * j + 1], packed[4 * j + 2], packed[4 * j + 3]);
+                    }
+                }
+                ptx::tc_fence_before();
+                ptx::mbar_arrive(&tempty[g]);
+            } else {  // EPI_DOWN
+                int hid_row = 0;
+                if (row < n_rows) {
+                    const int sq = row / ep.R, rr = row - sq * ep.R;
+                    hid_row = sq * ep.gamma + stage2_hidden_index(rr, ep.M);
+                }
+#pragma unroll 1
+                for (int c = 0; c < BN; c += 32) {
+                    uint32_t ra[32];
+                    ptx::tmem_ld_32cols(tb + c, ra);
+                    if (row < n_rows) {
+                        const uint4* res = reinterpret_cast<const uint4*>(
+                            ep.hidden + static_cast<size_t>(hid_row) * ep.ld_out + nt * BN + c);
+                        uint4* dst = reinterpret_cast<uint4*>(ep.out + static_cast<size_t>(row) * ep.ld_out + nt * BN + c);
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const uint4 hv = res[j];
+                            const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w};
+                            uint32_t o[4];
+#pragma unroll
+                            for (int t = 0; t < 4; ++t) {
+                                const __nv_bfloat162 h2 = *reinterpret_cast<const __nv_bfloat162*>(&hw[t]);
+                                const float x0 = __bfloat162float(h2.x) + __uint_as_float(ra[8 * j + 2 * t]);
+                                const float x1 = __bfloat162float(h2.y) + __uint_as_float(ra[8 * j + 2 * t + 1]);
+                                o[t] = pack_bf16x2(x0, x1);
+                            }
+                            dst[j] = make_uint4(o[0], o[1], o[2], o[3]);
+                        }
+                    }
+                }
+                ptx::tc_fence_before();
+                ptx::mbar_arrive(&tempty[g]);
+            }
+        }
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem_base, 512);
+    }
+}
+
+// ------------------------------------------------------------------------------ host side
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            p = nullptr;
+        return reinterpret_cast<EncodeTiledFn>(p);
+    }();
+    return fn;
+}
+
+// Row-major bf16 matrix [outer, inner] read in boxes of box_inner x box_outer with 128B swizzle.
+cudaError_t make_tmap(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer, uint32_t box_inner,
+                      uint32_t box_outer) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return cudaErrorNotSupported;
+    const cuuint64_t dims[2] = {inner, outer};
+    const cuuint64_t strides[1] = {inner * 2};
+    const cuuint32_t box[2] = {box_inner, box_outer};
+    const cuuint32_t es[2] = {1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+template <int EPI, int MT, int NB, int BN, int STAGES>
+cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& tw0, const CUtensorMap& tw1,
+                     int n_rows, int K, int n_ntiles, int n_mgroups, const EpiParams& ep) {
+    using C = TileCfg<MT, NB, BN, STAGES>;
+    auto kern = tc_gemm_kernel<EPI, MT, NB, BN, STAGES>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    const int n_units = n_ntiles * n_mgroups;
+    const int grid = n_units < ctx.num_sms ? n_units : ctx.num_sms;
+    const int stream_once = n_mgroups == 1 ? 1 : 0;
+    kern<<<grid, kThreads, C::kSmemBytes, ctx.stream>>>(tx, tw0, tw1, n_rows, K, n_ntiles, n_mgroups, stream_once,
+                                                       ep, ctx.status);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_lmhead_tc(const Ctx& ctx, const void* lm_head, const void* x, int n_rows, int d, int V,
+                             float inv_temp, Partial* partials) {
+    if (n_rows <= 0) return cudaSuccess;
+    CUtensorMap tx, tw;
+    cudaError_t e = make_tmap(&tx, x, d, n_rows, kBK, kBM);
+    if (e == cudaSuccess) e = make_tmap(&tw, lm_head, d, V, kBK, kBlockV);
+    if (e != cudaSuccess) return e;
+    EpiParams ep{};
+    ep.partials = partials;
+    ep.V = V;
+    ep.inv_temp = inv_temp;
+    const int n_tiles = (V + kBlockV - 1) / kBlockV;
+    const int m_tiles = (n_rows + kBM - 1) / kBM;
+    if (m_tiles == 1)
+        return run_gemm<EPI_LMHEAD, 1, 1, kBlockV, 4>(ctx, tx, tw, tw, n_rows, d, n_tiles, 1, ep);
+    return run_gemm<EPI_LMHEAD, 2, 1, kBlockV, 3>(ctx, tx, tw, tw, n_rows, d, n_tiles, (m_tiles + 1) / 2, ep);
+}
+
+cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, const void* w_gate, const void* w_up,
+                             const void* w_down, const void* hidden, int n_rows, int d, int I, int R, int M,
+                             int gamma, void* A, void* h_prime) {
+    if (n_rows <= 0) return cudaSuccess;
+    constexpr int BN = 64;
+    const int m_tiles = (n_rows + kBM - 1) / kBM;
+    CUtensorMap tx, tg, tu, ta, td;
+    cudaError_t e = make_tmap(&tx, X, 2 * d, n_rows, kBK, kBM);
+    if (e == cudaSuccess) e = make_tmap(&tg, w_gate, 2 * d, I, kBK, BN);
+    if (e == cudaSuccess) e = make_tmap(&tu, w_up, 2 * d, I, kBK, BN);
+    if (e == cudaSuccess) e = make_tmap(&ta, A, I, n_rows, kBK, kBM);
+    if (e == cudaSuccess) e = make_tmap(&td, w_down, I, d, kBK, BN);
+    if (e != cudaSuccess) return e;
+    EpiParams ep{};
+    ep.out = static_cast<__nv_bfloat16*>(A);
+    ep.ld_out = I;
+    if (m_tiles == 1)
+        e = run_gemm<EPI_GATEUP, 1, 2, BN, 6>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, 1, ep);
+    else
+        e = run_gemm<EPI_GATEUP, 2, 2, BN, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, (m_tiles + 1) / 2, ep);
+    if (e != cudaSuccess) return e;
+    EpiParams ed{};
+    ed.out = static_cast<__nv_bfloat16*>(h_prime);
+    ed.ld_out = d;
+    ed.hidden = static_cast<const __nv_bfloat16*>(hidden);
+    ed.R = R;
+    ed.M = M;
+    ed.gamma = gamma;
+    if (m_tiles == 1)
+        return run_gemm<EPI_DOWN, 1, 1, BN, 8>(ctx, ta, td, td, n_rows, I, d / BN, 1, ed);
+    return run_gemm<EPI_DOWN, 2, 1, BN, 5>(ctx, ta, td, td, n_rows, I, d / BN, (m_tiles + 1) / 2, ed);
+}
+
+}  // namespace tf

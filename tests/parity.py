@@ -1,0 +1,190 @@
+"""GPU-vs-oracle parity checks (test infrastructure; used by tests/ and __graft_entry__.smoke()).
+
+Both sides read the same seeded inputs from synth/. The oracle runs in float64 (optionally with
+bf16 rounding at the points where the CUDA path stores bf16). Comparison rules:
+
+* log-probabilities (stage-1 top-K1, stage-2 top-K2, node scores): every value the GPU reports
+  for a token id must be within `tol_lp` of the oracle's exact log-probability of that id, and
+  the GPU's sorted values must match the oracle's sorted top values rank by rank within
+  `tol_lp` (so a swap of two near-equal entries is allowed, a wrong value is not). Node scores
+  are sums of up to depth log-probabilities and get depth * tol_lp.
+* ids: the top-M candidate set of every depth (which decides the M-ary tree) must equal the
+  oracle's whenever the oracle's gap at rank M exceeds `tol_sel`; stage-2 rows are paired with
+  oracle rows by (depth, previous token).
+* tree: when the oracle's order margin exceeds `tol_sel` the token, parent and depth arrays
+  must be bit-exact (same pop order); when only the set margin does, the trees must be equal
+  as sets of token paths. Otherwise only validity is checked (prefix-closed, M-ary rule,
+  scores = sums of the GPU's own child log-probs).
+* mask / position ids: always bit-exact against the oracle's mask of the GPU's own tree, and
+  against the oracle's tree when that was required to match.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import synth
+from oracle import treeflash_oracle as O
+
+TOLS = {
+    # lp: stage-1 log-probs vs the plain fp64 oracle; lp2: stage-2 log-probs vs the plain oracle
+    # (the bf16 path rounds x, SiLU(G)*U and h' to bf16 before the next GEMM, see the design
+    # notes for the bound); lp_emul: everything vs the oracle that rounds at those points;
+    # sel: selection margin above which the tree structure must match exactly.
+    "f32": dict(lp=1e-4, lp2=1e-4, lp_emul=1e-4, sel=1e-3),
+    "bf16": dict(lp=2e-2, lp2=6e-2, lp_emul=5e-3, sel=2e-2),
+}
+
+
+def oracle_weights(inp):
+    return O.weights_f64(inp, synth.to_f64)
+
+
+def run_oracle(cfg, inp, emulate_bf16=False, seqs=None, W=None):
+    W = W if W is not None else oracle_weights(inp)
+    H = synth.to_f64(inp["hidden"])
+    seqs = range(cfg.batch) if seqs is None else seqs
+    out = []
+    for s in seqs:
+        out.append(O.draft_sequence(H[s], int(inp["root_tok"][s]), int(inp["root_pos"][s]), W,
+                                    M=cfg.M, K2=cfg.K2, B=cfg.B, temperature=cfg.temperature,
+                                    eps=cfg.rms_eps, mode=cfg.mode, emulate_bf16=emulate_bf16,
+                                    keep=cfg.K2 if cfg.K2 < cfg.B else None))
+    return out
+
+
+def device_inputs(inp, device="cuda"):
+    keys = ("hidden", "lm_head", "embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down", "root_tok",
+            "root_pos")
+    return {k: inp[k].to(device).contiguous() for k in keys}
+
+
+def run_gpu(cfg, dinp, drafter=None):
+    from paper_2606_03819_gb300 import Dims, Drafter
+    dims = Dims.from_config(cfg)
+    dr = drafter or Drafter(dims, dinp)
+    out = dr.draft(dinp["hidden"], dinp["root_tok"], dinp["root_pos"])
+    flags = dr.status()
+    res = {k: (v.cpu().numpy() if v is not None else None) for k, v in out.items()}
+    res["flags"] = flags
+    res["root_pos"] = dinp["root_pos"].cpu().numpy()
+    return res
+
+
+def _check_row(gpu_ids, gpu_lp, full_lp, tol, what):
+    """GPU top list vs the oracle's full distribution of the same row."""
+    ids = np.asarray(gpu_ids)
+    assert (ids >= 0).all() and (ids < full_lp.shape[0]).all(), f"{what}: id out of range"
+    assert len(set(ids.tolist())) == len(ids), f"{what}: duplicate ids"
+    err_id = np.abs(gpu_lp - full_lp[ids]).max()
+    top = np.sort(full_lp)[::-1][: len(ids)]
+    err_rank = np.abs(np.sort(gpu_lp)[::-1] - top).max()
+    assert err_id <= tol, f"{what}: logp of reported ids off by {err_id:.3g} > {tol}"
+    assert err_rank <= tol, f"{what}: sorted top values off by {err_rank:.3g} > {tol}"
+    return max(err_id, err_rank)
+
+
+def compare(cfg, gpu, orc, tol_lp, tol_sel, check_structure=True, tol_lp2=None):
+    """Assert parity of one batch; returns a small report dict."""
+    tol_lp2 = tol_lp if tol_lp2 is None else tol_lp2
+    rep = dict(max_err_s1=0.0, max_err_s2=0.0, max_err_score=0.0, rows_s2=0, rows_s2_skipped=0,
+               exact_trees=0, set_trees=0, valid_only_trees=0)
+    M, g = cfg.M, cfg.gamma
+    for s, o in enumerate(orc):
+        # ---- stage 1
+        for i in range(g):
+            e = _check_row(gpu["top_ids"][s, i], gpu["top_logp"][s, i], o.s1_logp[i], tol_lp, f"seq {s} depth {i + 1}")
+            rep["max_err_s1"] = max(rep["max_err_s1"], e)
+            if i < g - 1 and O.topk_margin(o.s1_logp[i], M) > tol_sel:
+                assert set(gpu["top_ids"][s, i, :M].tolist()) == set(o.top_ids[i, :M].tolist()), \
+                    f"seq {s} depth {i + 1}: top-M set differs"
+        # ---- stage 2, rows paired by (depth, previous token)
+        if cfg.mode == "ar":
+            hid, prev = O.stage2_conditioning(g, M, int(o.tree.tok[0]), o.top_ids)
+            okey = {(int(h), int(p)): r for r, (h, p) in enumerate(zip(hid, prev))}
+            ghid, gprev = O.stage2_conditioning(g, M, int(o.tree.tok[0]), gpu["top_ids"][s])
+            for r, (h, p) in enumerate(zip(ghid, gprev)):
+                orow = okey.get((int(h), int(p)))
+                if orow is None:
+                    rep["rows_s2_skipped"] += 1
+                    continue
+                e = _check_row(gpu["child_ids"][s, r], gpu["child_logp"][s, r], o.s2_logp[orow], tol_lp2,
+                               f"seq {s} stage-2 row {r}")
+                rep["max_err_s2"] = max(rep["max_err_s2"], e)
+                rep["rows_s2"] += 1
+        # ---- tree
+        tok, par, dep, sc = (gpu["node_tok"][s], gpu["node_parent"][s], gpu["node_depth"][s],
+                             gpu["node_score"][s])
+        _check_tree_valid(cfg, gpu, s)
+        if check_structure:
+            set_m, order_m = O.selection_margins(o, M, cfg.K2, cfg.B, cfg.mode)
+            if order_m > tol_sel:
+                np.testing.assert_array_equal(tok, o.tree.tok, err_msg=f"seq {s} tokens")
+                np.testing.assert_array_equal(par, o.tree.parent, err_msg=f"seq {s} parents")
+                np.testing.assert_array_equal(dep, o.tree.depth, err_msg=f"seq {s} depths")
+                np.testing.assert_array_equal(gpu["mask"][s], o.mask, err_msg=f"seq {s} mask")
+                np.testing.assert_array_equal(gpu["pos_ids"][s], o.pos, err_msg=f"seq {s} pos")
+                present = o.tree.parent >= 0
+                present[0] = True
+                err = np.abs(sc[present] - o.tree.score[present])
+                lim = np.maximum(dep[present], 1) * max(tol_lp, tol_lp2)
+                assert (err <= lim).all(), f"seq {s}: node score off by {err.max():.3g}"
+                rep["max_err_score"] = max(rep["max_err_score"], float(err.max()))
+                rep["exact_trees"] += 1
+            elif set_m > tol_sel:
+                gp = _paths(tok, par)
+                assert gp == set(O.tree_paths(o.tree)), f"seq {s}: tree differs as a set"
+                rep["set_trees"] += 1
+            else:
+                rep["valid_only_trees"] += 1
+        # ---- mask of the GPU's own tree
+        m, pos = O.tree_mask(par.astype(np.int64), dep.astype(np.int64), int(gpu["root_pos"][s]))
+        np.testing.assert_array_equal(gpu["mask"][s], m, err_msg=f"seq {s} mask of own tree")
+        np.testing.assert_array_equal(gpu["pos_ids"][s], pos, err_msg=f"seq {s} pos of own tree")
+    return rep
+
+
+def _paths(tok, par):
+    paths = {0: ()}
+    out = set()
+    for i in range(1, tok.shape[0]):
+        if par[i] < 0:
+            continue
+        paths[i] = paths[int(par[i])] + (int(tok[i]),)
+        out.add(paths[i])
+    return out
+
+
+def _check_tree_valid(cfg, gpu, s):
+    tok, par, dep, sc = (gpu["node_tok"][s], gpu["node_parent"][s], gpu["node_depth"][s], gpu["node_score"][s])
+    n = cfg.B + 1
+    assert tok.shape == (n,)
+    assert par[0] == -1 and dep[0] == 0 and sc[0] == 0.0
+    seen = set()
+    for i in range(1, n):
+        p = int(par[i])
+        if p < 0:
+            assert tok[i] == -1 and dep[i] == -1
+            continue
+        assert 0 <= p < i, f"seq {s} node {i}: parent {p}"
+        assert dep[i] == dep[p] + 1 <= cfg.gamma
+        assert sc[i] <= sc[p] + 1e-6
+        assert (p, int(tok[i])) not in seen
+        seen.add((p, int(tok[i])))
+        # score = parent score + the GPU's own log-prob of this token in the child list used
+        if cfg.mode == "ar":
+            if dep[i] == 1:
+                row = 0
+            else:
+                pt = int(tok[p])
+                cand = gpu["top_ids"][s, dep[p] - 1, : cfg.M].tolist()
+                assert pt in cand, f"seq {s} node {p} expanded outside the M-ary tree"
+                row = 1 + (dep[p] - 1) * cfg.M + cand.index(pt)
+            ids, lp = gpu["child_ids"][s, row], gpu["child_logp"][s, row]
+        else:
+            if cfg.mode == "marginal_mary" and dep[i] > 1:
+                assert int(tok[p]) in gpu["top_ids"][s, dep[p] - 1, : cfg.M].tolist()
+            ids, lp = gpu["top_ids"][s, dep[i] - 1, : cfg.K2], gpu["top_logp"][s, dep[i] - 1, : cfg.K2]
+        where = np.nonzero(ids == tok[i])[0]
+        assert where.size == 1, f"seq {s} node {i}: token not in its child list"
+        assert abs(sc[i] - (sc[p] + lp[where[0]])) <= 1e-5 * max(1.0, abs(sc[i]))

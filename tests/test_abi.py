@@ -1,0 +1,103 @@
+"""The C-ABI library builds, loads and exports every symbol include/treeflash.h declares; host-side
+argument validation works without a GPU (no compute call is made here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2606_03819_gb300 import binding
+    if not os.path.exists(binding.LIB_PATH):
+        from paper_2606_03819_gb300 import build
+        build.build()
+    return binding.load_library()
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "treeflash.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(tf_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_header_declares_the_north_star_calls():
+    names = declared_functions()
+    for n in ("tf_stage1_marginals", "tf_stage2_ar_approx", "tf_build_tree", "tf_tree_mask"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    from paper_2606_03819_gb300 import binding
+    names = declared_functions()
+    assert set(names) == set(binding.EXPORTS)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_version_and_status_strings(lib):
+    assert lib.tf_version() >= 100
+    for s in range(7):
+        assert lib.tf_status_string(s)
+
+
+def _dims(**kw):
+    from paper_2606_03819_gb300.binding import Dims
+    base = dict(batch=1, d=128, V=2048, I=512, gamma=4, M=4, K2=12, B=12, dtype="f32", mode="ar")
+    base.update(kw)
+    return Dims(**base)
+
+
+def test_workspace_size_and_validation(lib):
+    from paper_2606_03819_gb300 import binding as Bn
+    assert Bn.tf_workspace_size(_dims()) > 0
+    q8 = Bn.Dims.from_config(synth.get_config("q8_b64"))
+    n = Bn.tf_workspace_size(q8)
+    # partials of the larger pass: 241 rows x 594 blocks x 72 bytes, plus h', X, A
+    assert n >= 241 * 594 * 72 + 241 * 4096 * 2 * 4
+    bad = [dict(batch=0), dict(V=8, K2=12), dict(gamma=0), dict(M=0), dict(temperature=0.0),
+           dict(mode="nope"), dict(I=0)]
+    for kw in bad:
+        if kw.get("mode") == "nope":
+            continue
+        with pytest.raises(Bn.TreeFlashError) as e:
+            Bn.tf_workspace_size(_dims(**kw))
+        assert e.value.status == Bn.TF_ERR_INVALID_ARG, kw
+    for kw in (dict(M=33), dict(K2=65), dict(B=2000), dict(gamma=65), dict(dtype="bf16", d=100),
+               dict(dtype="bf16", I=100)):
+        with pytest.raises(Bn.TreeFlashError) as e:
+            Bn.tf_workspace_size(_dims(**kw))
+        assert e.value.status == Bn.TF_ERR_UNSUPPORTED, kw
+
+
+def test_null_arguments_are_rejected_before_any_gpu_work(lib):
+    from paper_2606_03819_gb300 import binding as Bn
+    d = _dims()
+    c = d.c()
+    w = Bn.TfWeights()
+    # null workspace -> TF_ERR_WORKSPACE; null dims -> TF_ERR_INVALID_ARG; all host-side
+    assert lib.tf_stage1_marginals(None, ctypes.byref(w), None, None, None, None, 0, None) == Bn.TF_ERR_INVALID_ARG
+    assert lib.tf_stage1_marginals(ctypes.byref(c), ctypes.byref(w), None, None, None, None, 0,
+                                   None) == Bn.TF_ERR_WORKSPACE
+    assert lib.tf_build_tree(ctypes.byref(c), *([None] * 10), None) == Bn.TF_ERR_INVALID_ARG
+    assert lib.tf_tree_mask(ctypes.byref(c), None, None, None, None, None, None) == Bn.TF_ERR_INVALID_ARG
+    assert lib.tf_status_reset(None, 0, None) == Bn.TF_ERR_WORKSPACE
+    flags = ctypes.c_int32()
+    assert lib.tf_status_read(None, 0, ctypes.byref(flags), None) == Bn.TF_ERR_WORKSPACE
+    n = ctypes.c_size_t()
+    assert lib.tf_workspace_size(ctypes.byref(c), None) == Bn.TF_ERR_INVALID_ARG
+
+
+def test_product_path_never_imports_the_oracle():
+    # the binding and package sources must not reference oracle/ (no CPU fallback)
+    pkg = os.path.join(ROOT, "paper_2606_03819_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h", ".cpp")):
+                txt = open(os.path.join(dirpath, f)).read()
+                assert "oracle" not in txt.lower(), f

@@ -1,0 +1,224 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle on the same seeded inputs.
+
+Tolerances (tests/parity.py): fp32 inputs 1e-4 absolute on log-probabilities; bf16 inputs with
+fp32 accumulation 2e-2 absolute against the plain fp64 oracle and 5e-3 against the oracle that
+rounds to bf16 where the CUDA path stores bf16. Tree structure is compared bit-exactly wherever
+the oracle's selection margin exceeds 1e-3 (fp32) / 2e-2 (bf16).
+"""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import treeflash_oracle as O
+
+pytestmark = pytest.mark.gpu
+
+import parity  # noqa: E402  (tests/ is on sys.path)
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_03819_gb300 import binding
+    if not __import__("os").path.exists(binding.LIB_PATH):
+        from paper_2606_03819_gb300 import build
+        build.build()
+    binding.load_library()
+
+
+def check(cfg, emulate_also=True, inp=None, orc_seqs=None):
+    inp = inp if inp is not None else synth.make_inputs(cfg)
+    dinp = parity.device_inputs(inp)
+    gpu = parity.run_gpu(cfg, dinp)
+    tol = parity.TOLS[cfg.dtype]
+    W = parity.oracle_weights(inp)
+    reps = {}
+    seqs = list(range(cfg.batch)) if orc_seqs is None else orc_seqs
+    sub = {k: (v[seqs] if isinstance(v, np.ndarray) and v.ndim >= 1 and v.shape[0] == cfg.batch else v)
+           for k, v in gpu.items()}
+    orc = parity.run_oracle(cfg, inp, emulate_bf16=False, seqs=seqs, W=W)
+    reps["pure"] = parity.compare(cfg, sub, orc, tol["lp"], tol["sel"],
+                                  check_structure=cfg.dtype == "f32", tol_lp2=tol["lp2"])
+    if cfg.dtype == "bf16" and emulate_also:
+        orc_e = parity.run_oracle(cfg, inp, emulate_bf16=True, seqs=seqs, W=W)
+        reps["emul"] = parity.compare(cfg, sub, orc_e, tol["lp_emul"], tol["sel"])
+    assert not (gpu["flags"] & ~16), f"device flags {gpu['flags']}"
+    return gpu, reps
+
+
+# ------------------------------------------------------------------ fp32 (CUDA-core) path
+
+
+@pytest.mark.parametrize("name", ["tiny_f32", "tiny_peaked"])
+def test_fp32_tiny(name):
+    _, reps = check(synth.get_config(name))
+    print(reps)
+
+
+@pytest.mark.parametrize("mode", ["marginal", "marginal_mary"])
+def test_fp32_marginal_modes(mode):
+    check(synth.get_config("tiny_peaked", mode=mode))
+
+
+def test_fp32_brute_force_v16():
+    cfg = synth.get_config("tiny_v16", h_entropy=(1.0, 1.5), wd_std=0.5)
+    gpu, _ = check(cfg)
+    inp = synth.make_inputs(cfg)
+    o = parity.run_oracle(cfg, inp)[0]
+    src = O.ChildSource("ar", cfg.gamma, cfg.M, o.top_ids, o.s1_logp, o.s2_logp)
+    uni = sorted(O.eligible_universe(src), key=lambda x: (-x[0], x[1]))
+    best = {p for _, _, p in uni[: cfg.B]}
+    assert parity._paths(gpu["node_tok"][0], gpu["node_parent"][0]) == best
+
+
+# ------------------------------------------------------------------ bf16 (tcgen05) path
+
+BF16_SMALL = [
+    # (batch, V, gamma, M, K2, B): stage-1 rows b*gamma, stage-2 rows b*(1+M(gamma-1))
+    (2, 2000, 4, 4, 12, 12),     # 8 / 26 rows: one M-tile, ragged last vocabulary block
+    (12, 2304, 4, 4, 12, 12),    # 48 / 156 rows: two M-tiles in one unit
+    (24, 2049, 4, 4, 12, 12),    # 96 / 312 rows: three M-tiles (half-empty last group), V = 8*256+1
+    (40, 1536, 4, 4, 8, 16),     # 160 / 520 rows: two M-tiles already in stage 1; K2 < B
+]
+
+
+@pytest.mark.parametrize("b,V,gamma,M,K2,B", BF16_SMALL)
+def test_bf16_small(b, V, gamma, M, K2, B):
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=b, V=V, gamma=gamma, M=M, K2=K2, B=B)
+    _, reps = check(cfg)
+    print(reps)
+
+
+def test_bf16_d_and_I_several_k_blocks():
+    # d = 320 (5 K-steps of 64), I = 192 (3 N-tiles of 64 in the MLP), gamma 5, M 3
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=3, d=320, I=192, V=3000, gamma=5, M=3,
+                           K2=16, B=16)
+    check(cfg)
+
+
+@pytest.mark.parametrize("mode", ["marginal", "marginal_mary"])
+def test_bf16_marginal_modes(mode):
+    check(synth.get_config("tiny_peaked", dtype="bf16", batch=3, V=2000, mode=mode))
+
+
+def test_bf16_zero_approximator_equals_mary_marginal_tree():
+    # W_down = 0 gives h' = h exactly, so TreeFlash's tree is the M-ary marginal tree
+    from paper_2606_03819_gb300 import Dims
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=4, V=2000)
+    inp = synth.make_inputs(cfg)
+    inp["w_down"].zero_()
+    d = parity.device_inputs(inp)
+    a = parity.run_gpu(cfg, d)
+    b = parity.run_gpu(cfg.replace(mode="marginal_mary"), d)
+    for k in ("node_tok", "node_parent", "node_depth", "mask", "pos_ids"):
+        np.testing.assert_array_equal(a[k], b[k], err_msg=k)
+    np.testing.assert_array_equal(a["node_score"], b["node_score"])
+
+
+def test_bf16_batch_equals_single_sequences():
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=5, V=2000)
+    inp = synth.make_inputs(cfg)
+    full = parity.run_gpu(cfg, parity.device_inputs(inp))
+    one = cfg.replace(batch=1)
+    for s in range(cfg.batch):
+        sub = dict(inp)
+        for k in ("hidden", "root_tok", "root_pos"):
+            sub[k] = inp[k][s:s + 1].contiguous()
+        r = parity.run_gpu(one, parity.device_inputs(sub))
+        for k in ("top_ids", "top_logp", "child_ids", "child_logp", "node_tok", "node_parent", "node_score",
+                  "mask", "pos_ids"):
+            np.testing.assert_array_equal(r[k][0], full[k][s], err_msg=f"{k} seq {s}")
+
+
+def test_bf16_recompute_path_is_exact():
+    # 80 vocabulary rows of one 256-block aligned with every hidden state: the top-64 of each row
+    # all sit in that block, so its 8-entry list is certified incomplete and recomputed
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=1, V=4096, K2=64, B=64, M=4)
+    inp = synth.make_inputs(cfg)
+    g = torch.Generator().manual_seed(5)
+    dirn = inp["hidden"][0].float().mean(0)
+    W = inp["lm_head"].float()
+    W[512:592] = dirn / dirn.norm() * (0.2 + 0.05 * torch.rand(80, 1, generator=g))
+    inp["lm_head"] = W.to(torch.bfloat16)
+    gpu = parity.run_gpu(cfg, parity.device_inputs(inp))
+    assert gpu["flags"] & 16, "the certification should have triggered a recompute"
+    orc = parity.run_oracle(cfg, inp, emulate_bf16=True)
+    parity.compare(cfg, gpu, orc, parity.TOLS["bf16"]["lp_emul"], parity.TOLS["bf16"]["sel"])
+
+
+def test_host_path_matches_device_path():
+    from paper_2606_03819_gb300 import Dims, alloc_workspace, binding
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=3, V=2000)
+    inp = synth.make_inputs(cfg)
+    d = parity.device_inputs(inp)
+    dev = parity.run_gpu(cfg, d)
+    dims = Dims.from_config(cfg)
+    ws = alloc_workspace(dims)
+    n = cfg.B + 1
+    pin = lambda t: t.pin_memory()
+    out = dict(node_tok=torch.empty(cfg.batch, n, dtype=torch.int32), node_parent=torch.empty(cfg.batch, n, dtype=torch.int32),
+               node_depth=torch.empty(cfg.batch, n, dtype=torch.int32), node_score=torch.empty(cfg.batch, n),
+               mask=torch.empty(cfg.batch, n, n, dtype=torch.uint8), pos_ids=torch.empty(cfg.batch, n, dtype=torch.int32),
+               dev_status=torch.empty(cfg.batch, dtype=torch.int32))
+    out = {k: pin(v) for k, v in out.items()}
+    st = binding.tf_draft_tree_host(dims, d, pin(inp["hidden"]), pin(inp["root_tok"]), pin(inp["root_pos"]),
+                                    out["node_tok"], out["node_parent"], out["node_depth"], out["node_score"],
+                                    out["mask"], out["pos_ids"], out["dev_status"], ws)
+    assert st == 0
+    for k in ("node_tok", "node_parent", "node_depth", "node_score", "mask", "pos_ids"):
+        np.testing.assert_array_equal(out[k].numpy(), dev[k], err_msg=k)
+
+
+def test_bad_root_token_is_flagged_not_fatal():
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=2, V=2000)
+    inp = synth.make_inputs(cfg)
+    inp["root_tok"][1] = cfg.V + 7
+    gpu = parity.run_gpu(cfg, parity.device_inputs(inp))
+    assert gpu["flags"] & 1
+    assert gpu["dev_status"][1] & 1 and not gpu["dev_status"][0] & 1
+
+
+def test_underfull_universe_is_flagged():
+    cfg = synth.get_config("tiny_peaked", gamma=1, M=2, K2=4, B=8)
+    inp = synth.make_inputs(cfg)
+    gpu = parity.run_gpu(cfg, parity.device_inputs(inp))
+    assert gpu["dev_status"][0] & 2
+    assert (gpu["node_parent"][0, 5:] == -1).all() and (gpu["node_tok"][0, 5:] == -1).all()
+    assert gpu["mask"][0, 5:].sum() == 0 and gpu["mask"][0, :, 5:].sum() == 0
+    orc = parity.run_oracle(cfg, inp)
+    assert orc[0].tree.underfull
+    np.testing.assert_array_equal(gpu["node_tok"][0], orc[0].tree.tok)
+
+
+# ------------------------------------------------------------------ full sizes (the measured shapes)
+
+_cache = {}
+
+
+def _inputs(name):
+    if name not in _cache:
+        _cache.clear()
+        _cache[name] = synth.make_inputs(synth.get_config(name))
+    return _cache[name]
+
+
+@pytest.mark.parametrize("name", ["q8_b64", "q8_b32"])
+def test_full_size_qwen3_8b_shape(name):
+    cfg = synth.get_config(name)
+    gpu, reps = check(cfg, inp=_inputs(name))
+    print(name, reps)
+    # depth-1 to depth-16 entropies ramp, so the tree must reach beyond depth 2
+    assert gpu["node_depth"][0].max() >= 3
+
+
+def test_full_size_batch32_sampled_sequences():
+    cfg = synth.get_config("batch32")
+    check(cfg, orc_seqs=[0, 17, 31], emulate_also=False)
+
+
+@pytest.mark.parametrize("name", ["wide_peaked", "wide_flat"])
+def test_full_size_wide_sampled_sequence(name):
+    cfg = synth.get_config(name)
+    check(cfg, orc_seqs=[3], emulate_also=False)
