@@ -1,0 +1,423 @@
+"""Benchmark of the TreeFlash drafting hot path: one step = one whole draft-tree build.
+
+A step runs every call of the path on the batch of the measured workload (Qwen3-8B shape,
+gamma=16, M=16, B=64, batch 1): the stage-1 LM-head pass and its top-k merge, the
+AR-approximator (Eq. 1), the stage-2 LM-head pass and merge, the best-first tree build and the
+mask. Inputs are seeded synthetic tensors already resident in HBM; W_lm (1.245 GB) is streamed
+twice per step, far beyond the 129 MB L2, so nothing is flushed between steps.
+
+Output: one JSON line on rank 0 (see --help for the arms). The `roofline` object covers the
+dominant kernel (the fused LM-head pass): algorithmic bytes per launch (|W_lm| + the activation
+rows) over its average CUDA-event duration inside the timed region. `e2e` is the same metric
+through tf_draft_tree_host with the step's inputs and outputs in pinned host memory, copies
+inside the timed region. `cpu_baseline` is the fp64 oracle on the host cores on a bounded sample.
+
+Multi-GPU (torchrun, one rank per GPU): every rank builds its own trees (independent replicas,
+no collective on the data path); value = all trees built / max over ranks of the timed span.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "µs per draft-tree build (trees/s) at Qwen3-8B shape, B=32/64; % of HBM roofline"
+WORKLOAD = "q8_b64"
+FALLBACK_HBM_GBS = 6800.0
+
+
+# ------------------------------------------------------------------------------ distributed
+
+def dist_env():
+    return int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), \
+        int(os.environ.get("LOCAL_RANK", "0"))
+
+
+def init_dist(backend: str):
+    import torch.distributed as dist
+    rank, world, _ = dist_env()
+    if world > 1 and not dist.is_initialized():
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend=backend, rank=rank, world_size=world)
+    return rank, world
+
+
+def barrier(world: int, device=None):
+    if world > 1:
+        import torch.distributed as dist
+        if device is not None and dist.get_backend() == "nccl":
+            dist.barrier(device_ids=[device.index])
+        else:
+            dist.barrier()
+
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device if dist.get_backend() == "nccl" else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while the timed region runs."""
+
+    FIELDS = "clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown," \
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown," \
+             "clocks_event_reasons.sw_power_cap"
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.25)
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in (self.out or "").splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        # samples under load: the upper part of the trace (the sampler brackets the region)
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------ helpers
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for f in ("tc_gemm.cu", "tc_ptx.cuh", "common.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2606_03819_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic():
+    """dram bytes per launch of the LM-head pass from the committed ncu summary, or None when
+    the kernel sources changed since the counters were taken."""
+    p = os.path.join(ROOT, "profiles", "lmhead_traffic.json")
+    try:
+        d = json.load(open(p))
+    except (OSError, ValueError):
+        return None
+    if d.get("source_hash") != kernel_source_hash():
+        return None
+    return d.get("dram_bytes_per_launch")
+
+
+def algorithmic_bytes(cfg):
+    """Bytes a tree build must move at least: W_lm twice (stage 2 needs the global stage-1
+    top-M first, and W_lm is ~10x the L2), the three approximator matrices, the gathered
+    embedding rows and the hidden states. Outputs are ignored."""
+    e = 2 if cfg.dtype == "bf16" else 4
+    lm = cfg.V * cfg.d * e
+    mlp = (2 * cfg.I * 2 * cfg.d + cfg.d * cfg.I) * e   # W_gate, W_up [I, 2d]; W_down [d, I]
+    rows = cfg.batch * cfg.R
+    gathered = rows * cfg.d * e
+    hidden = cfg.batch * cfg.gamma * cfg.d * e
+    return 2 * lm + mlp + gathered + hidden, lm
+
+
+# ------------------------------------------------------------------------------ oracle timing
+
+class OracleSample:
+    """The fp64 oracle on one sequence of the workload, with the vocabulary cut to a fraction
+    (the LM-head passes, log-softmax and sorting scale with V; the approximator does not).
+    Weights are widened to float64 once, outside any timing."""
+
+    def __init__(self, cfg, inp):
+        import synth
+        self.cfg = cfg
+        self.W = {k: synth.to_f64(inp[k]) for k in ("embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down")}
+        self.lm = synth.to_f64(inp["lm_head"])
+        self.H = synth.to_f64(inp["hidden"][0])
+        self.root = int(inp["root_tok"][0])
+
+    def run(self, fraction: float):
+        """Returns (seconds for the sample, estimated seconds for a whole tree, vocabulary used)."""
+        import numpy as np
+        from oracle import treeflash_oracle as O
+        cfg = self.cfg
+        Vs = max(cfg.K2 + cfg.M, int(math.ceil(cfg.V * fraction)))
+        W = dict(self.W, lm_head=self.lm[:Vs])
+        root = self.root % Vs
+        hid, prev = O.stage2_conditioning(cfg.gamma, cfg.M, root, np.zeros((cfg.gamma, cfg.M), dtype=np.int64))
+        t0 = time.perf_counter()
+        O.ar_approximator(self.H[hid], W["embed"][prev], W["norm_h"], W["norm_e"], W["w_gate"], W["w_up"],
+                          W["w_down"], cfg.rms_eps)
+        t_mlp = time.perf_counter() - t0
+        t0 = time.perf_counter()
+        O.draft_sequence(self.H, root, 0, W, M=cfg.M, K2=cfg.K2, B=cfg.B, temperature=cfg.temperature,
+                         eps=cfg.rms_eps, mode=cfg.mode)
+        t = time.perf_counter() - t0
+        full = t_mlp + max(t - t_mlp, 0.0) * cfg.V / Vs
+        return t, full, Vs
+
+
+def cpu_threads():
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(k, "").isdigit():
+            return int(os.environ[k])
+    return os.cpu_count() or 1
+
+
+# ------------------------------------------------------------------------------ arms
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if world > 1:
+        init_dist("gloo")
+        if rank != 0:
+            return
+    import synth
+    cfg = synth.get_config(args.workload)
+    inp = synth.make_inputs(cfg)
+    orc = OracleSample(cfg, inp)
+    # calibrate on 1/64 of the vocabulary, then size every step so the run stays ~2 minutes
+    _, full_est, _ = orc.run(1 / 64)
+    n = max(1, args.steps + args.warmup)
+    frac = min(1.0, max(1 / 256, 120.0 / (n * max(full_est, 1e-3))))
+    for _ in range(args.warmup):
+        orc.run(frac)
+    ests = []
+    for _ in range(max(1, args.steps)):
+        _, full, Vs = orc.run(frac)
+        ests.append(full)
+    t_tree = sum(ests) / len(ests)
+    value = 1.0 / t_tree
+    cores = cpu_threads()
+    sample = f"fp64 oracle, 1 sequence, vocabulary cut to {Vs} of {cfg.V} per step; time scaled to the full V"
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "trees/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_tree * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": cfg.name, "batch": cfg.batch, "d": cfg.d, "V": cfg.V, "I": cfg.I,
+                       "gamma": cfg.gamma, "M": cfg.M, "K2": cfg.K2, "B": cfg.B},
+            "cpu_baseline": {"value": value, "unit": "trees/s", "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "trees/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_gpu(args):
+    import torch
+    rank, world, local = dist_env()
+    if world > 1:
+        init_dist("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    import synth
+    import paper_2606_03819_gb300 as tf
+    from paper_2606_03819_gb300 import binding as Bn
+
+    cfg = synth.get_config(args.workload, seed=rank)
+    inp = synth.make_inputs(cfg)
+    d = {k: v.to(dev) for k, v in inp.items() if isinstance(v, torch.Tensor)}
+    dims = Bn.Dims.from_config(cfg)
+    dr = tf.Drafter(dims, d, dev)
+    hp = Bn.tf_workspace_h_prime(dims, dr.ws)
+    H = d["hidden"]
+    n1, n2 = cfg.batch * cfg.gamma, cfg.batch * cfg.R
+    stream = torch.cuda.current_stream(dev)
+
+    def step(ev=None):
+        # exactly the kernels of tf_stage1_marginals + tf_stage2_ar_approx + tf_build_tree +
+        # tf_tree_mask, issued as their pieces so the LM-head passes can be timed on their own
+        Bn.tf_status_reset(dr.ws)
+        if ev is not None:
+            ev[0].record(stream)
+        Bn.tf_lmhead_partials(dims, d["lm_head"], H, n1, dr.ws)
+        if ev is not None:
+            ev[1].record(stream)
+        Bn.tf_lmhead_merge(dims, d["lm_head"], H, n1, dims.K1, dr.top_ids, dr.top_logp, dr.ws)
+        Bn.tf_ar_approx(dims, d, H, d["root_tok"], dr.top_ids, None, dr.ws)
+        if ev is not None:
+            ev[2].record(stream)
+        Bn.tf_lmhead_partials(dims, d["lm_head"], hp, n2, dr.ws)
+        if ev is not None:
+            ev[3].record(stream)
+        Bn.tf_lmhead_merge(dims, d["lm_head"], hp, n2, dims.K2, dr.child_ids, dr.child_logp, dr.ws)
+        dr.build(d["root_tok"], d["root_pos"])
+
+    kernels_per_step = 9   # 2x LM-head pass, 2x merge, gather+norm, gate/up, down, tree, mask
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize(dev)
+    flags = Bn.tf_status_read(dr.ws)
+    # sanity: the step's result is the composite API's result
+    ref = {k: v.clone() for k, v in dr.draft(H, d["root_tok"], d["root_pos"]).items() if v is not None}
+    step()
+    torch.cuda.synchronize(dev)
+    for k in ("node_tok", "node_parent", "mask"):
+        assert torch.equal(ref[k], getattr(dr, k)), k
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    barrier(world, dev)
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local) as clk:
+        t_start.record(stream)
+        for i in range(args.steps):
+            step(evs[i])
+        t_end.record(stream)
+        torch.cuda.synchronize(dev)
+    barrier(world, dev)
+    elapsed_ms = t_start.elapsed_time(t_end)
+    elapsed_ms = max_over_ranks(elapsed_ms, world, dev)
+    lm1 = [e[0].elapsed_time(e[1]) for e in evs]
+    lm2 = [e[2].elapsed_time(e[3]) for e in evs]
+    flags |= Bn.tf_status_read(dr.ws)
+
+    trees = cfg.batch * args.steps * world
+    value = trees / (elapsed_ms / 1e3)
+    ms_per_step = elapsed_ms / args.steps
+    peak, peak_kind = peaks()
+    step_bytes, lm_bytes = algorithmic_bytes(cfg)
+    e = 2
+    lm_launch_bytes = [lm_bytes + n1 * cfg.d * e, lm_bytes + n2 * cfg.d * e]
+    avg_launch_ms = (sum(lm1) + sum(lm2)) / (2 * args.steps)
+    achieved = (sum(lm_launch_bytes) / 2) / (avg_launch_ms / 1e3) / 1e9
+    traffic = profiled_traffic()
+
+    # ---- end to end through the host-buffer entry point
+    e2e = None
+    if args.e2e_steps > 0:
+        n = cfg.B + 1
+        pin = lambda t: t.pin_memory()
+        h_hidden, h_root, h_pos = pin(inp["hidden"]), pin(inp["root_tok"]), pin(inp["root_pos"])
+        outs = dict(node_tok=torch.empty(cfg.batch, n, dtype=torch.int32),
+                    node_parent=torch.empty(cfg.batch, n, dtype=torch.int32),
+                    node_depth=torch.empty(cfg.batch, n, dtype=torch.int32),
+                    node_score=torch.empty(cfg.batch, n, dtype=torch.float32),
+                    mask=torch.empty(cfg.batch, n, n, dtype=torch.uint8),
+                    pos_ids=torch.empty(cfg.batch, n, dtype=torch.int32),
+                    dev_status=torch.empty(cfg.batch, dtype=torch.int32))
+        outs = {k: pin(v) for k, v in outs.items()}
+
+        def host_step():
+            return Bn.tf_draft_tree_host(dims, d, h_hidden, h_root, h_pos, outs["node_tok"], outs["node_parent"],
+                                         outs["node_depth"], outs["node_score"], outs["mask"], outs["pos_ids"],
+                                         outs["dev_status"], dr.ws)
+        for _ in range(3):
+            host_step()
+        barrier(world, dev)
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            host_step()
+        t_e2e = max_over_ranks(time.perf_counter() - t0, world, dev)
+        assert torch.equal(outs["node_tok"], ref["node_tok"].cpu())
+        h2d = sum(t.numel() * t.element_size() for t in (h_hidden, h_root, h_pos))
+        d2h = sum(t.numel() * t.element_size() for t in outs.values())
+        e2e = {"value": cfg.batch * args.e2e_steps * world / t_e2e, "unit": "trees/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    # ---- CPU baseline: the oracle on the host cores (rank 0, N = 1 only)
+    cpu = None
+    if rank == 0 and world == 1 and args.cpu_baseline_s > 0:
+        orc = OracleSample(cfg, inp)
+        _, full_est, _ = orc.run(1 / 64)
+        frac = min(1.0, max(1 / 64, args.cpu_baseline_s / max(full_est, 1e-3)))
+        t, full, Vs = orc.run(frac)
+        cpu = {"value": 1.0 / full, "unit": "trees/s", "cores": cpu_threads(), "kind": "oracle",
+               "sample": f"fp64 numpy oracle, 1 sequence, vocabulary cut to {Vs} of {cfg.V} "
+                         f"({t:.1f} s), LM-head/softmax/sort time scaled to the full V"}
+
+    if rank != 0:
+        return
+    clocks = clk.summary()
+    line = {
+        "metric": METRIC, "value": value, "unit": "trees/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "us_per_tree": ms_per_step * 1e3 / cfg.batch,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,0.02) weights, hidden states scaled to 2-4 nat marginals)",
+        "config": {"workload": cfg.name, "batch": cfg.batch, "d": cfg.d, "V": cfg.V, "I": cfg.I,
+                   "gamma": cfg.gamma, "M": cfg.M, "K2": cfg.K2, "B": cfg.B, "R": cfg.R,
+                   "l2": "no flush: inputs larger than L2 (W_lm 1.245 GB streamed twice per step)",
+                   "parallelism": f"replicas x{world}"},
+        "step_roofline": {"algorithmic_bytes": step_bytes, "achieved_gbs": step_bytes / (ms_per_step / 1e3) / 1e9,
+                          "peak_gbs": peak, "frac": step_bytes / (ms_per_step / 1e3) / 1e9 / peak,
+                          "peak_kind": peak_kind},
+        "roofline": {"bound": "hbm", "kernel": "tc_gemm_kernel<LMHEAD> (stage-1 and stage-2 launches)",
+                     "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                     "traffic": traffic, "peak_kind": peak_kind,
+                     "launch_ms": {"stage1": statistics.mean(lm1), "stage2": statistics.mean(lm2)},
+                     "bytes_per_launch": {"stage1": lm_launch_bytes[0], "stage2": lm_launch_bytes[1]}},
+        "clocks": clocks, "e2e": e2e, "gpu_launches": kernels_per_step * args.steps,
+        "cpu_baseline": cpu, "device_flags": flags,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=WORKLOAD,
+                    help="synthetic workload (synth.CONFIGS); default the measured Qwen3-8B-shape B=64 step")
+    ap.add_argument("--e2e-steps", type=int, default=300)
+    ap.add_argument("--cpu-baseline-s", type=float, default=20.0,
+                    help="approximate seconds of oracle work for the cpu_baseline sample (0 = skip)")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

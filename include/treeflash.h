@@ -218,6 +218,12 @@ tf_status tf_ar_approx(const tf_dims* dims, const tf_weights* w, const void* hid
                        const int32_t* root_tok, const int32_t* top_ids, void* h_prime,
                        void* ws, size_t ws_bytes, tf_stream_t stream);
 
+/* Device address of h' [b, R, d] (dims->dtype) inside a workspace laid out for `dims`: where
+ * tf_ar_approx and tf_stage2_ar_approx leave the approximator's output. Host only; the address
+ * is valid while the workspace is. Lets a caller run tf_lmhead_partials/tf_lmhead_merge on h'
+ * as separate calls without a copy. */
+tf_status tf_workspace_h_prime(const tf_dims* dims, void* ws, size_t ws_bytes, void** h_prime);
+
 #ifdef __cplusplus
 }
 #endif

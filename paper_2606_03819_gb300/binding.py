@@ -45,7 +45,8 @@ class TfWeights(ctypes.Structure):
 
 EXPORTS = ("tf_status_string", "tf_version", "tf_workspace_size", "tf_status_reset", "tf_status_read",
            "tf_stage1_marginals", "tf_stage2_ar_approx", "tf_build_tree", "tf_tree_mask",
-           "tf_draft_tree_host", "tf_lmhead_partials", "tf_lmhead_merge", "tf_ar_approx")
+           "tf_draft_tree_host", "tf_lmhead_partials", "tf_lmhead_merge", "tf_ar_approx",
+           "tf_workspace_h_prime")
 
 _lib = None
 
@@ -75,7 +76,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
         "tf_draft_tree_host": (ctypes.c_int, [D, W, P, P, P, P, P, P, P, P, P, P, P, SZ, P]),
         "tf_lmhead_partials": (ctypes.c_int, [D, P, P, I32, P, SZ, P]),
         "tf_lmhead_merge": (ctypes.c_int, [D, P, P, I32, I32, P, P, P, SZ, P]),
-        "tf_ar_approx": (ctypes.c_int, [D, W, P, P, P, P, P, P, SZ, P]),
+        "tf_ar_approx": (ctypes.c_int, [D, W, P, P, P, P, P, SZ, P]),
+        "tf_workspace_h_prime": (ctypes.c_int, [D, P, SZ, ctypes.POINTER(P)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -233,3 +235,14 @@ def tf_ar_approx(dims: Dims, w: dict, hidden, root_tok, top_ids, h_prime, ws, st
     _check("tf_ar_approx", load_library().tf_ar_approx(
         ctypes.byref(dims.c()), ctypes.byref(weights_struct(w)), _ptr(hidden), _ptr(root_tok), _ptr(top_ids),
         _ptr(h_prime), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def tf_workspace_h_prime(dims: Dims, ws) -> torch.Tensor:
+    """h' [b, R, d] as a tensor view of the workspace (no copy)."""
+    p = ctypes.c_void_p()
+    _check("tf_workspace_h_prime", load_library().tf_workspace_h_prime(
+        ctypes.byref(dims.c()), _ptr(ws), ws.numel(), ctypes.byref(p)))
+    off = p.value - ws.data_ptr()
+    esize = 2 if dims.dtype == "bf16" else 4
+    n = dims.batch * dims.R * dims.d * esize
+    return ws[off:off + n].view(dims.torch_dtype).view(dims.batch, dims.R, dims.d)

@@ -327,6 +327,17 @@ tf_status tf_tree_mask(const tf_dims* dims, const int32_t* node_parent, const in
     return cuda_status(launch_tree_mask(ctx, D.b, D.B, node_parent, node_depth, root_pos, mask, pos_ids));
 }
 
+tf_status tf_workspace_h_prime(const tf_dims* dims, void* ws, size_t ws_bytes, void** h_prime) {
+    if (!h_prime) return TF_ERR_INVALID_ARG;
+    Dims D;
+    TF_TRY(check_dims(dims, &D));
+    if (D.mode != TF_MODE_AR) return TF_ERR_INVALID_ARG;
+    const Layout L = layout(D);
+    TF_TRY(check_ws(L, ws, ws_bytes));
+    *h_prime = at<void>(ws, L.hp);
+    return TF_OK;
+}
+
 tf_status tf_draft_tree_host(const tf_dims* dims, const tf_weights* w, const void* hidden, const int32_t* root_tok,
                              const int32_t* root_pos, int32_t* node_tok, int32_t* node_parent, int32_t* node_depth,
                              float* node_score, uint8_t* mask, int32_t* pos_ids, int32_t* dev_status, void* ws,

@@ -27,12 +27,15 @@ import synth
 from oracle import treeflash_oracle as O
 
 TOLS = {
-    # lp: stage-1 log-probs vs the plain fp64 oracle; lp2: stage-2 log-probs vs the plain oracle
-    # (the bf16 path rounds x, SiLU(G)*U and h' to bf16 before the next GEMM, see the design
-    # notes for the bound); lp_emul: everything vs the oracle that rounds at those points;
-    # sel: selection margin above which the tree structure must match exactly.
+    # lp: stage-1 log-probs vs the plain fp64 oracle; lp2: stage-2 log-probs vs the plain oracle,
+    # on top of the oracle's own emulated-minus-plain difference (the bf16 path rounds x,
+    # SiLU(G)*U and h' to bf16 before the next GEMM); lp_emul: everything vs the oracle that
+    # rounds at those points (the
+    # remaining difference is fp32-vs-fp64 accumulation flipping a bf16 rounding, worth up to
+    # |w| * ulp(h') per flipped element); sel: selection margin above which the tree structure
+    # must match exactly (twice the per-log-prob tolerance).
     "f32": dict(lp=1e-4, lp2=1e-4, lp_emul=1e-4, sel=1e-3),
-    "bf16": dict(lp=2e-2, lp2=6e-2, lp_emul=5e-3, sel=2e-2),
+    "bf16": dict(lp=2e-2, lp2=2e-2, lp_emul=2e-2, sel=4e-2),
 }
 
 
@@ -84,8 +87,12 @@ def _check_row(gpu_ids, gpu_lp, full_lp, tol, what):
     return max(err_id, err_rank)
 
 
-def compare(cfg, gpu, orc, tol_lp, tol_sel, check_structure=True, tol_lp2=None):
-    """Assert parity of one batch; returns a small report dict."""
+def compare(cfg, gpu, orc, tol_lp, tol_sel, check_structure=True, tol_lp2=None, orc_round=None):
+    """Assert parity of one batch; returns a small report dict.
+
+    orc_round: the bf16-emulating oracle's results for the same sequences. When given, every
+    stage-2 row may additionally deviate by the oracle's own emulated-minus-plain difference at
+    the reported ids (|gpu - plain| <= |gpu - emulated| + |emulated - plain|)."""
     tol_lp2 = tol_lp if tol_lp2 is None else tol_lp2
     rep = dict(max_err_s1=0.0, max_err_s2=0.0, max_err_score=0.0, rows_s2=0, rows_s2_skipped=0,
                exact_trees=0, set_trees=0, valid_only_trees=0)
@@ -103,12 +110,24 @@ def compare(cfg, gpu, orc, tol_lp, tol_sel, check_structure=True, tol_lp2=None):
             hid, prev = O.stage2_conditioning(g, M, int(o.tree.tok[0]), o.top_ids)
             okey = {(int(h), int(p)): r for r, (h, p) in enumerate(zip(hid, prev))}
             ghid, gprev = O.stage2_conditioning(g, M, int(o.tree.tok[0]), gpu["top_ids"][s])
+            if orc_round is not None:
+                ehid, eprev = O.stage2_conditioning(g, M, int(o.tree.tok[0]), orc_round[s].top_ids)
+                ekey = {(int(h), int(p)): r for r, (h, p) in enumerate(zip(ehid, eprev))}
             for r, (h, p) in enumerate(zip(ghid, gprev)):
                 orow = okey.get((int(h), int(p)))
                 if orow is None:
                     rep["rows_s2_skipped"] += 1
                     continue
-                e = _check_row(gpu["child_ids"][s, r], gpu["child_logp"][s, r], o.s2_logp[orow], tol_lp2,
+                tol_row = tol_lp2
+                if orc_round is not None:
+                    erow = ekey.get((int(h), int(p)))
+                    if erow is None:
+                        rep["rows_s2_skipped"] += 1
+                        continue
+                    ids = gpu["child_ids"][s, r]
+                    tol_row = tol_lp2 + float(np.abs(orc_round[s].s2_logp[erow][ids] - o.s2_logp[orow][ids]).max())
+                    rep["max_round_allowance"] = max(rep.get("max_round_allowance", 0.0), tol_row - tol_lp2)
+                e = _check_row(gpu["child_ids"][s, r], gpu["child_logp"][s, r], o.s2_logp[orow], tol_row,
                                f"seq {s} stage-2 row {r}")
                 rep["max_err_s2"] = max(rep["max_err_s2"], e)
                 rep["rows_s2"] += 1

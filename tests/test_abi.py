@@ -101,3 +101,20 @@ def test_product_path_never_imports_the_oracle():
             if f.endswith((".py", ".cu", ".cuh", ".h", ".cpp")):
                 txt = open(os.path.join(dirpath, f)).read()
                 assert "oracle" not in txt.lower(), f
+
+
+def _header_arity():
+    src = open(os.path.join(ROOT, "include", "treeflash.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    out = {}
+    for m in re.finditer(r"\b(tf_[a-z0-9_]+)\s*\(([^)]*)\)\s*;", src):
+        args = m.group(2).strip()
+        out[m.group(1)] = 0 if args in ("", "void") else args.count(",") + 1
+    return out
+
+
+def test_binding_signatures_match_header_arity(lib):
+    arity = _header_arity()
+    assert set(arity) == set(declared_functions())
+    for name, n in arity.items():
+        assert len(getattr(lib, name).argtypes) == n, name

@@ -1,9 +1,10 @@
 """GPU parity: the CUDA path through the C ABI against the fp64 oracle on the same seeded inputs.
 
 Tolerances (tests/parity.py): fp32 inputs 1e-4 absolute on log-probabilities; bf16 inputs with
-fp32 accumulation 2e-2 absolute against the plain fp64 oracle and 5e-3 against the oracle that
-rounds to bf16 where the CUDA path stores bf16. Tree structure is compared bit-exactly wherever
-the oracle's selection margin exceeds 1e-3 (fp32) / 2e-2 (bf16).
+fp32 accumulation 2e-2 absolute against the oracle that rounds to bf16 where the CUDA path stores
+bf16; against the plain fp64 oracle 2e-2 for stage 1, and for stage 2 (whose input h' went
+through three bf16 roundings) 2e-2 plus the oracle's own emulated-minus-plain difference. Tree structure is compared bit-exactly wherever the oracle's
+selection margin exceeds 1e-3 (fp32) / 4e-2 (bf16).
 """
 import numpy as np
 import pytest
@@ -39,11 +40,12 @@ def check(cfg, emulate_also=True, inp=None, orc_seqs=None):
     sub = {k: (v[seqs] if isinstance(v, np.ndarray) and v.ndim >= 1 and v.shape[0] == cfg.batch else v)
            for k, v in gpu.items()}
     orc = parity.run_oracle(cfg, inp, emulate_bf16=False, seqs=seqs, W=W)
-    reps["pure"] = parity.compare(cfg, sub, orc, tol["lp"], tol["sel"],
-                                  check_structure=cfg.dtype == "f32", tol_lp2=tol["lp2"])
-    if cfg.dtype == "bf16" and emulate_also:
-        orc_e = parity.run_oracle(cfg, inp, emulate_bf16=True, seqs=seqs, W=W)
-        reps["emul"] = parity.compare(cfg, sub, orc_e, tol["lp_emul"], tol["sel"])
+    orc_e = parity.run_oracle(cfg, inp, emulate_bf16=True, seqs=seqs, W=W) if cfg.dtype == "bf16" else None
+    if orc_e is not None:
+        reps["emul"] = parity.compare(cfg, sub, orc_e, tol["lp_emul"], tol["sel"],
+                                      check_structure=emulate_also)
+    reps["pure"] = parity.compare(cfg, sub, orc, tol["lp"], tol["sel"], check_structure=cfg.dtype == "f32",
+                                  tol_lp2=tol["lp2"], orc_round=orc_e)
     assert not (gpu["flags"] & ~16), f"device flags {gpu['flags']}"
     return gpu, reps
 
