@@ -28,7 +28,7 @@ struct Dims {
 };
 
 struct Layout {
-    size_t status, partials, X, A, hp;
+    size_t status, partials, X, A, hp, kpart;
     size_t h_hidden, h_root, h_pos, top_ids, top_logp, child_ids, child_logp;
     size_t n_tok, n_par, n_dep, n_score, n_mask, n_pos, n_stat;
     size_t total;
@@ -91,6 +91,10 @@ Layout layout(const Dims& D) {
     L.X = take(rows2 * 2 * D.d * D.esize);
     L.A = take(rows2 * D.I * D.esize);
     L.hp = take(rows2 * D.d * D.esize);
+    // split-K partial sums of the bf16 approximator GEMMs: [k_splits][rows][max(2I, d)] fp32
+    L.kpart = D.dtype == TF_BF16 ? take(static_cast<size_t>(kMaxKSplits) * rows2 *
+                                        (2 * static_cast<size_t>(D.I) > static_cast<size_t>(D.d) ? 2 * D.I : D.d) * 4)
+                                 : take(0);
     L.h_hidden = take(rows1 * D.d * D.esize);
     L.h_root = take(D.b * sizeof(int32_t));
     L.h_pos = take(D.b * sizeof(int32_t));
@@ -168,7 +172,7 @@ tf_status do_ar_approx(const Ctx& ctx, const Dims& D, const Layout& L, void* ws,
     const int rows = D.b * D.R;
     if (D.dtype == TF_BF16)
         return cuda_status(launch_swiglu_tc(ctx, X, w->w_gate, w->w_up, w->w_down, hidden, rows, D.d, D.I, D.R, D.M,
-                                            D.gamma, A, hp));
+                                            D.gamma, A, hp, at<float>(ws, L.kpart)));
     return cuda_status(launch_swiglu_simt(ctx, X, w->w_gate, w->w_up, w->w_down, hidden, rows, D.d, D.I, D.R, D.M,
                                           D.gamma, A, hp));
 }

@@ -17,6 +17,7 @@ constexpr int kMaxM = 32;           // largest M (the builder tests membership w
 constexpr int kMaxB = 1023;         // largest draft budget
 constexpr int kMaxGamma = 64;
 constexpr int kMergeExpandLists = 8;  // lists a merge may recompute exactly (>= (kMaxK-1)/8 + 1)
+constexpr int kMaxKSplits = 4;        // split-K factor of the approximator GEMMs (workspace sized for it)
 
 // Per (row, vocabulary block) summary written by the LM-head pass: the block's max logit m,
 // sum_v exp(z_v - m), and its kListLen largest logits in (value desc, id asc) order; unused
@@ -95,7 +96,13 @@ cudaError_t launch_gather_norm(const Ctx&, int dtype, const void* hidden, const 
                                int V, float eps, void* X);
 cudaError_t launch_swiglu_tc(const Ctx&, const void* X, const void* w_gate, const void* w_up,
                              const void* w_down, const void* hidden, int n_rows, int d, int I,
-                             int R, int M, int gamma, void* A, void* h_prime);
+                             int R, int M, int gamma, void* A, void* h_prime, float* partial);
+// split-K reductions of the approximator GEMMs (partial sums in fp32, [k_splits][rows][N])
+cudaError_t launch_swiglu_reduce(const Ctx&, const float* partial, int k_splits, int n_rows, int I,
+                                 __nv_bfloat16* A);
+cudaError_t launch_down_reduce(const Ctx&, const float* partial, int k_splits, int n_rows, int d,
+                               const __nv_bfloat16* hidden, int R, int M, int gamma,
+                               __nv_bfloat16* h_prime);
 cudaError_t launch_swiglu_simt(const Ctx&, const void* X, const void* w_gate, const void* w_up,
                                const void* w_down, const void* hidden, int n_rows, int d, int I,
                                int R, int M, int gamma, void* A, void* h_prime);

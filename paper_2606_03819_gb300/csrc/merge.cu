@@ -4,8 +4,9 @@
 // One CTA per row. Inputs are the row's per-block summaries (max, sum of exp, 8 largest). The
 // CTA
 //   1. combines the block (max, sum) pairs into the row's log-sum-exp;
-//   2. finds the k-th largest candidate key (value desc, id asc) among all kept entries with an
-//      8-pass radix select over 64-bit keys;
+//   2. keeps as candidates the entries at or above the k-th largest block maximum (at least k
+//      keys lie there, so the top k do too) and finds the k-th largest candidate key (value
+//      desc, id asc) with an 8-pass radix select over 64-bit keys;
 //   3. certifies the result: a block whose list is full (8 entries) and whose smallest kept
 //      entry still beats the k-th key may hide further members of the top-k. Such blocks
 //      (at most (k-1)/8 of them, since their 8 entries all lie in the top k-1) get their 256
@@ -95,19 +96,37 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(const Partial* _
                                                                 const T* __restrict__ lm_head,
                                                                 const T* __restrict__ x, int32_t* __restrict__ out_ids,
                                                                 float* __restrict__ out_logp, int* status) {
-    extern __shared__ unsigned long long keys[];  // n_tiles * 8 + kMergeExpandLists * kMaxK
+    // dynamic shared memory: the row's block summaries, then candidate keys
+    extern __shared__ __align__(16) uint8_t dsm[];
+    Partial* P = reinterpret_cast<Partial*>(dsm);
+    const int n_base = n_tiles * kListLen;
+    const int cap = n_base + kMergeExpandLists * kMaxK;
+    unsigned long long* cand = reinterpret_cast<unsigned long long*>(dsm + static_cast<size_t>(n_tiles) * sizeof(Partial));
+    unsigned long long* lmax = cand + cap;       // per-block best key
+    uint8_t* expanded = reinterpret_cast<uint8_t*>(lmax + n_tiles);
     __shared__ int hist[256];
     __shared__ float red_m[kThreads / 32], red_s[kThreads / 32];
-    __shared__ int sel_digit, sel_rem, n_flag, flag_list[kMergeExpandLists + 1], n_sel;
+    __shared__ int sel_digit, sel_rem, n_flag, flag_list[kMergeExpandLists + 1], n_cand, n_sel, n_valid;
     __shared__ unsigned long long sel[kMaxK];
     __shared__ float zbuf[kBlockV];
     __shared__ float lse_s;
 
     const int row = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const Partial* P = partials + static_cast<size_t>(row) * n_tiles;
-    const int n_base = n_tiles * kListLen;
-    uint8_t* expanded = reinterpret_cast<uint8_t*>(keys + n_base + kMergeExpandLists * kMaxK);
+
+    // 0. stage the row's summaries (contiguous, 72 B = 9 x 8 B each) with 8-byte loads; a row
+    //    starts on an 8-byte boundary for any n_tiles (16 only when n_tiles is even)
+    {
+        const uint2* src = reinterpret_cast<const uint2*>(partials + static_cast<size_t>(row) * n_tiles);
+        uint2* dst = reinterpret_cast<uint2*>(P);
+        const int n8 = n_tiles * static_cast<int>(sizeof(Partial) / 8);
+        for (int i = tid; i < n8; i += kThreads) dst[i] = src[i];
+    }
+    if (tid == 0) {
+        n_cand = 0;
+        n_valid = 0;
+    }
+    __syncthreads();
 
     // 1. log-sum-exp over blocks
     float m = -INFINITY, s = 0.0f;
@@ -122,14 +141,15 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(const Partial* _
         red_m[warp] = m;
         red_s[warp] = s;
     }
-    // 2. candidate keys (0 marks an empty slot; every real key is larger)
-    for (int i = tid; i < n_base; i += kThreads) {
-        const int t = i / kListLen, j = i % kListLen;
-        const int id = P[t].id[j];
-        keys[i] = id >= 0 ? cand_key(P[t].v[j], id) : 0ull;
+    // per-block best keys (0 = empty block)
+    int my_valid = 0;
+    for (int t = tid; t < n_tiles; t += kThreads) {
+        const int id = P[t].id[0];
+        lmax[t] = id >= 0 ? cand_key(P[t].v[0], id) : 0ull;
+        expanded[t] = 0;
+        my_valid += id >= 0 ? 1 : 0;
     }
-    for (int i = tid; i < kMergeExpandLists * kMaxK; i += kThreads) keys[n_base + i] = 0ull;
-    for (int t = tid; t < n_tiles; t += kThreads) expanded[t] = 0;
+    atomicAdd(&n_valid, my_valid);
     __syncthreads();
     if (tid == 0) {
         float M = -INFINITY, S = 0.0f;
@@ -139,18 +159,33 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(const Partial* _
         if (!isfinite(lse)) set_status(status, TF_DEV_NONFINITE);
     }
 
+    // 2. candidates: every kept entry at or above the k-th largest block maximum. At least k
+    //    keys are >= that bound (the k block maxima), so the top k are all among them.
+    const unsigned long long theta0 =
+        n_valid >= k ? block_kth_largest(lmax, n_tiles, k, hist, &sel_digit, &sel_rem) : 0ull;
+    for (int t = tid; t < n_tiles; t += kThreads) {
+        for (int j = 0; j < kListLen; ++j) {
+            const int id = P[t].id[j];
+            if (id < 0) break;
+            const unsigned long long key = cand_key(P[t].v[j], id);
+            if (key < theta0) break;            // lists are sorted: the rest is smaller
+            cand[atomicAdd(&n_cand, 1)] = key;
+        }
+    }
+    __syncthreads();
+
     // 3. select, certify, recompute flagged blocks, repeat
-    int n_keys = n_base + kMergeExpandLists * kMaxK;
     int n_expanded = 0;
     unsigned long long theta = 0;
-    for (int round = 0;; ++round) {
-        theta = block_kth_largest(keys, n_keys, k, hist, &sel_digit, &sel_rem);
+    for (;;) {
+        const int nc = n_cand;
+        theta = nc >= k ? block_kth_largest(cand, nc, k, hist, &sel_digit, &sel_rem) : 0ull;
         if (tid == 0) n_flag = 0;
         __syncthreads();
         for (int t = tid; t < n_tiles; t += kThreads) {
-            if (expanded[t]) continue;
-            const unsigned long long last = keys[t * kListLen + kListLen - 1];
-            if (last != 0ull && last > theta) {
+            if (expanded[t] || P[t].id[kListLen - 1] < 0) continue;
+            const unsigned long long last = cand_key(P[t].v[kListLen - 1], P[t].id[kListLen - 1]);
+            if (last > theta) {
                 const int slot = atomicAdd(&n_flag, 1);
                 if (slot < kMergeExpandLists + 1) flag_list[slot] = t;
             }
@@ -179,14 +214,18 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(const Partial* _
                 if (lane == 0) zbuf[c] = acc * inv_temp;
             }
             __syncthreads();
-            unsigned long long* dst = keys + n_base + (n_expanded + f) * kMaxK;
+            // the block's old (truncated) entries leave the candidate set
+            for (int i = tid; i < n_cand; i += kThreads) {
+                const int id = key_id(cand[i]);
+                if (id >= v0 && id < v0 + cols) cand[i] = 0ull;
+            }
+            __syncthreads();
             for (int c = tid; c < cols; c += kThreads) {
                 const unsigned long long kc = cand_key(zbuf[c], v0 + c);
                 int rank = 0;
                 for (int j = 0; j < cols; ++j) rank += cand_key(zbuf[j], v0 + j) > kc ? 1 : 0;
-                if (rank < kMaxK) dst[rank] = kc;
+                if (rank < k) cand[atomicAdd(&n_cand, 1)] = kc;
             }
-            for (int i = tid; i < kListLen; i += kThreads) keys[t * kListLen + i] = 0ull;
             if (tid == 0) expanded[t] = 1;
             __syncthreads();
         }
@@ -196,8 +235,9 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(const Partial* _
     // 4. the k winners, sorted
     if (tid == 0) n_sel = 0;
     __syncthreads();
-    for (int i = tid; i < n_keys; i += kThreads) {
-        const unsigned long long key = keys[i];
+    const int nc = n_cand;
+    for (int i = tid; i < nc; i += kThreads) {
+        const unsigned long long key = cand[i];
         if (key != 0ull && key >= theta) {
             const int slot = atomicAdd(&n_sel, 1);
             if (slot < kMaxK) sel[slot] = key;
@@ -206,8 +246,7 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(const Partial* _
     __syncthreads();
     const int ns = min(n_sel, k);
     const float lse = lse_s;
-    for (int i = tid; i < k; i += kThreads) {
-        if (i >= ns) continue;
+    for (int i = tid; i < ns; i += kThreads) {
         const unsigned long long key = sel[i];
         int rank = 0;
         for (int j = 0; j < ns; ++j) rank += sel[j] > key ? 1 : 0;
@@ -224,7 +263,8 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(const Partial* _
 }  // namespace
 
 size_t merge_smem_bytes(int n_tiles) {
-    return static_cast<size_t>(n_tiles * kListLen + kMergeExpandLists * kMaxK) * sizeof(unsigned long long) +
+    return static_cast<size_t>(n_tiles) * sizeof(Partial) +
+           static_cast<size_t>(n_tiles * kListLen + kMergeExpandLists * kMaxK + n_tiles) * sizeof(unsigned long long) +
            static_cast<size_t>(n_tiles + 15) / 16 * 16;
 }
 

@@ -34,7 +34,7 @@ constexpr int kBM = 128;      // activation rows per M-tile (TMEM lanes)
 constexpr int kThreads = 320;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
-enum { EPI_LMHEAD = 0, EPI_GATEUP = 1, EPI_DOWN = 2 };
+enum { EPI_LMHEAD = 0, EPI_GATEUP = 1, EPI_DOWN = 2, EPI_PARTIAL = 3 };
 
 struct EpiParams {
     Partial* partials;           // LMHEAD: [n_rows, n_tiles]
@@ -44,7 +44,25 @@ struct EpiParams {
     int ld_out;
     const __nv_bfloat16* hidden; // DOWN: residual rows, [b * gamma, ld_out]
     int R, M, gamma;
+    float* partial;              // PARTIAL: fp32 [k_splits][n_rows][ld_partial], accumulator nb at
+    int ld_partial;              //          columns nb * n_total + n
+    size_t partial_split_stride; // elements between consecutive k-splits
+    int n_total;                 // N of the whole GEMM (n_ntiles * BN)
 };
+
+// Work unit u -> (N tile, M-tile group, K split); consecutive units share the N tile and K split
+// (the same weight tile) and differ in the M-tile group, so batched rows reuse it from L2.
+struct Unit {
+    int nt, mg, kx;
+};
+__device__ __forceinline__ Unit decode_unit(int u, int n_mgroups, int k_splits) {
+    Unit w;
+    w.mg = u % n_mgroups;
+    const int rest = u / n_mgroups;
+    w.kx = rest % k_splits;
+    w.nt = rest / k_splits;
+    return w;
+}
 
 template <int MT, int NB, int BN, int STAGES>
 struct TileCfg {
@@ -65,11 +83,75 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Running (max, sum of exp) and sorted top-kListLen of one row, fed 32 logits at a time.
+struct RowTop {
+    float m, s;
+    float tv[kListLen];
+    int ti[kListLen];
+};
+
+// Insert x (known to beat tv[kListLen-1]) into the descending list. Every position is computed
+// from the old list at once (no chain of swaps): new[t] = old[t-1] if x beats old[t-1], else x
+// if x beats old[t], else old[t]. Equal values keep the earlier (smaller) id first.
+__device__ __forceinline__ void top_insert(RowTop& rt, float x, int id) {
+    bool gt[kListLen];
+#pragma unroll
+    for (int t = 0; t < kListLen; ++t) gt[t] = x > rt.tv[t];
+    float nv[kListLen];
+    int ni[kListLen];
+    nv[0] = gt[0] ? x : rt.tv[0];
+    ni[0] = gt[0] ? id : rt.ti[0];
+#pragma unroll
+    for (int t = 1; t < kListLen; ++t) {
+        nv[t] = gt[t - 1] ? rt.tv[t - 1] : (gt[t] ? x : rt.tv[t]);
+        ni[t] = gt[t - 1] ? rt.ti[t - 1] : (gt[t] ? id : rt.ti[t]);
+    }
+#pragma unroll
+    for (int t = 0; t < kListLen; ++t) {
+        rt.tv[t] = nv[t];
+        rt.ti[t] = ni[t];
+    }
+}
+
+// One 32-column chunk of accumulators (logits of vocabulary ids v0 .. v0+31 for this row).
+// Max and sum use trees, not serial chains, so the 32 values proceed in parallel.
+__device__ __forceinline__ void lmhead_chunk(RowTop& rt, const uint32_t (&r)[32], int v0, int V, float inv_temp) {
+    float v[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = (v0 + j < V) ? __uint_as_float(r[j]) * inv_temp : -INFINITY;
+    float t[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) t[j] = fmaxf(v[2 * j], v[2 * j + 1]);
+#pragma unroll
+    for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+        for (int j = 0; j < w; ++j) t[j] = fmaxf(t[j], t[j + w]);
+    const float cmax = t[0];
+    const float mn = fmaxf(rt.m, cmax);
+    if (mn > -INFINITY) {
+        float e[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) e[j] = __expf(v[2 * j] - mn) + __expf(v[2 * j + 1] - mn);
+#pragma unroll
+        for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+            for (int j = 0; j < w; ++j) e[j] += e[j + w];
+        rt.s = rt.s * __expf(rt.m - mn) + e[0];
+        rt.m = mn;
+    }
+    if (cmax > rt.tv[kListLen - 1]) {
+        // ids grow with j, so a strict > keeps the smaller id first among equal values
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (v[j] > rt.tv[kListLen - 1]) top_insert(rt, v[j], v0 + j);
+    }
+}
+
 template <int EPI, int MT, int NB, int BN, int STAGES>
 __global__ void __launch_bounds__(kThreads, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_w0,
                const __grid_constant__ CUtensorMap tmap_w1, int n_rows, int K, int n_ntiles,
-               int n_mgroups, int w_stream_once, EpiParams ep, int* status) {
+               int n_mgroups, int k_splits, int w_stream_once, EpiParams ep, int* status) {
     using C = TileCfg<MT, NB, BN, STAGES>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -84,8 +166,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int n_units = n_ntiles * n_mgroups;
-    const int nk = K / kBK;
+    const int n_units = n_ntiles * n_mgroups * k_splits;
+    const int nk = K / kBK / k_splits;      // K-steps per unit (K % (64 * k_splits) == 0)
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -123,8 +205,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             uint32_t last_parity[STAGES > 0 ? STAGES : 1];
             bool ok = true;
             for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
-                const int nt = u / n_mgroups, mg = u % n_mgroups;
-                for (int kb = 0; kb < nk; ++kb) {
+                const Unit w = decode_unit(u, n_mgroups, k_splits);
+                const int nt = w.nt, mg = w.mg;
+                for (int kb = w.kx * nk; kb < (w.kx + 1) * nk; ++kb) {
                     if (!ptx::mbar_wait(&empty[stage], phase ^ 1u, abort_flag, kWaitLimitNs)) {
                         ok = false;
                         break;
@@ -171,7 +254,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                     ok = ptx::mbar_wait(&tempty[g0 + j], (use[g0 + j] & 1u) ^ 1u, abort_flag, kWaitLimitNs);
                 if (!ok) break;
                 ptx::tc_fence_after();
-                for (int kb = 0; kb < nk; ++kb) {
+                for (int kb = 0; kb < nk; ++kb) {     // position inside the unit's K range
                     if (!ptx::mbar_wait(&full[stage], phase, abort_flag, kWaitLimitNs)) {
                         ok = false;
                         break;
@@ -228,53 +311,38 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             }
             ++use;
             ptx::tc_fence_after();
-            const int nt = u / n_mgroups, mg = u % n_mgroups;
+            const Unit w = decode_unit(u, n_mgroups, k_splits);
+            const int nt = w.nt, mg = w.mg;
             const int row = (mg * MT + (MT == 2 ? g : 0)) * kBM + q * 32 + lane;
             const uint32_t tb = tmem_base + 256u * g + (static_cast<uint32_t>(q * 32) << 16);
 
             if constexpr (EPI == EPI_LMHEAD) {
-                float m = -INFINITY, s = 0.0f;
-                float tv[kListLen];
-                int ti[kListLen];
+                RowTop rt;
+                rt.m = -INFINITY;
+                rt.s = 0.0f;
 #pragma unroll
                 for (int j = 0; j < kListLen; ++j) {
-                    tv[j] = -INFINITY;
-                    ti[j] = -1;
+                    rt.tv[j] = -INFINITY;
+                    rt.ti[j] = -1;
                 }
+                // warps whose 32 rows are all padding skip the accumulators entirely
+                if (row - lane < n_rows) {
+                    static_assert(BN % 64 == 0, "the LM-head epilogue walks 64 columns per step");
+                    uint32_t ra[32], rb[32];
+                    ptx::tmem_ld_32cols_nowait(tb, ra);
+                    ptx::tmem_wait_ld_regs(ra);
 #pragma unroll 1
-                for (int c = 0; c < BN; c += 32) {
-                    uint32_t r[32];
-                    ptx::tmem_ld_32cols(tb + c, r);
-                    const int v0 = nt * BN + c;
-                    float z[32];
-                    float cmax = -INFINITY;
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        z[j] = (v0 + j < ep.V) ? __uint_as_float(r[j]) * ep.inv_temp : -INFINITY;
-                        cmax = fmaxf(cmax, z[j]);
-                    }
-                    if (cmax > m) {
-                        s *= __expf(m - cmax);
-                        m = cmax;
-                    }
-                    if (cmax > -INFINITY) {
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) s += __expf(z[j] - m);
-                    }
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        // ids arrive in increasing order, so a strict > keeps the smaller id first
-                        if (z[j] > tv[kListLen - 1]) {
-                            tv[kListLen - 1] = z[j];
-                            ti[kListLen - 1] = v0 + j;
-#pragma unroll
-                            for (int t = kListLen - 1; t > 0; --t) {
-                                if (tv[t] > tv[t - 1]) {
-                                    const float fv = tv[t]; tv[t] = tv[t - 1]; tv[t - 1] = fv;
-                                    const int iv = ti[t]; ti[t] = ti[t - 1]; ti[t - 1] = iv;
-                                }
-                            }
-                        }
+                    for (int c = 0; c < BN; c += 64) {
+                        // each TMEM load is in flight while the previous 32 columns are processed;
+                        // the warp reconverges before every warp-collective tcgen05 instruction
+                        ptx::tmem_ld_32cols_nowait(tb + c + 32, rb);
+                        lmhead_chunk(rt, ra, nt * BN + c, ep.V, ep.inv_temp);
+                        __syncwarp();
+                        ptx::tmem_wait_ld_regs(rb);
+                        if (c + 64 < BN) ptx::tmem_ld_32cols_nowait(tb + c + 64, ra);
+                        lmhead_chunk(rt, rb, nt * BN + c + 32, ep.V, ep.inv_temp);
+                        __syncwarp();
+                        if (c + 64 < BN) ptx::tmem_wait_ld_regs(ra);
                     }
                 }
                 ptx::tc_fence_before();
@@ -282,13 +350,32 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 if (row < n_rows) {
                     Partial* p = ep.partials + static_cast<size_t>(row) * n_ntiles + nt;
                     float2* pf = reinterpret_cast<float2*>(p);
-                    pf[0] = make_float2(m, s);
+                    pf[0] = make_float2(rt.m, rt.s);
 #pragma unroll
-                    for (int j = 0; j < kListLen; j += 2) pf[1 + j / 2] = make_float2(tv[j], tv[j + 1]);
+                    for (int j = 0; j < kListLen; j += 2) pf[1 + j / 2] = make_float2(rt.tv[j], rt.tv[j + 1]);
                     int2* pi = reinterpret_cast<int2*>(p->id);
 #pragma unroll
-                    for (int j = 0; j < kListLen; j += 2) pi[j / 2] = make_int2(ti[j], ti[j + 1]);
+                    for (int j = 0; j < kListLen; j += 2) pi[j / 2] = make_int2(rt.ti[j], rt.ti[j + 1]);
                 }
+            } else if constexpr (EPI == EPI_PARTIAL) {
+                float* base = ep.partial + w.kx * ep.partial_split_stride + static_cast<size_t>(row) * ep.ld_partial;
+#pragma unroll 1
+                for (int nb = 0; nb < NB; ++nb) {
+#pragma unroll 1
+                    for (int c = 0; c < BN; c += 32) {
+                        uint32_t ra[32];
+                        ptx::tmem_ld_32cols(tb + nb * BN + c, ra);
+                        if (row < n_rows) {
+                            float4* dst = reinterpret_cast<float4*>(base + nb * ep.n_total + nt * BN + c);
+#pragma unroll
+                            for (int j = 0; j < 8; ++j)
+                                dst[j] = make_float4(__uint_as_float(ra[4 * j]), __uint_as_float(ra[4 * j + 1]),
+                                                     __uint_as_float(ra[4 * j + 2]), __uint_as_float(ra[4 * j + 3]));
+                        }
+                    }
+                }
+                ptx::tc_fence_before();
+                ptx::mbar_arrive(&tempty[g]);
             } else if constexpr (EPI == EPI_GATEUP) {
 #pragma unroll 1
                 for (int c = 0; c < BN; c += 32) {
@@ -392,16 +479,16 @@ cudaError_t make_tmap(CUtensorMap* map, const void* base, uint64_t inner, uint64
 
 template <int EPI, int MT, int NB, int BN, int STAGES>
 cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& tw0, const CUtensorMap& tw1,
-                     int n_rows, int K, int n_ntiles, int n_mgroups, const EpiParams& ep) {
+                     int n_rows, int K, int n_ntiles, int n_mgroups, const EpiParams& ep, int k_splits = 1) {
     using C = TileCfg<MT, NB, BN, STAGES>;
     auto kern = tc_gemm_kernel<EPI, MT, NB, BN, STAGES>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (e != cudaSuccess) return e;
-    const int n_units = n_ntiles * n_mgroups;
+    const int n_units = n_ntiles * n_mgroups * k_splits;
     const int grid = n_units < ctx.num_sms ? n_units : ctx.num_sms;
     const int stream_once = n_mgroups == 1 ? 1 : 0;
-    kern<<<grid, kThreads, C::kSmemBytes, ctx.stream>>>(tx, tw0, tw1, n_rows, K, n_ntiles, n_mgroups, stream_once,
-                                                       ep, ctx.status);
+    kern<<<grid, kThreads, C::kSmemBytes, ctx.stream>>>(tx, tw0, tw1, n_rows, K, n_ntiles, n_mgroups, k_splits,
+                                                       stream_once, ep, ctx.status);
     return cudaGetLastError();
 }
 
@@ -425,27 +512,63 @@ cudaError_t launch_lmhead_tc(const Ctx& ctx, const void* lm_head, const void* x,
     return run_gemm<EPI_LMHEAD, 2, 1, kBlockV, 3>(ctx, tx, tw, tw, n_rows, d, n_tiles, (m_tiles + 1) / 2, ep);
 }
 
+// Split-K factor for a GEMM with `base_units` (N tiles x M-tile groups) and nk K-steps: enough
+// units to cover the SMs, at most kMaxKSplits, and a divisor of nk.
+int choose_k_splits(int base_units, int nk, int num_sms) {
+    int ks = base_units >= num_sms ? 1 : num_sms / base_units;
+    if (ks > kMaxKSplits) ks = kMaxKSplits;
+    while (ks > 1 && nk % ks != 0) --ks;
+    return ks < 1 ? 1 : ks;
+}
+
 cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, const void* w_gate, const void* w_up,
                              const void* w_down, const void* hidden, int n_rows, int d, int I, int R, int M,
-                             int gamma, void* A, void* h_prime) {
+                             int gamma, void* A, void* h_prime, float* partial) {
     if (n_rows <= 0) return cudaSuccess;
-    constexpr int BN = 64;
+    constexpr int BN = 128;
     const int m_tiles = (n_rows + kBM - 1) / kBM;
+    const int n_mg = m_tiles == 1 ? 1 : (m_tiles + 1) / 2;
+    const int bn_gu = I % BN == 0 ? BN : 64;
+    const int bn_d = d % BN == 0 ? BN : 64;
     CUtensorMap tx, tg, tu, ta, td;
     cudaError_t e = make_tmap(&tx, X, 2 * d, n_rows, kBK, kBM);
-    if (e == cudaSuccess) e = make_tmap(&tg, w_gate, 2 * d, I, kBK, BN);
-    if (e == cudaSuccess) e = make_tmap(&tu, w_up, 2 * d, I, kBK, BN);
+    if (e == cudaSuccess) e = make_tmap(&tg, w_gate, 2 * d, I, kBK, bn_gu);
+    if (e == cudaSuccess) e = make_tmap(&tu, w_up, 2 * d, I, kBK, bn_gu);
     if (e == cudaSuccess) e = make_tmap(&ta, A, I, n_rows, kBK, kBM);
-    if (e == cudaSuccess) e = make_tmap(&td, w_down, I, d, kBK, BN);
+    if (e == cudaSuccess) e = make_tmap(&td, w_down, I, d, kBK, bn_d);
     if (e != cudaSuccess) return e;
+
+    // ---- gate/up: A = SiLU(X Wg^T) * (X Wu^T)
+    const int ks1 = choose_k_splits((I / bn_gu) * n_mg, 2 * d / kBK, ctx.num_sms);
     EpiParams ep{};
     ep.out = static_cast<__nv_bfloat16*>(A);
     ep.ld_out = I;
-    if (m_tiles == 1)
-        e = run_gemm<EPI_GATEUP, 1, 2, BN, 6>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, 1, ep);
-    else
-        e = run_gemm<EPI_GATEUP, 2, 2, BN, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, (m_tiles + 1) / 2, ep);
-    if (e != cudaSuccess) return e;
+    ep.partial = partial;
+    ep.ld_partial = 2 * I;
+    ep.partial_split_stride = static_cast<size_t>(n_rows) * 2 * I;
+    ep.n_total = I;
+    if (ks1 == 1) {
+        if (bn_gu == BN)
+            e = m_tiles == 1 ? run_gemm<EPI_GATEUP, 1, 2, BN, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, 1, ep)
+                             : run_gemm<EPI_GATEUP, 2, 2, BN, 3>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, n_mg, ep);
+        else
+            e = m_tiles == 1 ? run_gemm<EPI_GATEUP, 1, 2, 64, 6>(ctx, tx, tg, tu, n_rows, 2 * d, I / 64, 1, ep)
+                             : run_gemm<EPI_GATEUP, 2, 2, 64, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / 64, n_mg, ep);
+        if (e != cudaSuccess) return e;
+    } else {
+        if (bn_gu == BN)
+            e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 2, BN, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, 1, ep, ks1)
+                             : run_gemm<EPI_PARTIAL, 2, 2, BN, 3>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, n_mg, ep, ks1);
+        else
+            e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 2, 64, 6>(ctx, tx, tg, tu, n_rows, 2 * d, I / 64, 1, ep, ks1)
+                             : run_gemm<EPI_PARTIAL, 2, 2, 64, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / 64, n_mg, ep, ks1);
+        if (e != cudaSuccess) return e;
+        e = launch_swiglu_reduce(ctx, partial, ks1, n_rows, I, static_cast<__nv_bfloat16*>(A));
+        if (e != cudaSuccess) return e;
+    }
+
+    // ---- down + residual: h' = h + A Wd^T
+    const int ks2 = choose_k_splits((d / bn_d) * n_mg, I / kBK, ctx.num_sms);
     EpiParams ed{};
     ed.out = static_cast<__nv_bfloat16*>(h_prime);
     ed.ld_out = d;
@@ -453,9 +576,26 @@ cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, const void* w_gate, 
     ed.R = R;
     ed.M = M;
     ed.gamma = gamma;
-    if (m_tiles == 1)
-        return run_gemm<EPI_DOWN, 1, 1, BN, 8>(ctx, ta, td, td, n_rows, I, d / BN, 1, ed);
-    return run_gemm<EPI_DOWN, 2, 1, BN, 5>(ctx, ta, td, td, n_rows, I, d / BN, (m_tiles + 1) / 2, ed);
+    ed.partial = partial;
+    ed.ld_partial = d;
+    ed.partial_split_stride = static_cast<size_t>(n_rows) * d;
+    ed.n_total = d;
+    if (ks2 == 1) {
+        if (bn_d == BN)
+            return m_tiles == 1 ? run_gemm<EPI_DOWN, 1, 1, BN, 6>(ctx, ta, td, td, n_rows, I, d / BN, 1, ed)
+                                : run_gemm<EPI_DOWN, 2, 1, BN, 4>(ctx, ta, td, td, n_rows, I, d / BN, n_mg, ed);
+        return m_tiles == 1 ? run_gemm<EPI_DOWN, 1, 1, 64, 8>(ctx, ta, td, td, n_rows, I, d / 64, 1, ed)
+                            : run_gemm<EPI_DOWN, 2, 1, 64, 5>(ctx, ta, td, td, n_rows, I, d / 64, n_mg, ed);
+    }
+    if (bn_d == BN)
+        e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 1, BN, 6>(ctx, ta, td, td, n_rows, I, d / BN, 1, ed, ks2)
+                         : run_gemm<EPI_PARTIAL, 2, 1, BN, 4>(ctx, ta, td, td, n_rows, I, d / BN, n_mg, ed, ks2);
+    else
+        e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 1, 64, 8>(ctx, ta, td, td, n_rows, I, d / 64, 1, ed, ks2)
+                         : run_gemm<EPI_PARTIAL, 2, 1, 64, 5>(ctx, ta, td, td, n_rows, I, d / 64, n_mg, ed, ks2);
+    if (e != cudaSuccess) return e;
+    return launch_down_reduce(ctx, partial, ks2, n_rows, d, static_cast<const __nv_bfloat16*>(hidden), R, M, gamma,
+                              static_cast<__nv_bfloat16*>(h_prime));
 }
 
 }  // namespace tf

@@ -66,12 +66,19 @@ __global__ void __launch_bounds__(256) gather_norm_kernel(const T* __restrict__ 
 }
 
 // ------------------------------------------------------------------------------------------
-// OPT-Tree selection, one warp per sequence. The queue holds one entry per open child list:
-// (score, parent score, parent node, list row, rank in the list, depth, token). Popping rank k
-// of a list replaces the entry by rank k+1 of the same list (its next sibling), and an
-// expandable popped node adds rank 0 of its own child list. Because every list is sorted
-// (value desc, id asc), this pops exactly what pushing whole distributions would (Algorithm 1
-// Part 2 pushes q'^(m) entirely), with at most B + 1 entries live at any time.
+// OPT-Tree selection (Algorithm 1 Part 2), one warp per sequence. The queue holds one entry per
+// open child list: (path score, depth, parent node) packed into one 64-bit key, plus the list
+// row, the rank in the list, the parent's score and the token. Popping rank k of a list
+// replaces the entry by rank k+1 of the same list (its next sibling), and an expandable popped
+// node adds rank 0 of its own child list. Every list is sorted (value desc, id asc), so this
+// pops exactly what pushing whole distributions would, with at most B + 1 live entries.
+//
+// Queue order: larger score, then smaller depth, then smaller parent index. Two live entries
+// never share (depth, parent): each node opens at most one child list. So the key
+//   float_key(score) << 32 | (127 - depth) << 24 | (0xFFFFFF - parent)
+// is unique and its integer maximum is the next pop. Each lane keeps the best key of its own
+// slots (j = lane mod 32) and rescans only when one of them changed; a pop is two warp max
+// reductions and a ballot.
 // ------------------------------------------------------------------------------------------
 struct TreeArgs {
     int gamma, M, K1, K2, B, V, mode, R;
@@ -87,152 +94,184 @@ struct TreeArgs {
     int32_t* dev_status;
 };
 
-struct Q {
-    float* score;
-    float* pscore;
-    int* parent;
-    int* row;
-    int* rank;
-    int* depth;
-    int* tok;
-};
-
-__device__ __forceinline__ bool q_better(const Q& q, int a, int b) {
-    if (b < 0) return a >= 0;
-    if (a < 0) return false;
-    if (q.score[a] != q.score[b]) return q.score[a] > q.score[b];
-    if (q.depth[a] != q.depth[b]) return q.depth[a] < q.depth[b];
-    if (q.parent[a] != q.parent[b]) return q.parent[a] < q.parent[b];
-    return q.tok[a] < q.tok[b];
+__device__ __forceinline__ unsigned long long queue_key(float score, int depth, int parent) {
+    return (static_cast<unsigned long long>(float_key(score)) << 32) |
+           (static_cast<unsigned long long>(127 - depth) << 24) | static_cast<unsigned long long>(0xFFFFFF - parent);
 }
 
-__global__ void __launch_bounds__(32) build_tree_kernel(TreeArgs a) {
-    extern __shared__ uint8_t smem_raw[];
+constexpr int kTreeThreads = 256;
+
+// Shared-memory bytes of build_tree_kernel: queue, node arrays, stage-1 top-M, and (when they
+// fit) the sequence's child lists.
+__host__ __device__ inline size_t tree_smem_fixed(int B, int gamma, int M) {
+    return static_cast<size_t>(B + 2) * (8 + 4 * 4) + static_cast<size_t>(B + 1) * 4 * 4 +
+           static_cast<size_t>(gamma) * M * 4;
+}
+__host__ __device__ inline size_t tree_smem_lists(int mode, int gamma, int R, int K1, int K2) {
+    return mode == TF_MODE_AR ? static_cast<size_t>(R) * K2 * 8 : static_cast<size_t>(gamma) * K1 * 8;
+}
+constexpr size_t kTreeSmemLimit = 200 * 1024;
+
+__global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, int stage_lists) {
+    extern __shared__ __align__(16) uint8_t smem_raw[];
     const int cap = a.B + 2;
-    Q q;
-    q.score = reinterpret_cast<float*>(smem_raw);
-    q.pscore = q.score + cap;
-    q.parent = reinterpret_cast<int*>(q.pscore + cap);
-    q.row = q.parent + cap;
-    q.rank = q.row + cap;
-    q.depth = q.rank + cap;
-    q.tok = q.depth + cap;
+    const int n_out = a.B + 1;
+    unsigned long long* qkey = reinterpret_cast<unsigned long long*>(smem_raw);
+    float* qps = reinterpret_cast<float*>(qkey + cap);
+    int* qrow = reinterpret_cast<int*>(qps + cap);
+    int* qrank = qrow + cap;
+    int* qtok = qrank + cap;
+    int* o_tok = qtok + cap;
+    int* o_par = o_tok + n_out;
+    int* o_dep = o_par + n_out;
+    float* o_score = reinterpret_cast<float*>(o_dep + n_out);
+    int* topm = reinterpret_cast<int*>(o_score + n_out);          // [gamma, M]
+    uint8_t* lists = reinterpret_cast<uint8_t*>(topm + a.gamma * a.M);
 
     const int s = blockIdx.x;
-    const int lane = threadIdx.x;
-    const int n_out = a.B + 1;
-    int flags = 0;
-    const int root = a.root_tok[s];
-    if (root < 0 || root >= a.V) flags |= TF_DEV_BAD_TOKEN;
-
+    const int tid = threadIdx.x;
     const bool ar = a.mode == TF_MODE_AR;
-    const int list_len = a.K2;
-    // child list `row` of this sequence: stage-2 rows (AR) or stage-1 depths (marginal modes)
-    auto ids_of = [&](int row) -> const int32_t* {
-        return ar ? a.child_ids + (static_cast<size_t>(s) * a.R + row) * a.K2
-                  : a.top_ids + (static_cast<size_t>(s) * a.gamma + row) * a.K1;
-    };
-    auto lp_of = [&](int row) -> const float* {
-        return ar ? a.child_logp + (static_cast<size_t>(s) * a.R + row) * a.K2
-                  : a.top_logp + (static_cast<size_t>(s) * a.gamma + row) * a.K1;
-    };
-
-    int n_e = 0;
-    if (lane == 0) {
-        a.node_tok[static_cast<size_t>(s) * n_out] = root;
-        a.node_parent[static_cast<size_t>(s) * n_out] = -1;
-        a.node_depth[static_cast<size_t>(s) * n_out] = 0;
-        a.node_score[static_cast<size_t>(s) * n_out] = 0.0f;
-        const float lp = lp_of(0)[0];
-        q.score[0] = lp;
-        q.pscore[0] = 0.0f;
-        q.parent[0] = 0;
-        q.row[0] = 0;
-        q.rank[0] = 0;
-        q.depth[0] = 1;
-        q.tok[0] = ids_of(0)[0];
-    }
-    n_e = 1;
-    __syncwarp();
-
-    int count = 1;
-    while (count < n_out && n_e > 0) {
-        // warp-wide arg-max over live entries in the queue order
-        int best = -1;
-        for (int j = lane; j < n_e; j += 32)
-            if (q_better(q, j, best)) best = j;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const int other = __shfl_xor_sync(0xffffffffu, best, o);
-            if (q_better(q, other, best)) best = other;
+    const int n_rows_l = ar ? a.R : a.gamma;
+    const int stride = ar ? a.K2 : a.K1;
+    const int32_t* g_ids = ar ? a.child_ids + static_cast<size_t>(s) * a.R * a.K2
+                              : a.top_ids + static_cast<size_t>(s) * a.gamma * a.K1;
+    const float* g_lp = ar ? a.child_logp + static_cast<size_t>(s) * a.R * a.K2
+                           : a.top_logp + static_cast<size_t>(s) * a.gamma * a.K1;
+    const int32_t* ids_base = g_ids;
+    const float* lp_base = g_lp;
+    // stage the sequence's child lists and stage-1 top-M (every pop then touches shared memory only)
+    for (int i = tid; i < a.gamma * a.M; i += kTreeThreads)
+        topm[i] = a.top_ids[(static_cast<size_t>(s) * a.gamma + i / a.M) * a.K1 + i % a.M];
+    if (stage_lists) {
+        const int n = n_rows_l * stride;
+        int32_t* si = reinterpret_cast<int32_t*>(lists);
+        float* sl = reinterpret_cast<float*>(si + n);
+        for (int i = tid; i < n; i += kTreeThreads) {
+            si[i] = g_ids[i];
+            sl[i] = g_lp[i];
         }
-        const float sc = q.score[best], psc = q.pscore[best];
-        const int par = q.parent[best], row = q.row[best], rank = q.rank[best];
-        const int dep = q.depth[best], tok = q.tok[best];
+        ids_base = si;
+        lp_base = sl;
+    }
+    __syncthreads();
+
+    if (tid < 32) {
+        const int lane = tid;
+        constexpr unsigned kFull = 0xffffffffu;
+        int flags = 0;
+        const int root = a.root_tok[s];
+        if (root < 0 || root >= a.V) flags |= TF_DEV_BAD_TOKEN;
+        const int list_len = a.K2;
+        auto ids_of = [&](int row) -> const int32_t* { return ids_base + static_cast<size_t>(row) * stride; };
+        auto lp_of = [&](int row) -> const float* { return lp_base + static_cast<size_t>(row) * stride; };
+        if (lane == 0) {
+            o_tok[0] = root;
+            o_par[0] = -1;
+            o_dep[0] = 0;
+            o_score[0] = 0.0f;
+            qkey[0] = queue_key(lp_of(0)[0], 1, 0);
+            qps[0] = 0.0f;
+            qrow[0] = 0;
+            qrank[0] = 0;
+            qtok[0] = ids_of(0)[0];
+        }
+        int n_e = 1;
+        int count = 1;
         __syncwarp();
-        const int node = count++;
-        if (tok < 0 || tok >= a.V) flags |= TF_DEV_BAD_TOKEN;
-        if (!isfinite(sc)) flags |= TF_DEV_NONFINITE;
-        // expandable? (depth cap; M-ary rule via one compare per lane)
-        int crow = -1;
-        if (dep < a.gamma) {
-            if (a.mode == TF_MODE_MARGINAL) {
-                crow = dep;
-            } else {
-                const bool hit = lane < a.M &&
-                                 a.top_ids[(static_cast<size_t>(s) * a.gamma + dep - 1) * a.K1 + lane] == tok;
-                const unsigned bal = __ballot_sync(0xffffffffu, hit);
-                if (bal) {
-                    const int m = __ffs(bal) - 1;
-                    crow = ar ? 1 + (dep - 1) * a.M + m : dep;
+        unsigned long long lbest = 0ull;
+        int lidx = -1;
+        auto rescan = [&]() {
+            lbest = 0ull;
+            lidx = -1;
+            for (int j = lane; j < n_e; j += 32) {
+                const unsigned long long k = qkey[j];
+                if (k > lbest) {
+                    lbest = k;
+                    lidx = j;
                 }
             }
-        }
-        if (lane == 0) {
-            const size_t o = static_cast<size_t>(s) * n_out + node;
-            a.node_tok[o] = tok;
-            a.node_parent[o] = par;
-            a.node_depth[o] = dep;
-            a.node_score[o] = sc;
-            if (rank + 1 < list_len) {       // next sibling of the popped entry
-                q.rank[best] = rank + 1;
-                q.tok[best] = ids_of(row)[rank + 1];
-                q.score[best] = psc + lp_of(row)[rank + 1];
-            } else {                         // list exhausted: move the last entry here
-                const int last = n_e - 1;
-                q.score[best] = q.score[last];
-                q.pscore[best] = q.pscore[last];
-                q.parent[best] = q.parent[last];
-                q.row[best] = q.row[last];
-                q.rank[best] = q.rank[last];
-                q.depth[best] = q.depth[last];
-                q.tok[best] = q.tok[last];
+        };
+        rescan();
+        while (count < n_out && n_e > 0) {
+            const uint32_t hi = static_cast<uint32_t>(lbest >> 32), lo = static_cast<uint32_t>(lbest);
+            const uint32_t mhi = __reduce_max_sync(kFull, hi);
+            const uint32_t mlo = __reduce_max_sync(kFull, hi == mhi ? lo : 0u);
+            const unsigned win = __ballot_sync(kFull, lbest != 0ull && hi == mhi && lo == mlo);
+            if (win == 0u) break;
+            const int best = __shfl_sync(kFull, lidx, __ffs(win) - 1);
+            const float sc = key_float(mhi);
+            const int dep = 127 - static_cast<int>(mlo >> 24);
+            const int par = 0xFFFFFF - static_cast<int>(mlo & 0xFFFFFFu);
+            const int row = qrow[best], rank = qrank[best], tok = qtok[best];
+            const float psc = qps[best];
+            __syncwarp();
+            const int node = count++;
+            if (tok < 0 || tok >= a.V) flags |= TF_DEV_BAD_TOKEN;
+            if (!isfinite(sc)) flags |= TF_DEV_NONFINITE;
+            // expandable? (depth cap; M-ary rule via one compare per lane)
+            int crow = -1;
+            if (dep < a.gamma) {
+                if (a.mode == TF_MODE_MARGINAL) {
+                    crow = dep;
+                } else {
+                    const bool hit = lane < a.M && topm[(dep - 1) * a.M + lane] == tok;
+                    const unsigned bal = __ballot_sync(kFull, hit);
+                    if (bal) crow = ar ? 1 + (dep - 1) * a.M + (__ffs(bal) - 1) : dep;
+                }
             }
-        }
-        if (rank + 1 >= list_len) --n_e;
-        if (crow >= 0) {
+            const bool sibling = rank + 1 < list_len;
+            const int last = n_e - 1;
             if (lane == 0) {
-                q.score[n_e] = sc + lp_of(crow)[0];
-                q.pscore[n_e] = sc;
-                q.parent[n_e] = node;
-                q.row[n_e] = crow;
-                q.rank[n_e] = 0;
-                q.depth[n_e] = dep + 1;
-                q.tok[n_e] = ids_of(crow)[0];
+                o_tok[node] = tok;
+                o_par[node] = par;
+                o_dep[node] = dep;
+                o_score[node] = sc;
+                if (sibling) {                   // next sibling of the popped entry
+                    qrank[best] = rank + 1;
+                    qtok[best] = ids_of(row)[rank + 1];
+                    qkey[best] = queue_key(psc + lp_of(row)[rank + 1], dep, par);
+                } else if (best != last) {       // list exhausted: move the last entry here
+                    qkey[best] = qkey[last];
+                    qps[best] = qps[last];
+                    qrow[best] = qrow[last];
+                    qrank[best] = qrank[last];
+                    qtok[best] = qtok[last];
+                }
             }
-            ++n_e;
+            if (!sibling) --n_e;
+            int fresh = -1;
+            if (crow >= 0) {
+                fresh = n_e;
+                if (lane == 0) {
+                    qkey[n_e] = queue_key(sc + lp_of(crow)[0], dep + 1, node);
+                    qps[n_e] = sc;
+                    qrow[n_e] = crow;
+                    qrank[n_e] = 0;
+                    qtok[n_e] = ids_of(crow)[0];
+                }
+                ++n_e;
+            }
+            __syncwarp();
+            if (lane == (best & 31) || (!sibling && lane == (last & 31)) || (fresh >= 0 && lane == (fresh & 31)))
+                rescan();
         }
-        __syncwarp();
+        if (count < n_out) flags |= TF_DEV_UNDERFULL;
+        for (int i = count + lane; i < n_out; i += 32) {
+            o_tok[i] = -1;
+            o_par[i] = -1;
+            o_dep[i] = -1;
+            o_score[i] = -INFINITY;
+        }
+        if (lane == 0) a.dev_status[s] = flags;
     }
-    if (count < n_out) flags |= TF_DEV_UNDERFULL;
-    for (int i = count + lane; i < n_out; i += 32) {
+    __syncthreads();
+    for (int i = tid; i < n_out; i += kTreeThreads) {
         const size_t o = static_cast<size_t>(s) * n_out + i;
-        a.node_tok[o] = -1;
-        a.node_parent[o] = -1;
-        a.node_depth[o] = -1;
-        a.node_score[o] = -INFINITY;
+        a.node_tok[o] = o_tok[i];
+        a.node_parent[o] = o_par[i];
+        a.node_depth[o] = o_dep[i];
+        a.node_score[o] = o_score[i];
     }
-    if (lane == 0) a.dev_status[s] = flags;
 }
 
 // ------------------------------------------------------------------------------------------
@@ -293,12 +332,105 @@ __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __
 
 }  // namespace
 
+// bf16 rows with d % 8 == 0: 16-byte loads and stores, 8 elements per thread and step.
+__global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
+    const uint4* __restrict__ hidden, const uint4* __restrict__ embed, const uint4* __restrict__ norm_h,
+    const uint4* __restrict__ norm_e, const int32_t* __restrict__ root_tok, const int32_t* __restrict__ top_ids,
+    int gamma, int M, int K1, int R, int d, int V, float eps, uint4* __restrict__ X, int* status) {
+    constexpr int kMaxPerThread = 4;          // d <= 256 * 8 * 4 = 8192
+    __shared__ float red[2][8];
+    const int row = blockIdx.x;
+    const int sq = row / R, r = row - sq * R;
+    const int hid = sq * gamma + stage2_hidden_index(r, M);
+    int tok = (r == 0) ? root_tok[sq] : top_ids[(static_cast<size_t>(sq) * gamma + (r - 1) / M) * K1 + (r - 1) % M];
+    if (tok < 0 || tok >= V) {
+        if (threadIdx.x == 0) set_status(status, TF_DEV_BAD_TOKEN);
+        tok = 0;
+    }
+    const int dv = d / 8;
+    const uint4* h = hidden + static_cast<size_t>(hid) * dv;
+    const uint4* e = embed + static_cast<size_t>(tok) * dv;
+    uint4 hv[kMaxPerThread], ev[kMaxPerThread];
+    float sh = 0.0f, se = 0.0f;
+#pragma unroll
+    for (int i = 0; i < kMaxPerThread; ++i) {
+        const int c = threadIdx.x + i * 256;
+        if (c < dv) {
+            hv[i] = h[c];
+            ev[i] = e[c];
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < kMaxPerThread; ++i) {
+        const int c = threadIdx.x + i * 256;
+        if (c < dv) {
+            const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&hv[i]);
+            const __nv_bfloat16* eb = reinterpret_cast<const __nv_bfloat16*>(&ev[i]);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const float a = __bfloat162float(hb[j]), b = __bfloat162float(eb[j]);
+                sh = fmaf(a, a, sh);
+                se = fmaf(b, b, se);
+            }
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        sh += __shfl_xor_sync(0xffffffffu, sh, o);
+        se += __shfl_xor_sync(0xffffffffu, se, o);
+    }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        red[0][warp] = sh;
+        red[1][warp] = se;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float a = 0.0f, b = 0.0f;
+        for (int w = 0; w < 8; ++w) {
+            a += red[0][w];
+            b += red[1][w];
+        }
+        red[0][0] = rsqrtf(a / d + eps);
+        red[1][0] = rsqrtf(b / d + eps);
+    }
+    __syncthreads();
+    const float ih = red[0][0], ie = red[1][0];
+    uint4* xr = X + static_cast<size_t>(row) * 2 * dv;
+#pragma unroll
+    for (int i = 0; i < kMaxPerThread; ++i) {
+        const int c = threadIdx.x + i * 256;
+        if (c < dv) {
+            const uint4 wh = norm_h[c], we = norm_e[c];
+            const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&hv[i]);
+            const __nv_bfloat16* eb = reinterpret_cast<const __nv_bfloat16*>(&ev[i]);
+            const __nv_bfloat16* whb = reinterpret_cast<const __nv_bfloat16*>(&wh);
+            const __nv_bfloat16* web = reinterpret_cast<const __nv_bfloat16*>(&we);
+            uint4 oh, oe;
+            __nv_bfloat16* ohb = reinterpret_cast<__nv_bfloat16*>(&oh);
+            __nv_bfloat16* oeb = reinterpret_cast<__nv_bfloat16*>(&oe);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                ohb[j] = __float2bfloat16_rn(__bfloat162float(hb[j]) * ih * __bfloat162float(whb[j]));
+                oeb[j] = __float2bfloat16_rn(__bfloat162float(eb[j]) * ie * __bfloat162float(web[j]));
+            }
+            xr[c] = oh;
+            xr[dv + c] = oe;
+        }
+    }
+}
+
 cudaError_t launch_gather_norm(const Ctx& ctx, int dtype, const void* hidden, const void* embed, const void* norm_h,
                                const void* norm_e, const int32_t* root_tok, const int32_t* top_ids, int b, int gamma,
                                int M, int K1, int d, int V, float eps, void* X) {
     const int R = 1 + M * (gamma - 1);
     const int rows = b * R;
-    if (dtype == TF_BF16) {
+    if (dtype == TF_BF16 && d % 8 == 0 && d <= 8192) {
+        gather_norm_bf16x8_kernel<<<rows, 256, 0, ctx.stream>>>(
+            static_cast<const uint4*>(hidden), static_cast<const uint4*>(embed), static_cast<const uint4*>(norm_h),
+            static_cast<const uint4*>(norm_e), root_tok, top_ids, gamma, M, K1, R, d, V, eps, static_cast<uint4*>(X),
+            ctx.status);
+    } else if (dtype == TF_BF16) {
         gather_norm_kernel<__nv_bfloat16><<<rows, 256, 0, ctx.stream>>>(
             static_cast<const __nv_bfloat16*>(hidden), static_cast<const __nv_bfloat16*>(embed),
             static_cast<const __nv_bfloat16*>(norm_h), static_cast<const __nv_bfloat16*>(norm_e), root_tok, top_ids,
@@ -318,11 +450,14 @@ cudaError_t launch_build_tree(const Ctx& ctx, int b, int gamma, int M, int K1, i
                               int32_t* node_parent, int32_t* node_depth, float* node_score, int32_t* dev_status) {
     TreeArgs a{gamma, M, K1, K2, B, V, mode, R, root_tok, top_ids, top_logp, child_ids, child_logp,
                node_tok, node_parent, node_depth, node_score, dev_status};
-    const size_t smem = static_cast<size_t>(B + 2) * 7 * 4;
+    const size_t fixed = tree_smem_fixed(B, gamma, M);
+    const size_t lists = tree_smem_lists(mode, gamma, R, K1, K2);
+    const int stage = fixed + lists <= kTreeSmemLimit ? 1 : 0;
+    const size_t smem = fixed + (stage ? lists : 0);
     cudaError_t e = cudaFuncSetAttribute(build_tree_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    build_tree_kernel<<<b, 32, smem, ctx.stream>>>(a);
+    build_tree_kernel<<<b, kTreeThreads, smem, ctx.stream>>>(a, stage);
     return cudaGetLastError();
 }
 
