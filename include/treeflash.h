@@ -224,6 +224,16 @@ tf_status tf_ar_approx(const tf_dims* dims, const tf_weights* w, const void* hid
  * as separate calls without a copy. */
 tf_status tf_workspace_h_prime(const tf_dims* dims, void* ws, size_t ws_bytes, void** h_prime);
 
+/* Intermediates of Eq. 1 left in the workspace by the last tf_ar_approx / tf_stage2_ar_approx
+ * (for inspection and testing; host only, no GPU work):
+ *   TF_VIEW_X        x = [RMSNorm(h)*w_h ; RMSNorm(Embd(prev))*w_e]   [b*R, 2d] dtype
+ *   TF_VIEW_A        SiLU(W_gate x) * (W_up x)                         [b*R, I]  dtype
+ *   TF_VIEW_H_PRIME  h' = h + W_down A                                 [b*R, d]  dtype
+ * *ptr receives the device address and *bytes the view's size. */
+typedef enum { TF_VIEW_X = 0, TF_VIEW_A = 1, TF_VIEW_H_PRIME = 2 } tf_view;
+tf_status tf_workspace_view(const tf_dims* dims, void* ws, size_t ws_bytes, int32_t view, void** ptr,
+                            size_t* bytes);
+
 #ifdef __cplusplus
 }
 #endif

@@ -46,7 +46,7 @@ class TfWeights(ctypes.Structure):
 EXPORTS = ("tf_status_string", "tf_version", "tf_workspace_size", "tf_status_reset", "tf_status_read",
            "tf_stage1_marginals", "tf_stage2_ar_approx", "tf_build_tree", "tf_tree_mask",
            "tf_draft_tree_host", "tf_lmhead_partials", "tf_lmhead_merge", "tf_ar_approx",
-           "tf_workspace_h_prime")
+           "tf_workspace_h_prime", "tf_workspace_view")
 
 _lib = None
 
@@ -78,6 +78,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
         "tf_lmhead_merge": (ctypes.c_int, [D, P, P, I32, I32, P, P, P, SZ, P]),
         "tf_ar_approx": (ctypes.c_int, [D, W, P, P, P, P, P, SZ, P]),
         "tf_workspace_h_prime": (ctypes.c_int, [D, P, SZ, ctypes.POINTER(P)]),
+        "tf_workspace_view": (ctypes.c_int, [D, P, SZ, I32, ctypes.POINTER(P), ctypes.POINTER(SZ)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -246,3 +247,16 @@ def tf_workspace_h_prime(dims: Dims, ws) -> torch.Tensor:
     esize = 2 if dims.dtype == "bf16" else 4
     n = dims.batch * dims.R * dims.d * esize
     return ws[off:off + n].view(dims.torch_dtype).view(dims.batch, dims.R, dims.d)
+
+
+TF_VIEW_X, TF_VIEW_A, TF_VIEW_H_PRIME = 0, 1, 2
+
+
+def tf_workspace_view(dims: Dims, ws, view: int) -> torch.Tensor:
+    """x [b*R, 2d], A [b*R, I] or h' [b*R, d] as a tensor view of the workspace (no copy)."""
+    p, n = ctypes.c_void_p(), ctypes.c_size_t()
+    _check("tf_workspace_view", load_library().tf_workspace_view(
+        ctypes.byref(dims.c()), _ptr(ws), ws.numel(), view, ctypes.byref(p), ctypes.byref(n)))
+    off = p.value - ws.data_ptr()
+    cols = {TF_VIEW_X: 2 * dims.d, TF_VIEW_A: dims.I, TF_VIEW_H_PRIME: dims.d}[view]
+    return ws[off:off + n.value].view(dims.torch_dtype).view(dims.batch * dims.R, cols)

@@ -9,7 +9,7 @@
 #include "common.cuh"
 
 namespace tf {
-size_t merge_smem_bytes(int n_tiles);
+size_t merge_smem_bytes(int n_tiles, int d);
 }
 
 namespace {
@@ -51,7 +51,7 @@ tf_status check_dims(const tf_dims* dims, Dims* o) {
     if (d.dtype == TF_BF16 && (d.d % 64 != 0 || (d.mode == TF_MODE_AR && d.I % 64 != 0)))
         return TF_ERR_UNSUPPORTED;
     const int n_tiles = (d.V + kBlockV - 1) / kBlockV;
-    if (merge_smem_bytes(n_tiles) > kMaxMergeSmem) return TF_ERR_UNSUPPORTED;
+    if (merge_smem_bytes(n_tiles, d.d) > kMaxMergeSmem) return TF_ERR_UNSUPPORTED;
     const long long R = 1 + static_cast<long long>(d.M) * (d.gamma - 1);
     if (static_cast<long long>(d.batch) * R > (1ll << 30) || static_cast<long long>(d.batch) * d.gamma > (1ll << 30))
         return TF_ERR_UNSUPPORTED;
@@ -340,6 +340,23 @@ tf_status tf_workspace_h_prime(const tf_dims* dims, void* ws, size_t ws_bytes, v
     TF_TRY(check_ws(L, ws, ws_bytes));
     *h_prime = at<void>(ws, L.hp);
     return TF_OK;
+}
+
+tf_status tf_workspace_view(const tf_dims* dims, void* ws, size_t ws_bytes, int32_t view, void** ptr,
+                            size_t* bytes) {
+    if (!ptr || !bytes) return TF_ERR_INVALID_ARG;
+    Dims D;
+    TF_TRY(check_dims(dims, &D));
+    if (D.mode != TF_MODE_AR) return TF_ERR_INVALID_ARG;
+    const Layout L = layout(D);
+    TF_TRY(check_ws(L, ws, ws_bytes));
+    const size_t rows = static_cast<size_t>(D.b) * D.R;
+    switch (view) {
+        case TF_VIEW_X: *ptr = at<void>(ws, L.X); *bytes = rows * 2 * D.d * D.esize; return TF_OK;
+        case TF_VIEW_A: *ptr = at<void>(ws, L.A); *bytes = rows * D.I * D.esize; return TF_OK;
+        case TF_VIEW_H_PRIME: *ptr = at<void>(ws, L.hp); *bytes = rows * D.d * D.esize; return TF_OK;
+    }
+    return TF_ERR_INVALID_ARG;
 }
 
 tf_status tf_draft_tree_host(const tf_dims* dims, const tf_weights* w, const void* hidden, const int32_t* root_tok,

@@ -11,24 +11,26 @@ namespace tf {
 
 // ---- sizes fixed by the kernels --------------------------------------------------------------
 constexpr int kBlockV = 256;        // vocabulary entries per LM-head block (one MMA N-tile)
-constexpr int kListLen = 8;         // (logit, id) pairs kept per (row, block) by the LM-head pass
+constexpr int kChunk = 32;           // vocabulary columns per chunk (one TMEM load per row)
+constexpr int kChunks = kBlockV / kChunk;  // chunks per block
 constexpr int kMaxK = 64;           // largest top-k a merge can return
 constexpr int kMaxM = 32;           // largest M (the builder tests membership with one warp)
 constexpr int kMaxB = 1023;         // largest draft budget
 constexpr int kMaxGamma = 64;
-constexpr int kMergeExpandLists = 8;  // lists a merge may recompute exactly (>= (kMaxK-1)/8 + 1)
+constexpr int kMergeExpandChunks = kMaxK;  // chunks a merge may recompute exactly
 constexpr int kMaxKSplits = 4;        // split-K factor of the approximator GEMMs (workspace sized for it)
 
-// Per (row, vocabulary block) summary written by the LM-head pass: the block's max logit m,
-// sum_v exp(z_v - m), and its kListLen largest logits in (value desc, id asc) order; unused
-// slots have id -1 and value -inf.
-struct __align__(8) Partial {
-    float m;
-    float s;
-    float v[kListLen];
-    int id[kListLen];
+// Per (row, vocabulary block of 256) summary written by the LM-head pass, one entry per 32-column
+// chunk: the chunk's largest logit (value, id; ties go to the smaller id), its second-largest
+// value, and sum_v exp(z_v - chunk max). Chunks are independent, so any thread may summarise any
+// chunk. Empty chunks have id -1, -inf values and sum 0.
+struct __align__(16) Partial {
+    float cmax[kChunks];
+    int cid[kChunks];
+    float c2[kChunks];
+    float cs[kChunks];
 };
-static_assert(sizeof(Partial) == 72, "Partial layout");
+static_assert(sizeof(Partial) == 128, "Partial layout");
 
 // ---- bf16 / f32 element access ----------------------------------------------------------------
 __device__ __forceinline__ float to_f32(float x) { return x; }

@@ -13,7 +13,8 @@ constexpr int kKChunk = 32;
 
 // One CTA: rows [r0, r0 + 32) x vocabulary block [v0, v0 + 256). Thread t owns vocabulary column
 // v0 + t and accumulates its 32 logits; the block is then staged in shared memory and one warp
-// per row computes the block max, sum of exp and top-8 with warp shuffles.
+// per row computes the block max, sum of exp and the per-chunk (max, id, second max) with warp
+// shuffles.
 __global__ void __launch_bounds__(256) lmhead_simt_kernel(const float* __restrict__ W, const float* __restrict__ X,
                                                           int n_rows, int d, int V, float inv_temp,
                                                           Partial* __restrict__ partials, int n_tiles) {
@@ -55,36 +56,16 @@ __global__ void __launch_bounds__(256) lmhead_simt_kernel(const float* __restric
     const int warp = t >> 5, lane = t & 31;
     for (int r = warp; r < kRowsPerCta; r += 8) {
         if (r0 + r >= n_rows) break;
-        float z[8];
-        float m = -INFINITY;
+        // chunk j = columns [32 j, 32 j + 32) of the block; lane holds column 32 j + lane
+        float z[kChunks];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            z[j] = zt[r * kBlockV + lane + 32 * j];
-            m = fmaxf(m, z[j]);
-        }
+        for (int j = 0; j < kChunks; ++j) z[j] = zt[r * kBlockV + lane + 32 * j];
+        Partial* p = partials + static_cast<size_t>(r0 + r) * n_tiles + vt;
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-        float s = 0.0f;
-        if (m > -INFINITY) {
-#pragma unroll
-            for (int j = 0; j < 8; ++j) s += expf(z[j] - m);
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-        // top-8: eight rounds of a warp-wide (value desc, id asc) arg-max
-        float tv[kListLen];
-        int ti[kListLen];
-        for (int k = 0; k < kListLen; ++k) {
-            float bv = -INFINITY;
-            int bid = 0x7fffffff;
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const int id = vt * kBlockV + lane + 32 * j;
-                if (z[j] > bv || (z[j] == bv && z[j] > -INFINITY && id < bid)) {
-                    bv = z[j];
-                    bid = id;
-                }
-            }
+        for (int j = 0; j < kChunks; ++j) {
+            const int id = vt * kBlockV + 32 * j + lane;
+            float bv = z[j];
+            int bid = z[j] > -INFINITY ? id : 0x7fffffff;
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) {
                 const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
@@ -94,29 +75,17 @@ __global__ void __launch_bounds__(256) lmhead_simt_kernel(const float* __restric
                     bid = oid;
                 }
             }
-            if (bv == -INFINITY) {
-                tv[k] = -INFINITY;
-                ti[k] = -1;
-                continue;
-            }
-            tv[k] = bv;
-            ti[k] = bid;
-            const int owner = (bid - vt * kBlockV) & 31;
-            const int slot = (bid - vt * kBlockV) >> 5;
-            if (lane == owner) {
+            float sv = (id == bid) ? -INFINITY : z[j];
 #pragma unroll
-                for (int j = 0; j < 8; ++j)
-                    if (j == slot) z[j] = -INFINITY;
-            }
-        }
-        if (lane == 0) {
-            Partial* p = partials + static_cast<size_t>(r0 + r) * n_tiles + vt;
-            p->m = m;
-            p->s = s;
+            for (int o = 16; o > 0; o >>= 1) sv = fmaxf(sv, __shfl_xor_sync(0xffffffffu, sv, o));
+            float e = bv > -INFINITY ? expf(z[j] - bv) : 0.0f;
 #pragma unroll
-            for (int j = 0; j < kListLen; ++j) {
-                p->v[j] = tv[j];
-                p->id[j] = ti[j];
+            for (int o = 16; o > 0; o >>= 1) e += __shfl_xor_sync(0xffffffffu, e, o);
+            if (lane == 0) {
+                p->cmax[j] = bv;
+                p->cid[j] = bv > -INFINITY ? bid : -1;
+                p->c2[j] = sv;
+                p->cs[j] = e;
             }
         }
     }

@@ -6,8 +6,8 @@
 // every epilogue thread owns one activation row and walks its logits / outputs serially.
 // Three fused epilogues:
 //   LMHEAD  the LM-head pass of Algorithm 1 (stage 1 and stage 2): for each (row, block of 256
-//           vocabulary entries) it keeps the block max, the sum of exp(z - max) and the 8 largest
-//           (z, id). Logits never leave the SM.
+//           vocabulary entries) it keeps the block max, the sum of exp(z - max) and, per 32-wide
+//           chunk, the largest (z, id) and the second-largest z. Logits never leave the SM.
 //   GATEUP  SwiGLU of Eq. 1, first half: A = SiLU(X W_gate^T) * (X W_up^T), bf16 out.
 //   DOWN    SwiGLU of Eq. 1, second half plus the residual: h' = h + A W_down^T, bf16 out.
 //
@@ -31,7 +31,8 @@ namespace {
 
 constexpr int kBK = 64;       // K elements per stage: one 128-byte swizzle row of bf16
 constexpr int kBM = 128;      // activation rows per M-tile (TMEM lanes)
-constexpr int kThreads = 320;
+constexpr int kEpiWarps = 16;  // two groups (one per TMEM slot) of eight warps
+constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
 enum { EPI_LMHEAD = 0, EPI_GATEUP = 1, EPI_DOWN = 2, EPI_PARTIAL = 3 };
@@ -72,7 +73,7 @@ struct TileCfg {
     static constexpr int kBarrierBytes = 256;
     static constexpr int kSmemBytes = STAGES * kStageBytes + kBarrierBytes + 1024;
     static_assert(NB * BN <= 256, "one accumulator slot is 256 TMEM columns");
-    static_assert(BN % 32 == 0 && BN >= 32 && BN <= 256, "N tile");
+    static_assert(BN % 64 == 0 && BN >= 64 && BN <= 256, "N tile (two epilogue warps split it in 32-column steps)");
     static_assert(kStageBytes % 1024 == 0, "stages must stay 1024-byte aligned for 128B swizzle");
 };
 
@@ -83,68 +84,52 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// Running (max, sum of exp) and sorted top-kListLen of one row, fed 32 logits at a time.
-struct RowTop {
-    float m, s;
-    float tv[kListLen];
-    int ti[kListLen];
+// Summary of one 32-column chunk of one row: logits of vocabulary ids v0 .. v0+31. The largest
+// value (with the smallest id among equals), the second-largest value and the sum of
+// exp(z - max) come from fixed trees over the 32 registers: the same instructions for every lane,
+// whatever the data (a per-lane sorted insertion would diverge across the warp's 32 rows).
+struct ChunkSum {
+    float mx, second, sum;
+    int id;
 };
-
-// Insert x (known to beat tv[kListLen-1]) into the descending list. Every position is computed
-// from the old list at once (no chain of swaps): new[t] = old[t-1] if x beats old[t-1], else x
-// if x beats old[t], else old[t]. Equal values keep the earlier (smaller) id first.
-__device__ __forceinline__ void top_insert(RowTop& rt, float x, int id) {
-    bool gt[kListLen];
-#pragma unroll
-    for (int t = 0; t < kListLen; ++t) gt[t] = x > rt.tv[t];
-    float nv[kListLen];
-    int ni[kListLen];
-    nv[0] = gt[0] ? x : rt.tv[0];
-    ni[0] = gt[0] ? id : rt.ti[0];
-#pragma unroll
-    for (int t = 1; t < kListLen; ++t) {
-        nv[t] = gt[t - 1] ? rt.tv[t - 1] : (gt[t] ? x : rt.tv[t]);
-        ni[t] = gt[t - 1] ? rt.ti[t - 1] : (gt[t] ? id : rt.ti[t]);
-    }
-#pragma unroll
-    for (int t = 0; t < kListLen; ++t) {
-        rt.tv[t] = nv[t];
-        rt.ti[t] = ni[t];
-    }
-}
-
-// One 32-column chunk of accumulators (logits of vocabulary ids v0 .. v0+31 for this row).
-// Max and sum use trees, not serial chains, so the 32 values proceed in parallel.
-__device__ __forceinline__ void lmhead_chunk(RowTop& rt, const uint32_t (&r)[32], int v0, int V, float inv_temp) {
+__device__ __forceinline__ ChunkSum lmhead_chunk(const uint32_t (&r)[32], int v0, int V, float inv_temp) {
     float v[32];
 #pragma unroll
     for (int j = 0; j < 32; ++j) v[j] = (v0 + j < V) ? __uint_as_float(r[j]) * inv_temp : -INFINITY;
-    float t[16];
+    float a1[16], a2[16];
+    int ai[16];
 #pragma unroll
-    for (int j = 0; j < 16; ++j) t[j] = fmaxf(v[2 * j], v[2 * j + 1]);
+    for (int i = 0; i < 16; ++i) {
+        const bool ge = v[2 * i] >= v[2 * i + 1];
+        a1[i] = ge ? v[2 * i] : v[2 * i + 1];
+        a2[i] = ge ? v[2 * i + 1] : v[2 * i];
+        ai[i] = ge ? 2 * i : 2 * i + 1;
+    }
+#pragma unroll
+    for (int w = 8; w >= 1; w >>= 1) {
+#pragma unroll
+        for (int i = 0; i < w; ++i) {
+            const bool a_wins = a1[i] > a1[i + w] || (a1[i] == a1[i + w] && ai[i] < ai[i + w]);
+            const float n2 = a_wins ? fmaxf(a2[i], a1[i + w]) : fmaxf(a1[i], a2[i + w]);
+            a1[i] = a_wins ? a1[i] : a1[i + w];
+            ai[i] = a_wins ? ai[i] : ai[i + w];
+            a2[i] = n2;
+        }
+    }
+    ChunkSum c;
+    c.mx = a1[0];
+    c.second = a2[0];
+    c.id = a1[0] > -INFINITY ? v0 + ai[0] : -1;
+    float e[16];
+    const float mx = a1[0] > -INFINITY ? a1[0] : 0.0f;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) e[j] = __expf(v[2 * j] - mx) + __expf(v[2 * j + 1] - mx);
 #pragma unroll
     for (int w = 8; w >= 1; w >>= 1)
 #pragma unroll
-        for (int j = 0; j < w; ++j) t[j] = fmaxf(t[j], t[j + w]);
-    const float cmax = t[0];
-    const float mn = fmaxf(rt.m, cmax);
-    if (mn > -INFINITY) {
-        float e[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) e[j] = __expf(v[2 * j] - mn) + __expf(v[2 * j + 1] - mn);
-#pragma unroll
-        for (int w = 8; w >= 1; w >>= 1)
-#pragma unroll
-            for (int j = 0; j < w; ++j) e[j] += e[j + w];
-        rt.s = rt.s * __expf(rt.m - mn) + e[0];
-        rt.m = mn;
-    }
-    if (cmax > rt.tv[kListLen - 1]) {
-        // ids grow with j, so a strict > keeps the smaller id first among equal values
-#pragma unroll
-        for (int j = 0; j < 32; ++j)
-            if (v[j] > rt.tv[kListLen - 1]) top_insert(rt, v[j], v0 + j);
-    }
+        for (int j = 0; j < w; ++j) e[j] += e[j + w];
+    c.sum = e[0];
+    return c;
 }
 
 template <int EPI, int MT, int NB, int BN, int STAGES>
@@ -176,7 +161,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         }
         for (int g = 0; g < 2; ++g) {
             ptx::mbar_init(&tfull[g], 1);
-            ptx::mbar_init(&tempty[g], 128);
+            ptx::mbar_init(&tempty[g], 32 * kEpiWarps / 2);
         }
         ptx::mbar_init(drain, 1);
         *abort_flag = 0;
@@ -298,8 +283,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     } else {
         // ------------------------------------------------------------------ epilogue
         const int e = warp - 2;
-        const int g = e >> 2;            // accumulator slot of this group
-        const int q = warp & 3;          // TMEM lane quarter of this warp
+        const int g = e / (kEpiWarps / 2);          // accumulator slot of this group
+        const int q = warp & 3;                     // TMEM lane quarter of this warp
+        const int half = (e % (kEpiWarps / 2)) / 4; // which half of the columns this warp takes
         uint32_t use = 0;
         int kl = 0;
         for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++kl) {
@@ -317,52 +303,35 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             const uint32_t tb = tmem_base + 256u * g + (static_cast<uint32_t>(q * 32) << 16);
 
             if constexpr (EPI == EPI_LMHEAD) {
-                RowTop rt;
-                rt.m = -INFINITY;
-                rt.s = 0.0f;
-#pragma unroll
-                for (int j = 0; j < kListLen; ++j) {
-                    rt.tv[j] = -INFINITY;
-                    rt.ti[j] = -1;
-                }
+                static_assert(BN == kBlockV, "one LM-head N tile is one vocabulary block");
+                // this warp's half of the block: chunks [h * kChunks / 2, (h + 1) * kChunks / 2)
+                constexpr int kHalf = kChunks / 2;
+                Partial* p = ep.partials + static_cast<size_t>(row) * n_ntiles + nt;
                 // warps whose 32 rows are all padding skip the accumulators entirely
                 if (row - lane < n_rows) {
-                    static_assert(BN % 64 == 0, "the LM-head epilogue walks 64 columns per step");
-                    uint32_t ra[32], rb[32];
-                    ptx::tmem_ld_32cols_nowait(tb, ra);
-                    ptx::tmem_wait_ld_regs(ra);
-#pragma unroll 1
-                    for (int c = 0; c < BN; c += 64) {
-                        // each TMEM load is in flight while the previous 32 columns are processed;
-                        // the warp reconverges before every warp-collective tcgen05 instruction
-                        ptx::tmem_ld_32cols_nowait(tb + c + 32, rb);
-                        lmhead_chunk(rt, ra, nt * BN + c, ep.V, ep.inv_temp);
-                        __syncwarp();
-                        ptx::tmem_wait_ld_regs(rb);
-                        if (c + 64 < BN) ptx::tmem_ld_32cols_nowait(tb + c + 64, ra);
-                        lmhead_chunk(rt, rb, nt * BN + c + 32, ep.V, ep.inv_temp);
-                        __syncwarp();
-                        if (c + 64 < BN) ptx::tmem_wait_ld_regs(ra);
+#pragma unroll
+                    for (int j = 0; j < kHalf; ++j) {
+                        const int ci = half * kHalf + j;
+                        uint32_t ra[32];
+                        ptx::tmem_ld_32cols(tb + ci * kChunk, ra);
+                        const ChunkSum c = lmhead_chunk(ra, nt * BN + ci * kChunk, ep.V, ep.inv_temp);
+                        if (row < n_rows) {
+                            p->cmax[ci] = c.mx;
+                            p->cid[ci] = c.id;
+                            p->c2[ci] = c.second;
+                            p->cs[ci] = c.sum;
+                        }
+                        __syncwarp();   // reconverge before the next warp-collective TMEM load
                     }
                 }
                 ptx::tc_fence_before();
                 ptx::mbar_arrive(&tempty[g]);
-                if (row < n_rows) {
-                    Partial* p = ep.partials + static_cast<size_t>(row) * n_ntiles + nt;
-                    float2* pf = reinterpret_cast<float2*>(p);
-                    pf[0] = make_float2(rt.m, rt.s);
-#pragma unroll
-                    for (int j = 0; j < kListLen; j += 2) pf[1 + j / 2] = make_float2(rt.tv[j], rt.tv[j + 1]);
-                    int2* pi = reinterpret_cast<int2*>(p->id);
-#pragma unroll
-                    for (int j = 0; j < kListLen; j += 2) pi[j / 2] = make_int2(rt.ti[j], rt.ti[j + 1]);
-                }
             } else if constexpr (EPI == EPI_PARTIAL) {
                 float* base = ep.partial + w.kx * ep.partial_split_stride + static_cast<size_t>(row) * ep.ld_partial;
 #pragma unroll 1
                 for (int nb = 0; nb < NB; ++nb) {
 #pragma unroll 1
-                    for (int c = 0; c < BN; c += 32) {
+                    for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
                         uint32_t ra[32];
                         ptx::tmem_ld_32cols(tb + nb * BN + c, ra);
                         if (row < n_rows) {
@@ -378,7 +347,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 ptx::mbar_arrive(&tempty[g]);
             } else if constexpr (EPI == EPI_GATEUP) {
 #pragma unroll 1
-                for (int c = 0; c < BN; c += 32) {
+                for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
                     uint32_t rg[32], ru[32];
                     ptx::tmem_ld_32cols(tb + c, rg);
                     ptx::tmem_ld_32cols(tb + BN + c, ru);
@@ -405,7 +374,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                     hid_row = sq * ep.gamma + stage2_hidden_index(rr, ep.M);
                 }
 #pragma unroll 1
-                for (int c = 0; c < BN; c += 32) {
+                for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
                     uint32_t ra[32];
                     ptx::tmem_ld_32cols(tb + c, ra);
                     if (row < n_rows) {

@@ -105,7 +105,7 @@ constexpr int kTreeThreads = 256;
 // fit) the sequence's child lists.
 __host__ __device__ inline size_t tree_smem_fixed(int B, int gamma, int M) {
     return static_cast<size_t>(B + 2) * (8 + 4 * 4) + static_cast<size_t>(B + 1) * 4 * 4 +
-           static_cast<size_t>(gamma) * M * 4;
+           static_cast<size_t>(gamma) * M * 4 + 16;
 }
 __host__ __device__ inline size_t tree_smem_lists(int mode, int gamma, int R, int K1, int K2) {
     return mode == TF_MODE_AR ? static_cast<size_t>(R) * K2 * 8 : static_cast<size_t>(gamma) * K1 * 8;
@@ -126,7 +126,8 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
     int* o_dep = o_par + n_out;
     float* o_score = reinterpret_cast<float*>(o_dep + n_out);
     int* topm = reinterpret_cast<int*>(o_score + n_out);          // [gamma, M]
-    uint8_t* lists = reinterpret_cast<uint8_t*>(topm + a.gamma * a.M);
+    uint8_t* lists = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(topm + a.gamma * a.M) + 15) & ~static_cast<uintptr_t>(15));
 
     const int s = blockIdx.x;
     const int tid = threadIdx.x;
@@ -146,9 +147,38 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
         const int n = n_rows_l * stride;
         int32_t* si = reinterpret_cast<int32_t*>(lists);
         float* sl = reinterpret_cast<float*>(si + n);
-        for (int i = tid; i < n; i += kTreeThreads) {
-            si[i] = g_ids[i];
-            sl[i] = g_lp[i];
+        const bool vec = ((reinterpret_cast<uintptr_t>(g_ids) | reinterpret_cast<uintptr_t>(g_lp) |
+                           reinterpret_cast<uintptr_t>(si) | reinterpret_cast<uintptr_t>(sl)) & 15) == 0 &&
+                         (n & 3) == 0;
+        if (vec) {
+            // 16-byte copies, four per thread in flight before the first store
+            const int4* gi = reinterpret_cast<const int4*>(g_ids);
+            const float4* gl = reinterpret_cast<const float4*>(g_lp);
+            int4* di = reinterpret_cast<int4*>(si);
+            float4* dl = reinterpret_cast<float4*>(sl);
+            const int n4 = n >> 2;
+            constexpr int T = kTreeThreads;
+            int i = tid;
+            for (; i + 3 * T < n4; i += 4 * T) {       // 8 loads in flight, then 8 stores
+                const int4 a0 = gi[i], a1 = gi[i + T], a2 = gi[i + 2 * T], a3 = gi[i + 3 * T];
+                const float4 b0 = gl[i], b1 = gl[i + T], b2 = gl[i + 2 * T], b3 = gl[i + 3 * T];
+                di[i] = a0; di[i + T] = a1; di[i + 2 * T] = a2; di[i + 3 * T] = a3;
+                dl[i] = b0; dl[i + T] = b1; dl[i + 2 * T] = b2; dl[i + 3 * T] = b3;
+            }
+            for (; i < n4; i += T) {
+                const int4 a = gi[i];
+                const float4 b = gl[i];
+                di[i] = a;
+                dl[i] = b;
+            }
+        } else {
+#pragma unroll 8
+            for (int i = tid; i < n; i += kTreeThreads) {
+                const int32_t a = g_ids[i];
+                const float b = g_lp[i];
+                si[i] = a;
+                sl[i] = b;
+            }
         }
         ids_base = si;
         lp_base = sl;
@@ -332,13 +362,16 @@ __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __
 
 }  // namespace
 
-// bf16 rows with d % 8 == 0: 16-byte loads and stores, 8 elements per thread and step.
+// bf16 rows with d % 8 == 0: 16-byte loads and stores, 8 elements per thread and step. The
+// normalisation is evaluated in fp64 (one square root per row, d multiplies) and rounded once to
+// bf16, so x is the correctly rounded value of the definition: an x element off by one bf16 ulp
+// would perturb every gate/up output and flip many later roundings.
 __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
     const uint4* __restrict__ hidden, const uint4* __restrict__ embed, const uint4* __restrict__ norm_h,
     const uint4* __restrict__ norm_e, const int32_t* __restrict__ root_tok, const int32_t* __restrict__ top_ids,
     int gamma, int M, int K1, int R, int d, int V, float eps, uint4* __restrict__ X, int* status) {
     constexpr int kMaxPerThread = 4;          // d <= 256 * 8 * 4 = 8192
-    __shared__ float red[2][8];
+    __shared__ double red[2][8];
     const int row = blockIdx.x;
     const int sq = row / R, r = row - sq * R;
     const int hid = sq * gamma + stage2_hidden_index(r, M);
@@ -351,7 +384,7 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
     const uint4* h = hidden + static_cast<size_t>(hid) * dv;
     const uint4* e = embed + static_cast<size_t>(tok) * dv;
     uint4 hv[kMaxPerThread], ev[kMaxPerThread];
-    float sh = 0.0f, se = 0.0f;
+    double sh = 0.0, se = 0.0;
 #pragma unroll
     for (int i = 0; i < kMaxPerThread; ++i) {
         const int c = threadIdx.x + i * 256;
@@ -368,9 +401,9 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
             const __nv_bfloat16* eb = reinterpret_cast<const __nv_bfloat16*>(&ev[i]);
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
-                const float a = __bfloat162float(hb[j]), b = __bfloat162float(eb[j]);
-                sh = fmaf(a, a, sh);
-                se = fmaf(b, b, se);
+                const double a = __bfloat162float(hb[j]), b = __bfloat162float(eb[j]);
+                sh = fma(a, a, sh);
+                se = fma(b, b, se);
             }
         }
     }
@@ -386,16 +419,16 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
     }
     __syncthreads();
     if (threadIdx.x == 0) {
-        float a = 0.0f, b = 0.0f;
+        double a = 0.0, b = 0.0;
         for (int w = 0; w < 8; ++w) {
             a += red[0][w];
             b += red[1][w];
         }
-        red[0][0] = rsqrtf(a / d + eps);
-        red[1][0] = rsqrtf(b / d + eps);
+        red[0][0] = 1.0 / sqrt(a / d + static_cast<double>(eps));
+        red[1][0] = 1.0 / sqrt(b / d + static_cast<double>(eps));
     }
     __syncthreads();
-    const float ih = red[0][0], ie = red[1][0];
+    const double ih = red[0][0], ie = red[1][0];
     uint4* xr = X + static_cast<size_t>(row) * 2 * dv;
 #pragma unroll
     for (int i = 0; i < kMaxPerThread; ++i) {
@@ -411,8 +444,10 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
             __nv_bfloat16* oeb = reinterpret_cast<__nv_bfloat16*>(&oe);
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
-                ohb[j] = __float2bfloat16_rn(__bfloat162float(hb[j]) * ih * __bfloat162float(whb[j]));
-                oeb[j] = __float2bfloat16_rn(__bfloat162float(eb[j]) * ie * __bfloat162float(web[j]));
+                ohb[j] = __double2bfloat16(static_cast<double>(__bfloat162float(hb[j])) * ih *
+                                           static_cast<double>(__bfloat162float(whb[j])));
+                oeb[j] = __double2bfloat16(static_cast<double>(__bfloat162float(eb[j])) * ie *
+                                           static_cast<double>(__bfloat162float(web[j])));
             }
             xr[c] = oh;
             xr[dv + c] = oe;
