@@ -17,7 +17,8 @@
  * Conventions shared by every call:
  *  - Pointers are DEVICE pointers owned by the caller unless a parameter says "host". The
  *    library allocates no memory and keeps no state between calls; scratch lives in the
- *    caller's workspace (tf_workspace_size). Calls are asynchronous on `stream` (NULL = the
+ *    caller's workspace (tf_workspace_size). The one exception is the fixed scratch array of
+ *    tf_stage1_marginals_static (end of this file). Calls are asynchronous on `stream` (NULL = the
  *    legacy default stream) and return once the work is queued.
  *  - Shapes are row-major. b = batch (independent sequences), d = hidden size, V = vocabulary,
  *    I = approximator width, gamma = block size, M = stage-1 candidates per depth, K2 =
@@ -233,6 +234,35 @@ tf_status tf_workspace_h_prime(const tf_dims* dims, void* ws, size_t ws_bytes, v
 typedef enum { TF_VIEW_X = 0, TF_VIEW_A = 1, TF_VIEW_H_PRIME = 2 } tf_view;
 tf_status tf_workspace_view(const tf_dims* dims, void* ws, size_t ws_bytes, int32_t view, void** ptr,
                             size_t* bytes);
+
+/* ------------------------------------------------------------------------------------------
+ * For callers that cannot allocate device memory. The paper has no counterpart to this call:
+ * it serves callers that cannot provide a workspace, e.g. a plugin or custom operator inside a
+ * host framework that owns all device memory and hands out none, or code on a latency-critical
+ * path where cudaMalloc/cudaFree are ruled out because they can synchronise the device.
+ * ---------------------------------------------------------------------------------------- */
+
+/* Size of the library's own scratch array. Every GPU that loads the library holds this much
+ * device memory until the process exits, whether or not the call below is used. */
+#define TF_STATIC_SCRATCH_BYTES ((size_t)8 << 20)
+
+/* tf_stage1_marginals without a workspace: the same kernels and the same results (top_ids,
+ * top_logp as there), with the per-block partials and the status word in a fixed array inside
+ * the library instead of the caller's workspace. Allocates nothing.
+ *  dev_status [1] int32 out (device): the call's TF_DEV_* flags, overwritten (not OR-ed) when
+ *             the call's work completes on `stream`; TF_DEV_RECOMPUTED alone is no error.
+ * Limit: 256 + b * gamma * ceil(V / 256) * 128 bytes must fit in TF_STATIC_SCRATCH_BYTES, i.e.
+ * b * gamma * ceil(V / 256) <= 65534 (b * gamma <= 110 at V = 151936); larger requests return
+ * TF_ERR_UNSUPPORTED before any GPU work. Other arguments are checked as in
+ * tf_stage1_marginals (TF_ERR_INVALID_ARG, TF_ERR_UNSUPPORTED).
+ * The first call on a device looks up the array's device address (cudaGetSymbolAddress, with
+ * that device current) and caches it; make that first call before any stream capture.
+ * Every call on a device shares the one array: calls that can overlap on the GPU (different
+ * streams, or threads sharing a device without ordering) race and corrupt each other's results.
+ * Issue them on one stream, or order them. */
+tf_status tf_stage1_marginals_static(const tf_dims* dims, const tf_weights* w, const void* hidden,
+                                     int32_t* top_ids, float* top_logp, int32_t* dev_status,
+                                     tf_stream_t stream);
 
 #ifdef __cplusplus
 }

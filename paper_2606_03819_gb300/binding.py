@@ -46,7 +46,7 @@ class TfWeights(ctypes.Structure):
 EXPORTS = ("tf_status_string", "tf_version", "tf_workspace_size", "tf_status_reset", "tf_status_read",
            "tf_stage1_marginals", "tf_stage2_ar_approx", "tf_build_tree", "tf_tree_mask",
            "tf_draft_tree_host", "tf_lmhead_partials", "tf_lmhead_merge", "tf_ar_approx",
-           "tf_workspace_h_prime", "tf_workspace_view")
+           "tf_workspace_h_prime", "tf_workspace_view", "tf_stage1_marginals_static")
 
 _lib = None
 
@@ -79,6 +79,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
         "tf_ar_approx": (ctypes.c_int, [D, W, P, P, P, P, P, SZ, P]),
         "tf_workspace_h_prime": (ctypes.c_int, [D, P, SZ, ctypes.POINTER(P)]),
         "tf_workspace_view": (ctypes.c_int, [D, P, SZ, I32, ctypes.POINTER(P), ctypes.POINTER(SZ)]),
+        "tf_stage1_marginals_static": (ctypes.c_int, [D, W, P, P, P, P, P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -260,3 +261,15 @@ def tf_workspace_view(dims: Dims, ws, view: int) -> torch.Tensor:
     off = p.value - ws.data_ptr()
     cols = {TF_VIEW_X: 2 * dims.d, TF_VIEW_A: dims.I, TF_VIEW_H_PRIME: dims.d}[view]
     return ws[off:off + n.value].view(dims.torch_dtype).view(dims.batch * dims.R, cols)
+
+
+TF_STATIC_SCRATCH_BYTES = 8 << 20
+
+
+def tf_stage1_marginals_static(dims: Dims, w: dict, hidden, top_ids, top_logp, dev_status, stream=None):
+    """tf_stage1_marginals for callers that cannot allocate: no workspace, the library's own fixed
+    scratch array instead. dev_status is a 1-element int32 device tensor that receives the call's
+    TF_DEV_* flags. Calls that overlap on the GPU share that array and race."""
+    _check("tf_stage1_marginals_static", load_library().tf_stage1_marginals_static(
+        ctypes.byref(dims.c()), ctypes.byref(weights_struct(w)), _ptr(hidden), _ptr(top_ids),
+        _ptr(top_logp), _ptr(dev_status), _stream(stream)))

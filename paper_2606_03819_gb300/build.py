@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(PKG, "lib")
 LIB = os.path.join(OUT_DIR, "libtreeflash.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["api.cu", "tc_gemm.cu", "simt.cu", "merge.cu", "tree.cu", "reduce.cu"]
+SOURCES = ["api.cu", "tc_gemm.cu", "simt.cu", "merge.cu", "tree.cu", "reduce.cu", "static_scratch.cu"]
 
 
 def nvcc() -> str:
