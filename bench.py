@@ -385,7 +385,7 @@ def run_gpu(args):
         "data": "synthetic (seeded N(0,0.02) weights, hidden states scaled to 2-4 nat marginals)",
         "config": {"workload": cfg.name, "batch": cfg.batch, "d": cfg.d, "V": cfg.V, "I": cfg.I,
                    "gamma": cfg.gamma, "M": cfg.M, "K2": cfg.K2, "B": cfg.B, "R": cfg.R,
-                   "l2": "no flush: inputs larger than L2 (W_lm 1.245 GB streamed twice per step)",
+                   "l2": f"no flush: inputs larger than L2 (W_lm {lm_bytes / 1e9:.3f} GB streamed twice per step)",
                    "parallelism": f"replicas x{world}"},
         "step_roofline": {"algorithmic_bytes": step_bytes, "achieved_gbs": step_bytes / (ms_per_step / 1e3) / 1e9,
                           "peak_gbs": peak, "frac": step_bytes / (ms_per_step / 1e3) / 1e9 / peak,
