@@ -251,9 +251,9 @@ tf_status tf_workspace_view(const tf_dims* dims, void* ws, size_t ws_bytes, int3
  * the library instead of the caller's workspace. Allocates nothing.
  *  dev_status [1] int32 out (device): the call's TF_DEV_* flags, overwritten (not OR-ed) when
  *             the call's work completes on `stream`; TF_DEV_RECOMPUTED alone is no error.
- * Limit: 256 + b * gamma * ceil(V / 256) * 128 bytes must fit in TF_STATIC_SCRATCH_BYTES, i.e.
- * b * gamma * ceil(V / 256) <= 65534 (b * gamma <= 110 at V = 151936); larger requests return
- * TF_ERR_UNSUPPORTED before any GPU work. Other arguments are checked as in
+ * Limit: with n = b * gamma * ceil(V / 256), 256 + roundup(32 n, 256) + 128 n bytes must fit in
+ * TF_STATIC_SCRATCH_BYTES, i.e. n <= 52426 (b * gamma <= 88 at V = 151936); larger requests
+ * return TF_ERR_UNSUPPORTED before any GPU work. Other arguments are checked as in
  * tf_stage1_marginals (TF_ERR_INVALID_ARG, TF_ERR_UNSUPPORTED).
  * The first call on a device looks up the array's device address (cudaGetSymbolAddress, with
  * that device current) and caches it; make that first call before any stream capture.

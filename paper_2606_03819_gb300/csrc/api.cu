@@ -28,7 +28,7 @@ struct Dims {
 };
 
 struct Layout {
-    size_t status, partials, X, A, hp, kpart;
+    size_t status, halves, chunks, X, A, hp, kpart;
     size_t h_hidden, h_root, h_pos, top_ids, top_logp, child_ids, child_logp;
     size_t n_tok, n_par, n_dep, n_score, n_mask, n_pos, n_stat;
     size_t total;
@@ -87,7 +87,8 @@ Layout layout(const Dims& D) {
     const size_t rows = rows1 > rows2 ? rows1 : rows2;
     const size_t nn = static_cast<size_t>(D.b) * (D.B + 1);
     L.status = take(sizeof(int32_t));
-    L.partials = take(rows * D.n_tiles * sizeof(Partial));
+    L.halves = take(rows * D.n_tiles * kHalfBytesPerRowBlock);
+    L.chunks = take(rows * D.n_tiles * kChunkBytesPerRowBlock);
     L.X = take(rows2 * 2 * D.d * D.esize);
     L.A = take(rows2 * D.I * D.esize);
     L.hp = take(rows2 * D.d * D.esize);
@@ -148,9 +149,15 @@ tf_status cuda_status(cudaError_t e) { return e == cudaSuccess ? TF_OK : TF_ERR_
     } while (0)
 
 // ---- the pieces -----------------------------------------------------------------------------
+// The LM-head partials of n_rows rows, laid out for exactly that many rows (the merge of the same
+// rows reads them with the same n_rows).
+Partials partials_of(const Layout& L, void* ws, int n_rows) {
+    return Partials{at<float4>(ws, L.halves), at<float4>(ws, L.chunks), n_rows};
+}
+
 tf_status do_partials(const Ctx& ctx, const Dims& D, const Layout& L, void* ws, const void* lm_head, const void* x,
                       int n_rows) {
-    Partial* partials = at<Partial>(ws, L.partials);
+    const Partials partials = partials_of(L, ws, n_rows);
     if (D.dtype == TF_BF16)
         return cuda_status(launch_lmhead_tc(ctx, lm_head, x, n_rows, D.d, D.V, D.inv_temp, partials));
     return cuda_status(launch_lmhead_simt(ctx, D.dtype, lm_head, x, n_rows, D.d, D.V, D.inv_temp, partials));
@@ -158,7 +165,7 @@ tf_status do_partials(const Ctx& ctx, const Dims& D, const Layout& L, void* ws, 
 
 tf_status do_merge(const Ctx& ctx, const Dims& D, const Layout& L, void* ws, const void* lm_head, const void* x,
                    int n_rows, int k, int32_t* ids, float* logp) {
-    return cuda_status(launch_lmhead_merge(ctx, D.dtype, at<Partial>(ws, L.partials), n_rows, D.V, D.d, k,
+    return cuda_status(launch_lmhead_merge(ctx, D.dtype, partials_of(L, ws, n_rows), n_rows, D.V, D.d, k,
                                            D.inv_temp, lm_head, x, ids, logp));
 }
 

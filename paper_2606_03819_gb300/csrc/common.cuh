@@ -20,17 +20,30 @@ constexpr int kMaxGamma = 64;
 constexpr int kMergeExpandChunks = kMaxK;  // chunks a merge may recompute exactly
 constexpr int kMaxKSplits = 4;        // split-K factor of the approximator GEMMs (workspace sized for it)
 
-// Per (row, vocabulary block of 256) summary written by the LM-head pass, one entry per 32-column
-// chunk: the chunk's largest logit (value, id; ties go to the smaller id), its second-largest
-// value, and sum_v exp(z_v - chunk max). Chunks are independent, so any thread may summarise any
-// chunk. Empty chunks have id -1, -inf values and sum 0.
-struct __align__(16) Partial {
-    float cmax[kChunks];
-    int cid[kChunks];
-    float c2[kChunks];
-    float cs[kChunks];
+// What the LM-head pass leaves per (row, vocabulary block of 256). Both arrays are indexed
+// [block][part][row], so the 32 lanes of an epilogue warp (32 consecutive rows) store 512
+// contiguous bytes per record.
+//  - halves [n_tiles][2][n_rows]: per half block (128 columns = 4 chunks) the max logit m, the
+//    sum over the half of exp(z - m), and the half's best (value, id bits). The merge reads only
+//    these for the log-sum-exp and its first threshold.
+//  - chunks [n_tiles][kChunks][n_rows]: per 32-column chunk its largest, second and third largest
+//    logits and, in .w, the chunk-local offsets of the first two (bits 0-7 and 8-15). Read only
+//    for the halves that can hold members of the top k: the two largest are candidates, the third
+//    bounds every other logit of the chunk.
+// Ties go to the smaller id. Empty entries have -inf values and sum 0.
+struct Partials {
+    float4* halves;
+    float4* chunks;
+    int n_rows;
+    __host__ __device__ size_t half_at(int tile, int half, int row) const {
+        return (static_cast<size_t>(tile) * 2 + half) * n_rows + row;
+    }
+    __host__ __device__ size_t chunk_at(int tile, int chunk, int row) const {
+        return (static_cast<size_t>(tile) * kChunks + chunk) * n_rows + row;
+    }
 };
-static_assert(sizeof(Partial) == 128, "Partial layout");
+constexpr size_t kHalfBytesPerRowBlock = 2 * sizeof(float4);
+constexpr size_t kChunkBytesPerRowBlock = kChunks * sizeof(float4);
 
 // ---- bf16 / f32 element access ----------------------------------------------------------------
 __device__ __forceinline__ float to_f32(float x) { return x; }
@@ -85,10 +98,10 @@ struct Ctx {
 
 // LM-head pass (tensor-core path for bf16, CUDA-core path for f32)
 cudaError_t launch_lmhead_tc(const Ctx&, const void* lm_head, const void* x, int n_rows, int d,
-                             int V, float inv_temp, Partial* partials);
+                             int V, float inv_temp, Partials partials);
 cudaError_t launch_lmhead_simt(const Ctx&, int dtype, const void* lm_head, const void* x,
-                               int n_rows, int d, int V, float inv_temp, Partial* partials);
-cudaError_t launch_lmhead_merge(const Ctx&, int dtype, const Partial* partials, int n_rows, int V,
+                               int n_rows, int d, int V, float inv_temp, Partials partials);
+cudaError_t launch_lmhead_merge(const Ctx&, int dtype, Partials partials, int n_rows, int V,
                                 int d, int k, float inv_temp, const void* lm_head, const void* x,
                                 int32_t* out_ids, float* out_logp);
 // Eq. 1 pieces

@@ -1,17 +1,19 @@
 // Merge of the LM-head partials into log-softmax top-k (Algorithm 1 "TopM" of stage 1 and the
 // log-softmax + top-k of every stage-2 row).
 //
-// One CTA per row. Inputs are the row's per-block summaries (block max, sum of exp, and per
-// 32-column chunk the max with its id and the second-largest value). The CTA
-//   1. combines the block (max, sum) pairs into the row's log-sum-exp;
-//   2. keeps as candidates the chunk maxima at or above the k-th largest block maximum and finds
-//      the k-th largest candidate key (value desc, id asc) with a radix select over 64-bit keys;
-//   3. certifies the result: a chunk whose second-largest value reaches the k-th candidate may
+// One CTA per row. The CTA
+//   1. combines the row's half-block (max, sum of exp) pairs into its log-sum-exp and forms one
+//      key (value desc, id asc) per half block from the half's best entry;
+//   2. finds theta0, the k-th largest half-block key. Exactly the k halves at or above it can
+//      hold members of the top k (every key elsewhere is below its half's best, hence below
+//      theta0). Their chunks' two largest entries at or above theta0 are the candidates; the
+//      k-th largest candidate key comes from a radix select over 64-bit keys;
+//   3. certifies the result: a chunk whose third-largest value reaches the k-th candidate may
 //      hide further members of the top k. Those chunks' 32 logits are recomputed exactly from
-//      lm_head and x, replace the chunk maxima, and the selection is redone;
+//      lm_head and x, replace the chunk's two candidates, and the selection is redone;
 //   4. writes the k winners sorted, as (id, logit - LSE).
-// The result is the exact top-k of the full vocabulary whatever the input; on random data about
-// one chunk per two rows is recomputed (32 dot products, a few microseconds).
+// The result is the exact top-k of the full vocabulary whatever the input; a recompute needs
+// three members of the top k in one 32-column chunk (about one row in 500 on random data).
 #include <math.h>
 
 #include "common.cuh"
@@ -30,19 +32,22 @@ __device__ __forceinline__ void lse_combine(float& m, float& s, float m2, float 
     }
 }
 
-// k-th largest of keys[0..n) (n >= k >= 1), by 8-bit digits from the most significant byte.
+// k-th largest of keys[0..n) (n >= k >= 1), by 8-bit digits from the most significant byte. Once
+// the chosen digit's bin holds a single key, that key is the answer and is looked up directly
+// (float keys of one row share their top bytes, so this usually ends the search after two or
+// three digits instead of eight).
 __device__ unsigned long long block_kth_largest(const unsigned long long* keys, int n, int k, int* hist,
-                                                int* sel_digit, int* sel_rem) {
+                                                int* sel, unsigned long long* found) {
     unsigned long long prefix = 0;
     int rem = k;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int n_pad = (n + kThreads - 1) / kThreads * kThreads;
     for (int shift = 56; shift >= 0; shift -= 8) {
         for (int i = tid; i < 256; i += kThreads) hist[i] = 0;
         __syncthreads();
         const unsigned long long hi_mask = shift == 56 ? 0ull : (~0ull << (shift + 8));
-        // warp-aggregated counting: lanes holding the same digit add once (float keys of one
-        // row share their top bytes, so plain atomics would serialise on a few bins)
-        const int n_pad = (n + kThreads - 1) / kThreads * kThreads;
+        // warp-aggregated counting: lanes holding the same digit add once (plain atomics would
+        // serialise on the few bins the keys of one row fall into)
         for (int i = tid; i < n_pad; i += kThreads) {
             int digit = 256;
             if (i < n) {
@@ -73,8 +78,9 @@ __device__ unsigned long long block_kth_largest(const unsigned long long* keys, 
                 int c = excl;
                 for (int b = 7; b >= 0; --b) {
                     if (c + local[b] >= rem) {
-                        *sel_digit = lane * 8 + b;
-                        *sel_rem = rem - c;
+                        sel[0] = lane * 8 + b;
+                        sel[1] = rem - c;
+                        sel[2] = local[b];
                         break;
                     }
                     c += local[b];
@@ -82,9 +88,19 @@ __device__ unsigned long long block_kth_largest(const unsigned long long* keys, 
             }
         }
         __syncthreads();
-        prefix |= static_cast<unsigned long long>(*sel_digit) << shift;
-        rem = *sel_rem;
-        __syncthreads();
+        prefix |= static_cast<unsigned long long>(sel[0]) << shift;
+        rem = sel[1];
+        if (sel[2] == 1 && shift > 0) {
+            // the k-th key is the only key with this prefix
+            const unsigned long long mask = ~0ull << shift;
+            for (int i = tid; i < n; i += kThreads)
+                if ((keys[i] & mask) == prefix) *found = keys[i];
+            __syncthreads();
+            const unsigned long long r = *found;
+            __syncthreads();   // every thread has read *found and sel before either is reused
+            return r;
+        }
+        __syncthreads();       // every thread has read sel before the next digit rewrites it
     }
     return prefix;
 }
@@ -125,72 +141,97 @@ __device__ __forceinline__ float dot_row(const float* w, const float* xs, int d,
     return acc;
 }
 
+// Shared-memory layout of one merge CTA (dynamic part).
+constexpr int kDetailChunks = kMaxK * (kChunks / 2);           // chunks of the <= k halves kept
+constexpr int kCandCap = 2 * kDetailChunks + kMergeExpandChunks * kChunk;
+struct MergeSmem {
+    unsigned long long* hkey;   // [n_halves] best key of every half block (0 = empty)
+    unsigned long long* cand;   // [kCandCap]
+    float* c3;                  // [kDetailChunks] third value of each kept chunk (bound on the rest)
+    int* cbase;                 // [kDetailChunks] first vocabulary id of each kept chunk
+    uint8_t* expanded;          // [kDetailChunks] chunk recomputed
+    float* xs;                  // [d] x of the row in fp32, staged only for a recompute
+};
+__host__ __device__ inline size_t merge_layout(int n_tiles, int d, uint8_t* base, MergeSmem* m) {
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        uint8_t* p = base ? base + off : nullptr;
+        off += (bytes + 15) / 16 * 16;
+        return p;
+    };
+    uint8_t* hk = take(static_cast<size_t>(2) * n_tiles * 8);
+    uint8_t* cd = take(static_cast<size_t>(kCandCap) * 8);
+    uint8_t* c3 = take(static_cast<size_t>(kDetailChunks) * 4);
+    uint8_t* cb = take(static_cast<size_t>(kDetailChunks) * 4);
+    uint8_t* ex = take(kDetailChunks);
+    uint8_t* xs = take(static_cast<size_t>(d) * 4);
+    if (m) {
+        m->hkey = reinterpret_cast<unsigned long long*>(hk);
+        m->cand = reinterpret_cast<unsigned long long*>(cd);
+        m->c3 = reinterpret_cast<float*>(c3);
+        m->cbase = reinterpret_cast<int*>(cb);
+        m->expanded = ex;
+        m->xs = reinterpret_cast<float*>(xs);
+    }
+    return off;
+}
+
 template <typename T>
-__global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(const Partial* __restrict__ partials, int n_rows,
-                                                                int n_tiles, int V, int d, int k, float inv_temp,
+__global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partials, int n_rows, int n_tiles, int V,
+                                                                int d, int k, float inv_temp,
                                                                 const T* __restrict__ lm_head,
                                                                 const T* __restrict__ x, int32_t* __restrict__ out_ids,
                                                                 float* __restrict__ out_logp, int* status) {
-    // dynamic shared memory: the row's block summaries, candidate keys, per-block best key,
-    // per-chunk "already recomputed" flags
     extern __shared__ __align__(16) uint8_t dsm[];
-    Partial* P = reinterpret_cast<Partial*>(dsm);
-    const int n_chunks = n_tiles * kChunks;
-    const int cap = n_chunks + kMergeExpandChunks * kChunk;
-    unsigned long long* cand = reinterpret_cast<unsigned long long*>(dsm + static_cast<size_t>(n_tiles) * sizeof(Partial));
-    unsigned long long* lmax = cand + cap;
-    uint8_t* expanded = reinterpret_cast<uint8_t*>(lmax + n_tiles);
-    float* xs = reinterpret_cast<float*>(expanded + (n_chunks + 15) / 16 * 16);   // [d], only when needed
-    bool x_staged = false;
+    MergeSmem S;
+    merge_layout(n_tiles, d, dsm, &S);
     __shared__ int hist[256];
     __shared__ float red_m[kThreads / 32], red_s[kThreads / 32];
-    __shared__ int sel_digit, sel_rem, n_flag, flag_list[kMergeExpandChunks], n_cand, n_sel, n_valid;
-    __shared__ unsigned long long sel[kMaxK];
+    __shared__ int sel_info[3], n_flag, flag_list[kMergeExpandChunks], n_cand, n_sel, n_valid, n_chalf;
+    __shared__ int chalf[kMaxK];
+    __shared__ unsigned long long sel[kMaxK], found;
     __shared__ float zbuf[kMergeExpandChunks * kChunk];
     __shared__ float lse_s;
 
     const int row = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-
-    // 0. stage the row's summaries (contiguous, 128 B each) with 16-byte loads, eight in flight
-    //    per thread before the first store
-    {
-        const uint4* src = reinterpret_cast<const uint4*>(partials + static_cast<size_t>(row) * n_tiles);
-        uint4* dst = reinterpret_cast<uint4*>(P);
-        const int n16 = n_tiles * static_cast<int>(sizeof(Partial) / 16);
-        constexpr int T = kThreads;
-        int i = tid;
-        for (; i + 7 * T < n16; i += 8 * T) {
-            uint4 v[8];
-#pragma unroll
-            for (int j = 0; j < 8; ++j) v[j] = src[i + j * T];
-#pragma unroll
-            for (int j = 0; j < 8; ++j) dst[i + j * T] = v[j];
-        }
-        for (; i < n16; i += T) dst[i] = src[i];
-    }
+    const int nh = 2 * n_tiles;
     if (tid == 0) {
         n_cand = 0;
         n_valid = 0;
+        n_chalf = 0;
     }
-    __syncthreads();
 
-    // 1. log-sum-exp over blocks; per-block best key
+    // 1. half-block summaries (strided by n_rows, eight loads in flight per thread): the row's
+    //    log-sum-exp and one key per half
     float m = -INFINITY, s = 0.0f;
     int my_valid = 0;
-    for (int t = tid; t < n_tiles; t += kThreads) {
-        unsigned long long best = 0ull;
+    {
+        const float4* src = partials.halves + row;
+        const size_t stride = static_cast<size_t>(partials.n_rows);
+        for (int base = tid; base < nh; base += 8 * kThreads) {
+            float4 v[8];
 #pragma unroll
-        for (int c = 0; c < kChunks; ++c) {
-            if (P[t].cid[c] < 0) continue;
-            lse_combine(m, s, P[t].cmax[c], P[t].cs[c]);
-            const unsigned long long key = cand_key(P[t].cmax[c], P[t].cid[c]);
-            best = key > best ? key : best;
+            for (int j = 0; j < 8; ++j) {
+                const int i = base + j * kThreads;
+                if (i < nh) v[j] = src[static_cast<size_t>(i) * stride];
+            }
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int i = base + j * kThreads;
+                if (i >= nh) break;
+                const int id = __float_as_int(v[j].w);
+                unsigned long long key = 0ull;
+                if (id >= 0) {
+                    lse_combine(m, s, v[j].x, v[j].y);
+                    key = cand_key(v[j].z, id);
+                    ++my_valid;
+                }
+                S.hkey[i] = key;
+            }
         }
-        lmax[t] = best;
-        my_valid += best != 0ull ? 1 : 0;
     }
-    for (int i = tid; i < n_chunks; i += kThreads) expanded[i] = 0;
+    for (int i = tid; i < kDetailChunks; i += kThreads) S.expanded[i] = 0;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
@@ -201,45 +242,63 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(const Partial* _
         red_m[warp] = m;
         red_s[warp] = s;
     }
+    __syncthreads();
     atomicAdd(&n_valid, my_valid);
     __syncthreads();
     if (tid == 0) {
-        float M = -INFINITY, S = 0.0f;
-        for (int w = 0; w < kThreads / 32; ++w) lse_combine(M, S, red_m[w], red_s[w]);
-        const float lse = M + logf(S);
+        float M = -INFINITY, Ssum = 0.0f;
+        for (int w = 0; w < kThreads / 32; ++w) lse_combine(M, Ssum, red_m[w], red_s[w]);
+        const float lse = M + logf(Ssum);
         lse_s = lse;
         if (!isfinite(lse)) set_status(status, TF_DEV_NONFINITE);
     }
 
-    // 2. candidates: the chunk maxima at or above the k-th largest block maximum. At least k keys
-    //    are >= that bound (the k block maxima), so the top k are all among the chunk maxima
-    //    above it or hidden behind them (handled in 3).
+    // 2. theta0 and the halves at or above it (at most k: the keys are distinct)
     const unsigned long long theta0 =
-        n_valid >= k ? block_kth_largest(lmax, n_tiles, k, hist, &sel_digit, &sel_rem) : 0ull;
-    for (int i = tid; i < n_chunks; i += kThreads) {
-        const int t = i / kChunks, c = i - (i / kChunks) * kChunks;
-        if (P[t].cid[c] < 0) continue;
-        const unsigned long long key = cand_key(P[t].cmax[c], P[t].cid[c]);
-        if (key >= theta0) cand[atomicAdd(&n_cand, 1)] = key;
+        n_valid >= k ? block_kth_largest(S.hkey, nh, k, hist, sel_info, &found) : 0ull;
+    for (int i = tid; i < nh; i += kThreads) {
+        const unsigned long long key = S.hkey[i];
+        if (key != 0ull && key >= theta0) {
+            const int slot = atomicAdd(&n_chalf, 1);
+            if (slot < kMaxK) chalf[slot] = i;
+        }
+    }
+    __syncthreads();
+    const int nch = min(n_chalf, kMaxK);
+    // their chunks: the two largest entries at or above theta0 become candidates
+    for (int i = tid; i < nch * (kChunks / 2); i += kThreads) {
+        const int h = chalf[i >> 2];
+        const int tile = h >> 1, chunk = (h & 1) * (kChunks / 2) + (i & 3);
+        const float4 q = partials.chunks[partials.chunk_at(tile, chunk, row)];
+        const int v0 = tile * kBlockV + chunk * kChunk;
+        const int ids = __float_as_int(q.w);
+        S.cbase[i] = v0;
+        S.c3[i] = q.z;
+        if (q.x > -INFINITY) {
+            const unsigned long long key = cand_key(q.x, v0 + (ids & 255));
+            if (key >= theta0) S.cand[atomicAdd(&n_cand, 1)] = key;
+        }
+        if (q.y > -INFINITY) {
+            const unsigned long long key = cand_key(q.y, v0 + ((ids >> 8) & 255));
+            if (key >= theta0) S.cand[atomicAdd(&n_cand, 1)] = key;
+        }
     }
     __syncthreads();
 
-    // 3. select; a chunk whose second-largest value reaches the k-th candidate may hide members
-    //    of the top k (every chunk below theta0 cannot), so its 32 logits are recomputed exactly
-    //    and the selection is redone until no chunk is in doubt
+    // 3. select; a kept chunk whose third value reaches the k-th candidate may hide members of
+    //    the top k, so its 32 logits are recomputed exactly and the selection is redone
     int n_expanded = 0;
+    bool x_staged = false;
     unsigned long long theta = 0;
     for (;;) {
         const int nc = n_cand;
-        theta = nc >= k ? block_kth_largest(cand, nc, k, hist, &sel_digit, &sel_rem) : 0ull;
+        theta = nc >= k ? block_kth_largest(S.cand, nc, k, hist, sel_info, &found) : 0ull;
         const float tval = key_value(theta);
         if (tid == 0) n_flag = 0;
         __syncthreads();
-        for (int i = tid; i < n_chunks; i += kThreads) {
-            const int t = i / kChunks, c = i - (i / kChunks) * kChunks;
-            if (expanded[i] || !(P[t].c2[c] > -INFINITY)) continue;
-            if (lmax[t] < theta0) continue;                     // the whole block is below the top k
-            if (nc < k || P[t].c2[c] >= tval) {
+        for (int i = tid; i < nch * (kChunks / 2); i += kThreads) {
+            if (S.expanded[i] || !(S.c3[i] > -INFINITY)) continue;
+            if (nc < k || S.c3[i] >= tval) {
                 const int slot = atomicAdd(&n_flag, 1);
                 if (slot < kMergeExpandChunks) flag_list[slot] = i;
             }
@@ -256,30 +315,32 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(const Partial* _
         // exact logits of every flagged chunk: x staged once in shared memory, then one warp per
         // column with all of its 16-byte weight loads issued before the multiply-adds
         if (!x_staged) {
-            for (int i = tid; i < d; i += kThreads) xs[i] = to_f32(x[static_cast<size_t>(row) * d + i]);
+            for (int i = tid; i < d; i += kThreads) S.xs[i] = to_f32(x[static_cast<size_t>(row) * d + i]);
             x_staged = true;
             __syncthreads();
         }
         for (int q = warp; q < nf * kChunk; q += kThreads / 32) {
             const int f = q / kChunk, cc = q - f * kChunk;
-            const int v = flag_list[f] * kChunk + cc;
-            float acc = v < V ? dot_row(lm_head + static_cast<size_t>(v) * d, xs, d, lane) : -INFINITY;
+            const int v = S.cbase[flag_list[f]] + cc;
+            const float acc = v < V ? dot_row(lm_head + static_cast<size_t>(v) * d, S.xs, d, lane) : 0.0f;
             if (lane == 0) zbuf[q] = v < V ? acc * inv_temp : -INFINITY;
         }
         __syncthreads();
-        // the flagged chunks' maxima leave the candidate set; all their logits enter it
-        for (int i = tid; i < n_cand; i += kThreads) {
-            const int id = key_id(cand[i]);
-            for (int f = 0; f < nf; ++f)
-                if (id / kChunk == flag_list[f]) cand[i] = 0ull;
+        // the flagged chunks' two candidates leave the candidate set; all their logits enter it
+        for (int j = tid; j < n_cand; j += kThreads) {
+            const int id = key_id(S.cand[j]);
+            for (int f = 0; f < nf; ++f) {
+                const int v0 = S.cbase[flag_list[f]];
+                if (id >= v0 && id < v0 + kChunk) S.cand[j] = 0ull;
+            }
         }
         __syncthreads();
         for (int q = tid; q < nf * kChunk; q += kThreads) {
             const int f = q / kChunk, cc = q - f * kChunk;
-            const int v = flag_list[f] * kChunk + cc;
-            if (v < V) cand[atomicAdd(&n_cand, 1)] = cand_key(zbuf[q], v);
+            const int v = S.cbase[flag_list[f]] + cc;
+            if (v < V) S.cand[atomicAdd(&n_cand, 1)] = cand_key(zbuf[q], v);
         }
-        for (int f = tid; f < nf; f += kThreads) expanded[flag_list[f]] = 1;
+        for (int f = tid; f < nf; f += kThreads) S.expanded[flag_list[f]] = 1;
         n_expanded += nf;
         __syncthreads();
     }
@@ -289,7 +350,7 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(const Partial* _
     __syncthreads();
     const int nc = n_cand;
     for (int i = tid; i < nc; i += kThreads) {
-        const unsigned long long key = cand[i];
+        const unsigned long long key = S.cand[i];
         if (key != 0ull && key >= theta) {
             const int slot = atomicAdd(&n_sel, 1);
             if (slot < kMaxK) sel[slot] = key;
@@ -314,14 +375,9 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(const Partial* _
 
 }  // namespace
 
-size_t merge_smem_bytes(int n_tiles, int d) {
-    const size_t n_chunks = static_cast<size_t>(n_tiles) * kChunks;
-    return static_cast<size_t>(n_tiles) * sizeof(Partial) +
-           (n_chunks + kMergeExpandChunks * kChunk + n_tiles) * sizeof(unsigned long long) + (n_chunks + 15) / 16 * 16 +
-           static_cast<size_t>(d) * sizeof(float);
-}
+size_t merge_smem_bytes(int n_tiles, int d) { return merge_layout(n_tiles, d, nullptr, nullptr); }
 
-cudaError_t launch_lmhead_merge(const Ctx& ctx, int dtype, const Partial* partials, int n_rows, int V, int d, int k,
+cudaError_t launch_lmhead_merge(const Ctx& ctx, int dtype, Partials partials, int n_rows, int V, int d, int k,
                                 float inv_temp, const void* lm_head, const void* x, int32_t* out_ids,
                                 float* out_logp) {
     if (n_rows <= 0) return cudaSuccess;

@@ -13,11 +13,11 @@ constexpr int kKChunk = 32;
 
 // One CTA: rows [r0, r0 + 32) x vocabulary block [v0, v0 + 256). Thread t owns vocabulary column
 // v0 + t and accumulates its 32 logits; the block is then staged in shared memory and one warp
-// per row computes the block max, sum of exp and the per-chunk (max, id, second max) with warp
-// shuffles.
+// per row computes, with warp shuffles, the per-chunk three largest logits (ids of the first
+// two) and the per-half max, sum of exp and best entry.
 __global__ void __launch_bounds__(256) lmhead_simt_kernel(const float* __restrict__ W, const float* __restrict__ X,
                                                           int n_rows, int d, int V, float inv_temp,
-                                                          Partial* __restrict__ partials, int n_tiles) {
+                                                          Partials partials, int n_tiles) {
     __shared__ float xs[kRowsPerCta][kKChunk + 1];
     __shared__ float ws[kBlockV][kKChunk + 1];
     const int vt = blockIdx.x;
@@ -60,34 +60,53 @@ __global__ void __launch_bounds__(256) lmhead_simt_kernel(const float* __restric
         float z[kChunks];
 #pragma unroll
         for (int j = 0; j < kChunks; ++j) z[j] = zt[r * kBlockV + lane + 32 * j];
-        Partial* p = partials + static_cast<size_t>(r0 + r) * n_tiles + vt;
+        const int row = r0 + r;
+        float hm[2] = {-INFINITY, -INFINITY}, hsum[2] = {0.0f, 0.0f}, hbv[2] = {-INFINITY, -INFINITY};
+        int hbid[2] = {-1, -1};
 #pragma unroll
         for (int j = 0; j < kChunks; ++j) {
-            const int id = vt * kBlockV + 32 * j + lane;
-            float bv = z[j];
-            int bid = z[j] > -INFINITY ? id : 0x7fffffff;
+            const int cbase = vt * kBlockV + 32 * j;
+            // three rounds of a warp-wide (value desc, id asc) arg-max over the chunk
+            float x = z[j];
+            float tv[3];
+            int ti[3];
 #pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-                const int oid = __shfl_xor_sync(0xffffffffu, bid, o);
-                if (ov > bv || (ov == bv && oid < bid)) {
-                    bv = ov;
-                    bid = oid;
+            for (int t3 = 0; t3 < 3; ++t3) {
+                float bv = x;
+                int bid = x > -INFINITY ? lane : 64;
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+                    const int oid = __shfl_xor_sync(0xffffffffu, bid, o);
+                    if (ov > bv || (ov == bv && oid < bid)) {
+                        bv = ov;
+                        bid = oid;
+                    }
                 }
+                tv[t3] = bv;
+                ti[t3] = bv > -INFINITY ? bid : 0;
+                if (bv > -INFINITY && lane == bid) x = -INFINITY;
             }
-            float sv = (id == bid) ? -INFINITY : z[j];
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) sv = fmaxf(sv, __shfl_xor_sync(0xffffffffu, sv, o));
-            float e = bv > -INFINITY ? expf(z[j] - bv) : 0.0f;
+            float e = tv[0] > -INFINITY ? expf(z[j] - tv[0]) : 0.0f;
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) e += __shfl_xor_sync(0xffffffffu, e, o);
-            if (lane == 0) {
-                p->cmax[j] = bv;
-                p->cid[j] = bv > -INFINITY ? bid : -1;
-                p->c2[j] = sv;
-                p->cs[j] = e;
+            const int h = j / (kChunks / 2);
+            if (tv[0] > hbv[h]) {
+                hbv[h] = tv[0];
+                hbid[h] = cbase + ti[0];
             }
+            if (tv[0] > -INFINITY) {
+                const float mn = fmaxf(hm[h], tv[0]);
+                hsum[h] = hsum[h] * expf(hm[h] - mn) + e * expf(tv[0] - mn);
+                hm[h] = mn;
+            }
+            if (lane == 0)
+                partials.chunks[partials.chunk_at(vt, j, row)] =
+                    make_float4(tv[0], tv[1], tv[2], __int_as_float(ti[0] | (ti[1] << 8)));
         }
+        if (lane == 0)
+            for (int h = 0; h < 2; ++h)
+                partials.halves[partials.half_at(vt, h, row)] = make_float4(hm[h], hsum[h], hbv[h], __int_as_float(hbid[h]));
     }
 }
 
@@ -161,7 +180,7 @@ __global__ void __launch_bounds__(256) swiglu_simt_kernel(const float* __restric
 }  // namespace
 
 cudaError_t launch_lmhead_simt(const Ctx& ctx, int dtype, const void* lm_head, const void* x, int n_rows, int d,
-                               int V, float inv_temp, Partial* partials) {
+                               int V, float inv_temp, Partials partials) {
     if (dtype != TF_F32) return cudaErrorNotSupported;
     if (n_rows <= 0) return cudaSuccess;
     const int n_tiles = (V + kBlockV - 1) / kBlockV;

@@ -26,7 +26,8 @@ constexpr int kMaxDevices = 64;
 
 static_assert(kScratchBytes % 256 == 0 && kScratchBytes > kStatusBytes, "scratch size");
 
-// The scratch: the status word at offset 0, then the LM-head partials [rows][n_tiles]. Every call
+// The scratch: the status word at offset 0, then the LM-head partials (half-block summaries, then
+// chunk records, each [n_tiles][part][rows]). Every call
 // on a device shares it and it keeps whatever the last call left, so each call clears the status
 // word before its first kernel; the partials need no clearing (the LM-head pass writes every
 // entry the merge reads). In host code `g_scratch` names a host-side shadow of the symbol, not
@@ -72,7 +73,9 @@ extern "C" tf_status tf_stage1_marginals_static(const tf_dims* dims, const tf_we
     const int K1 = dims->M > dims->K2 ? dims->M : dims->K2;
     const float inv_temp = 1.0f / dims->temperature;
     // the scratch limit, then the pointers; both before any GPU work
-    if (kStatusBytes + static_cast<size_t>(rows) * n_tiles * sizeof(Partial) > kScratchBytes)
+    const size_t row_blocks = static_cast<size_t>(rows) * n_tiles;
+    const size_t halves_bytes = (row_blocks * kHalfBytesPerRowBlock + 255) / 256 * 256;
+    if (kStatusBytes + halves_bytes + row_blocks * kChunkBytesPerRowBlock > kScratchBytes)
         return TF_ERR_UNSUPPORTED;
     if (!w || !aligned16(w->lm_head) || !aligned16(hidden) || !top_ids || !top_logp || !dev_status)
         return TF_ERR_INVALID_ARG;
@@ -87,7 +90,8 @@ extern "C" tf_status tf_stage1_marginals_static(const tf_dims* dims, const tf_we
         return TF_ERR_CUDA;
 
     const Ctx ctx{reinterpret_cast<cudaStream_t>(stream), sms, reinterpret_cast<int*>(scratch)};
-    Partial* partials = reinterpret_cast<Partial*>(scratch + kStatusBytes);
+    const Partials partials{reinterpret_cast<float4*>(scratch + kStatusBytes),
+                            reinterpret_cast<float4*>(scratch + kStatusBytes + halves_bytes), rows};
     cudaError_t e = cudaMemsetAsync(ctx.status, 0, sizeof(int32_t), ctx.stream);
     if (e != cudaSuccess) return TF_ERR_CUDA;
     e = dims->dtype == TF_BF16

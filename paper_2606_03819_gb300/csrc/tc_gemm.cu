@@ -6,16 +6,18 @@
 // every epilogue thread owns one activation row and walks its logits / outputs serially.
 // Three fused epilogues:
 //   LMHEAD  the LM-head pass of Algorithm 1 (stage 1 and stage 2): for each (row, block of 256
-//           vocabulary entries) it keeps the block max, the sum of exp(z - max) and, per 32-wide
-//           chunk, the largest (z, id) and the second-largest z. Logits never leave the SM.
+//           vocabulary entries) it keeps per half block the max, the sum of exp(z - max) and the
+//           best (z, id), and per 32-wide chunk the three largest z with the ids of the first
+//           two. Logits never leave the SM.
 //   GATEUP  SwiGLU of Eq. 1, first half: A = SiLU(X W_gate^T) * (X W_up^T), bf16 out.
 //   DOWN    SwiGLU of Eq. 1, second half plus the residual: h' = h + A W_down^T, bf16 out.
 //
-// Warp roles (320 threads, one CTA per SM, persistent over work units):
+// Warp roles (576 threads, one CTA per SM, persistent over work units):
 //   warp 0      TMA producer: one elected lane streams X and W tiles into a ring of stages.
 //   warp 1      TMEM allocator and MMA issuer (one lane issues tcgen05.mma and commits).
-//   warps 2..9  epilogue, two groups of four; group g drains accumulator slot g (TMEM columns
-//               [256 g, 256 g + 256)); warp w may only touch TMEM lanes 32 (w % 4) .. + 31.
+//   warps 2..17 epilogue, two groups of eight; group g drains accumulator slot g (TMEM columns
+//               [256 g, 256 g + 256)); warp w may only touch TMEM lanes 32 (w % 4) .. + 31, and
+//               the two warps of a group on the same lanes split the columns in halves.
 // A work unit is (N tile, group of MT M-tiles). With MT = 2 both slots hold one unit (M-tile j
 // in slot j); with MT = 1 consecutive units alternate slots so the epilogue of one overlaps the
 // MMAs of the next. Every wait is bounded: after a time limit the kernel raises TF_DEV_TIMEOUT,
@@ -38,7 +40,7 @@ constexpr uint64_t kWaitLimitNs = 2000000000ull;
 enum { EPI_LMHEAD = 0, EPI_GATEUP = 1, EPI_DOWN = 2, EPI_PARTIAL = 3 };
 
 struct EpiParams {
-    Partial* partials;           // LMHEAD: [n_rows, n_tiles]
+    Partials partials;           // LMHEAD: per (row, vocabulary block) summaries
     int V;
     float inv_temp;
     __nv_bfloat16* out;          // GATEUP: A [n_rows, ld_out]; DOWN: h' [n_rows, ld_out]
@@ -84,52 +86,55 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// Summary of one 32-column chunk of one row: logits of vocabulary ids v0 .. v0+31. The largest
-// value (with the smallest id among equals), the second-largest value and the sum of
-// exp(z - max) come from fixed trees over the 32 registers: the same instructions for every lane,
-// whatever the data (a per-lane sorted insertion would diverge across the warp's 32 rows).
-struct ChunkSum {
-    float mx, second, sum;
-    int id;
+// Summary of one 32-column chunk of one row: logits of vocabulary ids v0 .. v0+31. The three
+// largest values, the chunk-local offsets of the first two (the smaller id first among equals)
+// and the sum of exp(z - max) come from one fixed tree over the 32 registers: the same
+// instructions for every lane whatever the data (a per-lane sorted insertion would diverge across
+// the warp's 32 rows). Each node carries its subtree's top three and its sum of exp(z - node
+// max), so a logit is dead once its leaf is formed; the tree is expanded depth first to keep
+// few nodes live.
+struct ChunkNode {
+    float a1, a2, a3, s;  // a1 >= a2 >= a3; s = sum over the subtree of exp(z - a1)
+    int i1, i2;           // chunk-local offsets of a1, a2
 };
-__device__ __forceinline__ ChunkSum lmhead_chunk(const uint32_t (&r)[32], int v0, int V, float inv_temp) {
-    float v[32];
-#pragma unroll
-    for (int j = 0; j < 32; ++j) v[j] = (v0 + j < V) ? __uint_as_float(r[j]) * inv_temp : -INFINITY;
-    float a1[16], a2[16];
-    int ai[16];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-        const bool ge = v[2 * i] >= v[2 * i + 1];
-        a1[i] = ge ? v[2 * i] : v[2 * i + 1];
-        a2[i] = ge ? v[2 * i + 1] : v[2 * i];
-        ai[i] = ge ? 2 * i : 2 * i + 1;
+__device__ __forceinline__ float chunk_logit(uint32_t r, int v, int V, float inv_temp) {
+    return v < V ? __uint_as_float(r) * inv_temp : -INFINITY;
+}
+// p covers smaller ids than q, so on equal values p's entry ranks first.
+__device__ __forceinline__ ChunkNode chunk_merge(const ChunkNode& p, const ChunkNode& q) {
+    const bool pw = p.a1 >= q.a1;
+    const ChunkNode& w = pw ? p : q;
+    const ChunkNode& l = pw ? q : p;
+    // the winner's second against the loser's first; p's ids rank first on equal values
+    const bool sw = pw ? (w.a2 >= l.a1) : (w.a2 > l.a1);
+    ChunkNode n;
+    n.a1 = w.a1;
+    n.i1 = w.i1;
+    n.a2 = sw ? w.a2 : l.a1;
+    n.i2 = sw ? w.i2 : l.i1;
+    n.a3 = sw ? fmaxf(w.a3, l.a1) : fmaxf(w.a2, l.a2);
+    n.s = w.s + (l.a1 > -INFINITY ? l.s * __expf(l.a1 - w.a1) : 0.0f);
+    return n;
+}
+template <int OFF, int N>
+__device__ __forceinline__ ChunkNode chunk_tree(const uint32_t (&r)[32], int v0, int V, float inv_temp) {
+    if constexpr (N == 2) {
+        const float x = chunk_logit(r[OFF], v0 + OFF, V, inv_temp);
+        const float y = chunk_logit(r[OFF + 1], v0 + OFF + 1, V, inv_temp);
+        const bool ge = x >= y;
+        ChunkNode n;
+        n.a1 = ge ? x : y;
+        n.a2 = ge ? y : x;
+        n.i1 = ge ? OFF : OFF + 1;
+        n.i2 = ge ? OFF + 1 : OFF;
+        n.a3 = -INFINITY;
+        n.s = n.a1 > -INFINITY ? 1.0f + __expf(n.a2 - n.a1) : 0.0f;
+        return n;
+    } else {
+        const ChunkNode p = chunk_tree<OFF, N / 2>(r, v0, V, inv_temp);
+        const ChunkNode q = chunk_tree<OFF + N / 2, N / 2>(r, v0, V, inv_temp);
+        return chunk_merge(p, q);
     }
-#pragma unroll
-    for (int w = 8; w >= 1; w >>= 1) {
-#pragma unroll
-        for (int i = 0; i < w; ++i) {
-            const bool a_wins = a1[i] > a1[i + w] || (a1[i] == a1[i + w] && ai[i] < ai[i + w]);
-            const float n2 = a_wins ? fmaxf(a2[i], a1[i + w]) : fmaxf(a1[i], a2[i + w]);
-            a1[i] = a_wins ? a1[i] : a1[i + w];
-            ai[i] = a_wins ? ai[i] : ai[i + w];
-            a2[i] = n2;
-        }
-    }
-    ChunkSum c;
-    c.mx = a1[0];
-    c.second = a2[0];
-    c.id = a1[0] > -INFINITY ? v0 + ai[0] : -1;
-    float e[16];
-    const float mx = a1[0] > -INFINITY ? a1[0] : 0.0f;
-#pragma unroll
-    for (int j = 0; j < 16; ++j) e[j] = __expf(v[2 * j] - mx) + __expf(v[2 * j + 1] - mx);
-#pragma unroll
-    for (int w = 8; w >= 1; w >>= 1)
-#pragma unroll
-        for (int j = 0; j < w; ++j) e[j] += e[j + w];
-    c.sum = e[0];
-    return c;
 }
 
 template <int EPI, int MT, int NB, int BN, int STAGES>
@@ -304,25 +309,37 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
 
             if constexpr (EPI == EPI_LMHEAD) {
                 static_assert(BN == kBlockV, "one LM-head N tile is one vocabulary block");
-                // this warp's half of the block: chunks [h * kChunks / 2, (h + 1) * kChunks / 2)
+                // this warp's half of the block: chunks [half * 4, half * 4 + 4)
                 constexpr int kHalf = kChunks / 2;
-                Partial* p = ep.partials + static_cast<size_t>(row) * n_ntiles + nt;
+                const Partials& P = ep.partials;
                 // warps whose 32 rows are all padding skip the accumulators entirely
                 if (row - lane < n_rows) {
+                    float hm = -INFINITY, hsum = 0.0f, hbv = -INFINITY;
+                    int hbid = -1;
 #pragma unroll
                     for (int j = 0; j < kHalf; ++j) {
                         const int ci = half * kHalf + j;
+                        const int v0 = nt * BN + ci * kChunk;
                         uint32_t ra[32];
                         ptx::tmem_ld_32cols(tb + ci * kChunk, ra);
-                        const ChunkSum c = lmhead_chunk(ra, nt * BN + ci * kChunk, ep.V, ep.inv_temp);
-                        if (row < n_rows) {
-                            p->cmax[ci] = c.mx;
-                            p->cid[ci] = c.id;
-                            p->c2[ci] = c.second;
-                            p->cs[ci] = c.sum;
+                        const ChunkNode c = chunk_tree<0, 32>(ra, v0, ep.V, ep.inv_temp);
+                        // half summary; chunks arrive in id order, so strict > keeps the smaller id
+                        if (c.a1 > hbv) {
+                            hbv = c.a1;
+                            hbid = v0 + c.i1;
                         }
+                        if (c.a1 > -INFINITY) {
+                            const float mn = fmaxf(hm, c.a1);
+                            hsum = hsum * __expf(hm - mn) + c.s * __expf(c.a1 - mn);
+                            hm = mn;
+                        }
+                        if (row < n_rows)
+                            P.chunks[P.chunk_at(nt, ci, row)] =
+                                make_float4(c.a1, c.a2, c.a3, __int_as_float(c.i1 | (c.i2 << 8)));
                         __syncwarp();   // reconverge before the next warp-collective TMEM load
                     }
+                    if (row < n_rows)
+                        P.halves[P.half_at(nt, half, row)] = make_float4(hm, hsum, hbv, __int_as_float(hbid));
                 }
                 ptx::tc_fence_before();
                 ptx::mbar_arrive(&tempty[g]);
@@ -464,7 +481,7 @@ cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& t
 }  // namespace
 
 cudaError_t launch_lmhead_tc(const Ctx& ctx, const void* lm_head, const void* x, int n_rows, int d, int V,
-                             float inv_temp, Partial* partials) {
+                             float inv_temp, Partials partials) {
     if (n_rows <= 0) return cudaSuccess;
     CUtensorMap tx, tw;
     cudaError_t e = make_tmap(&tx, x, d, n_rows, kBK, kBM);

@@ -53,11 +53,11 @@ def test_static_scratch_limit_is_checked_before_any_gpu_work():
     # (TF_ERR_INVALID_ARG). Neither reaches the GPU.
     from paper_2606_03819_gb300 import binding as Bn
     lib = _lib()
-    V = 151936                      # 594 blocks of 256: 256 + rows * 594 * 128 <= 8 MiB <=> rows <= 110
-    assert _call_static_raw(lib, _dims(batch=111, gamma=1, d=4096, V=V, dtype="bf16")) == Bn.TF_ERR_UNSUPPORTED
-    assert _call_static_raw(lib, _dims(batch=37, gamma=3, d=4096, V=V, dtype="bf16")) == Bn.TF_ERR_UNSUPPORTED
-    assert _call_static_raw(lib, _dims(batch=110, gamma=1, d=4096, V=V, dtype="bf16")) == Bn.TF_ERR_INVALID_ARG
-    assert _call_static_raw(lib, _dims(batch=11, gamma=10, d=4096, V=V, dtype="bf16")) == Bn.TF_ERR_INVALID_ARG
+    V = 151936                      # 594 blocks of 256, 160 bytes each per row: rows <= 88 fit in 8 MiB
+    assert _call_static_raw(lib, _dims(batch=89, gamma=1, d=4096, V=V, dtype="bf16")) == Bn.TF_ERR_UNSUPPORTED
+    assert _call_static_raw(lib, _dims(batch=30, gamma=3, d=4096, V=V, dtype="bf16")) == Bn.TF_ERR_UNSUPPORTED
+    assert _call_static_raw(lib, _dims(batch=88, gamma=1, d=4096, V=V, dtype="bf16")) == Bn.TF_ERR_INVALID_ARG
+    assert _call_static_raw(lib, _dims(batch=11, gamma=8, d=4096, V=V, dtype="bf16")) == Bn.TF_ERR_INVALID_ARG
     # invalid dims are rejected as by the workspace calls
     assert _call_static_raw(lib, _dims(V=8, K2=12)) == Bn.TF_ERR_INVALID_ARG
     assert _call_static_raw(lib, _dims(dtype="bf16", d=100)) == Bn.TF_ERR_UNSUPPORTED
@@ -135,11 +135,11 @@ def test_static_matches_workspace_call_on_two_calls_in_a_row(name, kw):
 
 @pytest.mark.gpu
 def test_static_at_its_size_limit():
-    # the largest request the scratch holds at the 151936-entry vocabulary: 110 rows
+    # the largest request the scratch holds at the 151936-entry vocabulary: 88 rows
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     _lib()
-    dims = _dims(batch=11, gamma=10, d=4096, V=151936, M=8, K2=32, dtype="bf16")
+    dims = _dims(batch=11, gamma=8, d=4096, V=151936, M=8, K2=32, dtype="bf16")
     gen = torch.Generator(device="cuda").manual_seed(99)
     w = _weights(dims, gen)
     for call in range(2):
