@@ -112,24 +112,39 @@ __host__ __device__ inline size_t tree_smem_lists(int mode, int gamma, int R, in
 }
 constexpr size_t kTreeSmemLimit = 200 * 1024;
 
-__global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, int stage_lists) {
-    extern __shared__ __align__(16) uint8_t smem_raw[];
-    const int cap = a.B + 2;
-    const int n_out = a.B + 1;
-    unsigned long long* qkey = reinterpret_cast<unsigned long long*>(smem_raw);
-    float* qps = reinterpret_cast<float*>(qkey + cap);
-    int* qrow = reinterpret_cast<int*>(qps + cap);
-    int* qrank = qrow + cap;
-    int* qtok = qrank + cap;
-    int* o_tok = qtok + cap;
-    int* o_par = o_tok + n_out;
-    int* o_dep = o_par + n_out;
-    float* o_score = reinterpret_cast<float*>(o_dep + n_out);
-    int* topm = reinterpret_cast<int*>(o_score + n_out);          // [gamma, M]
-    uint8_t* lists = reinterpret_cast<uint8_t*>(
-        (reinterpret_cast<uintptr_t>(topm + a.gamma * a.M) + 15) & ~static_cast<uintptr_t>(15));
+// Shared memory of both builders: queue arrays (used by the general builder only), output nodes,
+// stage-1 top-M and the staged child lists.
+struct TreeSmem {
+    unsigned long long* qkey;
+    float* qps;
+    int *qrow, *qrank, *qtok;
+    int *o_tok, *o_par, *o_dep;
+    float* o_score;
+    int* topm;        // [gamma, M]
+    uint8_t* lists;   // ids [rows][stride] int32, then log-probs [rows][stride] float
+};
+__device__ __forceinline__ TreeSmem tree_smem(uint8_t* base, const TreeArgs& a) {
+    TreeSmem t;
+    const int cap = a.B + 2, n_out = a.B + 1;
+    t.qkey = reinterpret_cast<unsigned long long*>(base);
+    t.qps = reinterpret_cast<float*>(t.qkey + cap);
+    t.qrow = reinterpret_cast<int*>(t.qps + cap);
+    t.qrank = t.qrow + cap;
+    t.qtok = t.qrank + cap;
+    t.o_tok = t.qtok + cap;
+    t.o_par = t.o_tok + n_out;
+    t.o_dep = t.o_par + n_out;
+    t.o_score = reinterpret_cast<float*>(t.o_dep + n_out);
+    t.topm = reinterpret_cast<int*>(t.o_score + n_out);
+    t.lists = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(t.topm + a.gamma * a.M) + 15) &
+                                         ~static_cast<uintptr_t>(15));
+    return t;
+}
 
-    const int s = blockIdx.x;
+// Stage sequence s's stage-1 top-M and, when stage_lists, its child lists (every pop then
+// touches shared memory only); returns where the lists are read from.
+__device__ __forceinline__ void stage_sequence(const TreeArgs& a, int s, const TreeSmem& t, int stage_lists,
+                                               const int32_t** ids_base, const float** lp_base) {
     const int tid = threadIdx.x;
     const bool ar = a.mode == TF_MODE_AR;
     const int n_rows_l = ar ? a.R : a.gamma;
@@ -138,51 +153,88 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
                               : a.top_ids + static_cast<size_t>(s) * a.gamma * a.K1;
     const float* g_lp = ar ? a.child_logp + static_cast<size_t>(s) * a.R * a.K2
                            : a.top_logp + static_cast<size_t>(s) * a.gamma * a.K1;
-    const int32_t* ids_base = g_ids;
-    const float* lp_base = g_lp;
-    // stage the sequence's child lists and stage-1 top-M (every pop then touches shared memory only)
+    *ids_base = g_ids;
+    *lp_base = g_lp;
     for (int i = tid; i < a.gamma * a.M; i += kTreeThreads)
-        topm[i] = a.top_ids[(static_cast<size_t>(s) * a.gamma + i / a.M) * a.K1 + i % a.M];
-    if (stage_lists) {
-        const int n = n_rows_l * stride;
-        int32_t* si = reinterpret_cast<int32_t*>(lists);
-        float* sl = reinterpret_cast<float*>(si + n);
-        const bool vec = ((reinterpret_cast<uintptr_t>(g_ids) | reinterpret_cast<uintptr_t>(g_lp) |
-                           reinterpret_cast<uintptr_t>(si) | reinterpret_cast<uintptr_t>(sl)) & 15) == 0 &&
-                         (n & 3) == 0;
-        if (vec) {
-            // 16-byte copies, four per thread in flight before the first store
-            const int4* gi = reinterpret_cast<const int4*>(g_ids);
-            const float4* gl = reinterpret_cast<const float4*>(g_lp);
-            int4* di = reinterpret_cast<int4*>(si);
-            float4* dl = reinterpret_cast<float4*>(sl);
-            const int n4 = n >> 2;
-            constexpr int T = kTreeThreads;
-            int i = tid;
-            for (; i + 3 * T < n4; i += 4 * T) {       // 8 loads in flight, then 8 stores
-                const int4 a0 = gi[i], a1 = gi[i + T], a2 = gi[i + 2 * T], a3 = gi[i + 3 * T];
-                const float4 b0 = gl[i], b1 = gl[i + T], b2 = gl[i + 2 * T], b3 = gl[i + 3 * T];
-                di[i] = a0; di[i + T] = a1; di[i + 2 * T] = a2; di[i + 3 * T] = a3;
-                dl[i] = b0; dl[i + T] = b1; dl[i + 2 * T] = b2; dl[i + 3 * T] = b3;
-            }
-            for (; i < n4; i += T) {
-                const int4 a = gi[i];
-                const float4 b = gl[i];
-                di[i] = a;
-                dl[i] = b;
-            }
-        } else {
-#pragma unroll 8
-            for (int i = tid; i < n; i += kTreeThreads) {
-                const int32_t a = g_ids[i];
-                const float b = g_lp[i];
-                si[i] = a;
-                sl[i] = b;
-            }
+        t.topm[i] = a.top_ids[(static_cast<size_t>(s) * a.gamma + i / a.M) * a.K1 + i % a.M];
+    if (!stage_lists) return;
+    const int n = n_rows_l * stride;
+    int32_t* si = reinterpret_cast<int32_t*>(t.lists);
+    float* sl = reinterpret_cast<float*>(si + n);
+    const bool vec = ((reinterpret_cast<uintptr_t>(g_ids) | reinterpret_cast<uintptr_t>(g_lp) |
+                       reinterpret_cast<uintptr_t>(si) | reinterpret_cast<uintptr_t>(sl)) & 15) == 0 &&
+                     (n & 3) == 0;
+    if (vec) {
+        // 16-byte copies, sixteen per thread in flight before the first store
+        const int4* gi = reinterpret_cast<const int4*>(g_ids);
+        const float4* gl = reinterpret_cast<const float4*>(g_lp);
+        int4* di = reinterpret_cast<int4*>(si);
+        float4* dl = reinterpret_cast<float4*>(sl);
+        const int n4 = n >> 2;
+        constexpr int T = kTreeThreads;
+        for (int base = tid; base < n4; base += 8 * T) {
+            int4 va[8];
+            float4 vb[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                if (base + j * T < n4) {
+                    va[j] = gi[base + j * T];
+                    vb[j] = gl[base + j * T];
+                }
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                if (base + j * T < n4) {
+                    di[base + j * T] = va[j];
+                    dl[base + j * T] = vb[j];
+                }
         }
-        ids_base = si;
-        lp_base = sl;
+    } else {
+#pragma unroll 8
+        for (int i = tid; i < n; i += kTreeThreads) {
+            const int32_t v = g_ids[i];
+            const float w = g_lp[i];
+            si[i] = v;
+            sl[i] = w;
+        }
     }
+    *ids_base = si;
+    *lp_base = sl;
+}
+
+// Nodes from shared memory to the outputs.
+__device__ __forceinline__ void write_nodes(const TreeArgs& a, int s, const TreeSmem& t) {
+    const int n_out = a.B + 1;
+    for (int i = threadIdx.x; i < n_out; i += kTreeThreads) {
+        const size_t o = static_cast<size_t>(s) * n_out + i;
+        a.node_tok[o] = t.o_tok[i];
+        a.node_parent[o] = t.o_par[i];
+        a.node_depth[o] = t.o_dep[i];
+        a.node_score[o] = t.o_score[i];
+    }
+}
+
+// General builder (any B): the queue in shared memory.
+__global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, int stage_lists) {
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    const TreeSmem t = tree_smem(smem_raw, a);
+    unsigned long long* qkey = t.qkey;
+    float* qps = t.qps;
+    int* qrow = t.qrow;
+    int* qrank = t.qrank;
+    int* qtok = t.qtok;
+    int* o_tok = t.o_tok;
+    int* o_par = t.o_par;
+    int* o_dep = t.o_dep;
+    float* o_score = t.o_score;
+    int* topm = t.topm;
+    const int n_out = a.B + 1;
+    const int s = blockIdx.x;
+    const int tid = threadIdx.x;
+    const bool ar = a.mode == TF_MODE_AR;
+    const int stride = ar ? a.K2 : a.K1;
+    const int32_t* ids_base;
+    const float* lp_base;
+    stage_sequence(a, s, t, stage_lists, &ids_base, &lp_base);
     __syncthreads();
 
     if (tid < 32) {
@@ -295,13 +347,150 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
         if (lane == 0) a.dev_status[s] = flags;
     }
     __syncthreads();
-    for (int i = tid; i < n_out; i += kTreeThreads) {
-        const size_t o = static_cast<size_t>(s) * n_out + i;
-        a.node_tok[o] = o_tok[i];
-        a.node_parent[o] = o_par[i];
-        a.node_depth[o] = o_dep[i];
-        a.node_score[o] = o_score[i];
+    write_nodes(a, s, t);
+}
+
+// Builder for B + 1 <= 32 S: the queue in registers, S slots per lane (slot j on lane j % 32,
+// register j / 32). Slots are appended in pop order and an exhausted list leaves an empty slot
+// (key 0, below every real key), so no entry ever moves. Pops, tie rules and results are those
+// of build_tree_kernel.
+template <int S>
+__global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a, int stage_lists) {
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    const TreeSmem t = tree_smem(smem_raw, a);
+    const int n_out = a.B + 1;
+    const int s = blockIdx.x;
+    const bool ar = a.mode == TF_MODE_AR;
+    const int stride = ar ? a.K2 : a.K1;
+    const int32_t* ids_base;
+    const float* lp_base;
+    stage_sequence(a, s, t, stage_lists, &ids_base, &lp_base);
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        const int lane = threadIdx.x;
+        constexpr unsigned kFull = 0xffffffffu;
+        int flags = 0;
+        const int root = a.root_tok[s];
+        if (root < 0 || root >= a.V) flags |= TF_DEV_BAD_TOKEN;
+        const int list_len = a.K2;
+        unsigned long long key[S];
+        int srow[S], srank[S], stok[S];
+        float spsc[S];
+#pragma unroll
+        for (int j = 0; j < S; ++j) {
+            key[j] = 0ull;
+            srow[j] = srank[j] = stok[j] = 0;
+            spsc[j] = 0.0f;
+        }
+        if (lane == 0) {
+            key[0] = queue_key(lp_base[0], 1, 0);
+            stok[0] = ids_base[0];
+            t.o_tok[0] = root;
+            t.o_par[0] = -1;
+            t.o_dep[0] = 0;
+            t.o_score[0] = 0.0f;
+        }
+        int n_e = 1;      // slots used so far
+        int count = 1;    // nodes placed
+        while (count < n_out) {
+            // this lane's best slot and its entry
+            unsigned long long lb = key[0];
+            int brow = srow[0], brank = srank[0], btok = stok[0];
+            float bpsc = spsc[0];
+#pragma unroll
+            for (int j = 1; j < S; ++j)
+                if (key[j] > lb) {
+                    lb = key[j];
+                    brow = srow[j];
+                    brank = srank[j];
+                    btok = stok[j];
+                    bpsc = spsc[j];
+                }
+            const uint32_t hi = static_cast<uint32_t>(lb >> 32), lo = static_cast<uint32_t>(lb);
+            const uint32_t mhi = __reduce_max_sync(kFull, hi);
+            if (mhi == 0u) break;                      // queue empty (every real key has hi > 0)
+            unsigned win = __ballot_sync(kFull, hi == mhi);
+            if (__popc(win) > 1) {
+                const uint32_t mlo = __reduce_max_sync(kFull, hi == mhi ? lo : 0u);
+                win = __ballot_sync(kFull, hi == mhi && lo == mlo);
+            }
+            const int wl = __ffs(win) - 1;
+            const uint32_t wlo = __shfl_sync(kFull, lo, wl);
+            const int row = __shfl_sync(kFull, brow, wl);
+            const int rank = __shfl_sync(kFull, brank, wl);
+            const int tok = __shfl_sync(kFull, btok, wl);
+            const float psc = __shfl_sync(kFull, bpsc, wl);
+            const float sc = key_float(mhi);
+            const int dep = 127 - static_cast<int>(wlo >> 24);
+            const int par = 0xFFFFFF - static_cast<int>(wlo & 0xFFFFFFu);
+            const int node = count++;
+            if (tok < 0 || tok >= a.V) flags |= TF_DEV_BAD_TOKEN;
+            if (!isfinite(sc)) flags |= TF_DEV_NONFINITE;
+            // expandable? (depth cap; M-ary rule via one compare per lane)
+            int crow = -1;
+            if (dep < a.gamma) {
+                if (a.mode == TF_MODE_MARGINAL) {
+                    crow = dep;
+                } else {
+                    const bool hit = lane < a.M && t.topm[(dep - 1) * a.M + lane] == tok;
+                    const unsigned bal = __ballot_sync(kFull, hit);
+                    if (bal) crow = ar ? 1 + (dep - 1) * a.M + (__ffs(bal) - 1) : dep;
+                }
+            }
+            // next sibling of the popped entry, and the first child of the new node (the same
+            // shared-memory words for every lane)
+            const bool sibling = rank + 1 < list_len;
+            unsigned long long sib_key = 0ull;
+            int sib_tok = 0;
+            if (sibling) {
+                const size_t at = static_cast<size_t>(row) * stride + rank + 1;
+                sib_tok = ids_base[at];
+                sib_key = queue_key(psc + lp_base[at], dep, par);
+            }
+            if (lane == wl) {
+                // the winner's best slot is the one holding its best key (keys are unique)
+#pragma unroll
+                for (int j = 0; j < S; ++j) {
+                    const bool m = key[j] == lb;
+                    key[j] = m ? sib_key : key[j];
+                    srank[j] = m ? rank + 1 : srank[j];
+                    stok[j] = m ? sib_tok : stok[j];
+                }
+            }
+            if (crow >= 0) {
+                const size_t at = static_cast<size_t>(crow) * stride;
+                const int ctok = ids_base[at];
+                const unsigned long long ckey = queue_key(sc + lp_base[at], dep + 1, node);
+                const bool mine = lane == (n_e & 31);
+#pragma unroll
+                for (int j = 0; j < S; ++j) {
+                    const bool m = mine && j == (n_e >> 5);
+                    key[j] = m ? ckey : key[j];
+                    srow[j] = m ? crow : srow[j];
+                    srank[j] = m ? 0 : srank[j];
+                    stok[j] = m ? ctok : stok[j];
+                    spsc[j] = m ? sc : spsc[j];
+                }
+                ++n_e;
+            }
+            if (lane == 0) {
+                t.o_tok[node] = tok;
+                t.o_par[node] = par;
+                t.o_dep[node] = dep;
+                t.o_score[node] = sc;
+            }
+        }
+        if (count < n_out) flags |= TF_DEV_UNDERFULL;
+        for (int i = count + lane; i < n_out; i += 32) {
+            t.o_tok[i] = -1;
+            t.o_par[i] = -1;
+            t.o_dep[i] = -1;
+            t.o_score[i] = -INFINITY;
+        }
+        if (lane == 0) a.dev_status[s] = flags;
     }
+    __syncthreads();
+    write_nodes(a, s, t);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -362,16 +551,47 @@ __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __
 
 }  // namespace
 
-// bf16 rows with d % 8 == 0: 16-byte loads and stores, 8 elements per thread and step. The
-// normalisation is evaluated in fp64 (one square root per row, d multiplies) and rounded once to
-// bf16, so x is the correctly rounded value of the definition: an x element off by one bf16 ulp
-// would perturb every gate/up output and flip many later roundings.
+// Error-free sum (Knuth's TwoSum): s + c tracks a running sum to about twice fp32 precision.
+__device__ __forceinline__ void two_sum_acc(float& s, float& c, float x) {
+    const float t = s + x;
+    const float z = t - s;
+    c += (s - (t - z)) + (x - z);
+    s = t;
+}
+
+// bf16 nearest-even rounding of the real value r + t, where r is an fp32 value and |t| is below
+// two fp32 ulps of r. Only an r within a few ulps of a bf16 midpoint can round differently from
+// r alone; for those the side of the midpoint is decided from (r - midpoint) + t, where
+// r - midpoint is exact (both share r's binade).
+__device__ __forceinline__ __nv_bfloat16 bf16_round_sum(float r, float t) {
+    const uint32_t u = __float_as_uint(r);
+    const uint32_t low = u & 0xffffu;
+    if ((u & 0x7f800000u) == 0x7f800000u || low < 0x8000u - 4u || low > 0x8000u + 4u) return __float2bfloat16_rn(r);
+    const uint32_t trunc = u & 0xffff0000u;
+    const float mid = __uint_as_float(trunc | 0x8000u);
+    const float dm = (r - mid) + t;
+    const float away = (u & 0x80000000u) ? -dm : dm;   // > 0: beyond the midpoint in magnitude
+    uint32_t bits = trunc;
+    if (away > 0.0f || (away == 0.0f && (trunc & 0x10000u))) bits += 0x10000u;
+    return __ushort_as_bfloat16(static_cast<unsigned short>(bits >> 16));
+}
+
+// bf16 rows with d % 8 == 0: 16-byte loads and stores, 8 elements per thread and step. x is the
+// correctly rounded bf16 value of the definition (an element off by one bf16 ulp would perturb
+// every gate/up output and flip many later roundings), computed without per-element fp64 work:
+//  - mean(h^2): every square of a bf16 value is exact in fp32; the sums are compensated
+//    (TwoSum), widened to fp64 only once per thread for the block reduction;
+//  - 1 / sqrt(mean + eps) in fp64 once per row, split into fp32 hi + lo;
+//  - h * w is exact in fp32 (two 8-bit significands); (h w) * hi is rounded once and its
+//    rounding error recovered with an FMA, so (h w) / sqrt(mean + eps) is known as r + t to
+//    about 2^-47 relative, which decides the bf16 rounding (bf16_round_sum).
 __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
     const uint4* __restrict__ hidden, const uint4* __restrict__ embed, const uint4* __restrict__ norm_h,
     const uint4* __restrict__ norm_e, const int32_t* __restrict__ root_tok, const int32_t* __restrict__ top_ids,
     int gamma, int M, int K1, int R, int d, int V, float eps, uint4* __restrict__ X, int* status) {
     constexpr int kMaxPerThread = 4;          // d <= 256 * 8 * 4 = 8192
     __shared__ double red[2][8];
+    __shared__ float scale[4];                // hi, lo of the hidden half; hi, lo of the embedding half
     const int row = blockIdx.x;
     const int sq = row / R, r = row - sq * R;
     const int hid = sq * gamma + stage2_hidden_index(r, M);
@@ -384,7 +604,6 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
     const uint4* h = hidden + static_cast<size_t>(hid) * dv;
     const uint4* e = embed + static_cast<size_t>(tok) * dv;
     uint4 hv[kMaxPerThread], ev[kMaxPerThread];
-    double sh = 0.0, se = 0.0;
 #pragma unroll
     for (int i = 0; i < kMaxPerThread; ++i) {
         const int c = threadIdx.x + i * 256;
@@ -393,6 +612,7 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
             ev[i] = e[c];
         }
     }
+    float sh = 0.0f, ch = 0.0f, se = 0.0f, ce = 0.0f;
 #pragma unroll
     for (int i = 0; i < kMaxPerThread; ++i) {
         const int c = threadIdx.x + i * 256;
@@ -401,34 +621,35 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
             const __nv_bfloat16* eb = reinterpret_cast<const __nv_bfloat16*>(&ev[i]);
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
-                const double a = __bfloat162float(hb[j]), b = __bfloat162float(eb[j]);
-                sh = fma(a, a, sh);
-                se = fma(b, b, se);
+                const float a = __bfloat162float(hb[j]), b = __bfloat162float(eb[j]);
+                two_sum_acc(sh, ch, a * a);
+                two_sum_acc(se, ce, b * b);
             }
         }
     }
+    double dh = static_cast<double>(sh) + static_cast<double>(ch);
+    double de = static_cast<double>(se) + static_cast<double>(ce);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
-        sh += __shfl_xor_sync(0xffffffffu, sh, o);
-        se += __shfl_xor_sync(0xffffffffu, se, o);
+        dh += __shfl_xor_sync(0xffffffffu, dh, o);
+        de += __shfl_xor_sync(0xffffffffu, de, o);
     }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0) {
-        red[0][warp] = sh;
-        red[1][warp] = se;
+        red[0][warp] = dh;
+        red[1][warp] = de;
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-        double a = 0.0, b = 0.0;
-        for (int w = 0; w < 8; ++w) {
-            a += red[0][w];
-            b += red[1][w];
-        }
-        red[0][0] = 1.0 / sqrt(a / d + static_cast<double>(eps));
-        red[1][0] = 1.0 / sqrt(b / d + static_cast<double>(eps));
+    if (threadIdx.x < 2) {
+        double a = 0.0;
+        for (int w = 0; w < 8; ++w) a += red[threadIdx.x][w];
+        const double inv = 1.0 / sqrt(a / d + static_cast<double>(eps));
+        const float hi = __double2float_rn(inv);
+        scale[2 * threadIdx.x] = hi;
+        scale[2 * threadIdx.x + 1] = __double2float_rn(inv - static_cast<double>(hi));
     }
     __syncthreads();
-    const double ih = red[0][0], ie = red[1][0];
+    const float ih = scale[0], ih_lo = scale[1], ie = scale[2], ie_lo = scale[3];
     uint4* xr = X + static_cast<size_t>(row) * 2 * dv;
 #pragma unroll
     for (int i = 0; i < kMaxPerThread; ++i) {
@@ -444,10 +665,11 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
             __nv_bfloat16* oeb = reinterpret_cast<__nv_bfloat16*>(&oe);
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
-                ohb[j] = __double2bfloat16(static_cast<double>(__bfloat162float(hb[j])) * ih *
-                                           static_cast<double>(__bfloat162float(whb[j])));
-                oeb[j] = __double2bfloat16(static_cast<double>(__bfloat162float(eb[j])) * ie *
-                                           static_cast<double>(__bfloat162float(web[j])));
+                const float ph = __bfloat162float(hb[j]) * __bfloat162float(whb[j]);
+                const float pe = __bfloat162float(eb[j]) * __bfloat162float(web[j]);
+                const float rh = ph * ih, re = pe * ie;
+                ohb[j] = bf16_round_sum(rh, fmaf(ph, ih_lo, fmaf(ph, ih, -rh)));
+                oeb[j] = bf16_round_sum(re, fmaf(pe, ie_lo, fmaf(pe, ie, -re)));
             }
             xr[c] = oh;
             xr[dv + c] = oe;
@@ -489,10 +711,15 @@ cudaError_t launch_build_tree(const Ctx& ctx, int b, int gamma, int M, int K1, i
     const size_t lists = tree_smem_lists(mode, gamma, R, K1, K2);
     const int stage = fixed + lists <= kTreeSmemLimit ? 1 : 0;
     const size_t smem = fixed + (stage ? lists : 0);
-    cudaError_t e = cudaFuncSetAttribute(build_tree_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+    // the register-queue builder whenever B + 1 slots fit in four registers per lane
+    void (*kern)(TreeArgs, int) = B + 1 <= 32 ? build_tree_reg_kernel<1>
+                                  : B + 1 <= 64 ? build_tree_reg_kernel<2>
+                                  : B + 1 <= 96 ? build_tree_reg_kernel<3>
+                                  : B + 1 <= 128 ? build_tree_reg_kernel<4>
+                                                 : build_tree_kernel;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    build_tree_kernel<<<b, kTreeThreads, smem, ctx.stream>>>(a, stage);
+    kern<<<b, kTreeThreads, smem, ctx.stream>>>(a, stage);
     return cudaGetLastError();
 }
 
