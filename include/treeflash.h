@@ -109,6 +109,11 @@ const char* tf_status_string(tf_status status);
 /* Library version as major*10000 + minor*100 + patch. */
 int32_t tf_version(void);
 
+/* Number of kernels this library has launched in the calling process since it was loaded, over
+ * all devices and streams (a host-side counter; host only, no GPU work). Lets a caller count
+ * the kernels of a timed region: read it before and after. */
+uint64_t tf_kernel_launches(void);
+
 /* Validate `dims` and return the workspace bytes every call below needs for these dims
  * (the maximum over all calls, so one buffer serves the whole step). Host only; no GPU
  * work. The workspace must be device memory, 256-byte aligned, and must not be used by two

@@ -43,7 +43,7 @@ class TfWeights(ctypes.Structure):
                 ("lm_head", "embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down")]
 
 
-EXPORTS = ("tf_status_string", "tf_version", "tf_workspace_size", "tf_status_reset", "tf_status_read",
+EXPORTS = ("tf_status_string", "tf_version", "tf_kernel_launches", "tf_workspace_size", "tf_status_reset", "tf_status_read",
            "tf_stage1_marginals", "tf_stage2_ar_approx", "tf_build_tree", "tf_tree_mask",
            "tf_draft_tree_host", "tf_lmhead_partials", "tf_lmhead_merge", "tf_ar_approx",
            "tf_workspace_h_prime", "tf_workspace_view", "tf_stage1_marginals_static")
@@ -66,6 +66,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     sig = {
         "tf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
         "tf_version": (I32, []),
+        "tf_kernel_launches": (ctypes.c_uint64, []),
         "tf_workspace_size": (ctypes.c_int, [D, ctypes.POINTER(SZ)]),
         "tf_status_reset": (ctypes.c_int, [P, SZ, P]),
         "tf_status_read": (ctypes.c_int, [P, SZ, ctypes.POINTER(I32), P]),
@@ -155,6 +156,11 @@ def weights_struct(w: dict) -> TfWeights:
 
 def tf_version() -> int:
     return load_library().tf_version()
+
+
+def tf_kernel_launches() -> int:
+    """Kernels launched by the library so far in this process."""
+    return int(load_library().tf_kernel_launches())
 
 
 def tf_workspace_size(dims: Dims) -> int:

@@ -1,16 +1,22 @@
 // C ABI of the TreeFlash drafting path (declared in include/treeflash.h): argument checks,
-// workspace layout and the kernel sequence of every call. No allocation, no global state
-// besides the cached driver entry point used to build TMA descriptors.
+// workspace layout and the kernel sequence of every call. No allocation; the only global state
+// is the cached driver entry point used to build TMA descriptors and a launch counter.
 #include <math.h>
 #include <string.h>
 
 #include <algorithm>
+#include <atomic>
 
 #include "common.cuh"
 
 namespace tf {
 size_t merge_smem_bytes(int n_tiles, int d);
+
+namespace {
+std::atomic<unsigned long long> g_kernel_launches{0};
 }
+void note_launch() { g_kernel_launches.fetch_add(1, std::memory_order_relaxed); }
+}  // namespace tf
 
 namespace {
 
@@ -224,6 +230,8 @@ const char* tf_status_string(tf_status s) {
 }
 
 int32_t tf_version(void) { return 100; }
+
+uint64_t tf_kernel_launches(void) { return tf::g_kernel_launches.load(std::memory_order_relaxed); }
 
 tf_status tf_workspace_size(const tf_dims* dims, size_t* bytes) {
     if (!bytes) return TF_ERR_INVALID_ARG;

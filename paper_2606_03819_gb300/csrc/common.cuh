@@ -85,6 +85,37 @@ __host__ __device__ __forceinline__ int stage2_hidden_index(int r, int M) {
     return r == 0 ? 0 : (r - 1) / M + 1;
 }
 
+// ---- programmatic dependent launch ---------------------------------------------------------
+// Every kernel of the path is launched so that it may start while the previous kernel on the
+// stream is finishing. pdl_wait() blocks until the previous kernel has completed and its writes
+// are visible; each kernel calls it, on every path, before it reads anything an earlier kernel
+// wrote or writes anything an earlier kernel may still read. Only reads of the weights (which
+// no kernel writes) and on-chip set-up come before it. pdl_trigger() lets the next kernel be
+// scheduled; where it is called only decides how early the next kernel's set-up may overlap.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" :::); }
+
+// Host-side count of kernels launched by this library (tf_kernel_launches).
+void note_launch();
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                       Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+    if (e == cudaSuccess) note_launch();
+    return e;
+}
+
 }  // namespace tf
 
 // ---- launchers (one per kernel family); implemented in the .cu files -------------------------

@@ -182,6 +182,8 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
                                                                 const T* __restrict__ lm_head,
                                                                 const T* __restrict__ x, int32_t* __restrict__ out_ids,
                                                                 float* __restrict__ out_logp, int* status) {
+    pdl_trigger();
+    pdl_wait();
     extern __shared__ __align__(16) uint8_t dsm[];
     MergeSmem S;
     merge_layout(n_tiles, d, dsm, &S);
@@ -387,17 +389,18 @@ cudaError_t launch_lmhead_merge(const Ctx& ctx, int dtype, Partials partials, in
         auto kern = lmhead_merge_kernel<__nv_bfloat16>;
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
         if (e != cudaSuccess) return e;
-        kern<<<n_rows, kThreads, smem, ctx.stream>>>(partials, n_rows, n_tiles, V, d, k, inv_temp,
-                                                     static_cast<const __nv_bfloat16*>(lm_head),
-                                                     static_cast<const __nv_bfloat16*>(x), out_ids, out_logp,
-                                                     ctx.status);
+        e = launch_pdl(kern, dim3(n_rows), dim3(kThreads), smem, ctx.stream, partials, n_rows, n_tiles, V, d, k,
+                       inv_temp, static_cast<const __nv_bfloat16*>(lm_head), static_cast<const __nv_bfloat16*>(x),
+                       out_ids, out_logp, ctx.status);
+        if (e != cudaSuccess) return e;
     } else {
         auto kern = lmhead_merge_kernel<float>;
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
         if (e != cudaSuccess) return e;
-        kern<<<n_rows, kThreads, smem, ctx.stream>>>(partials, n_rows, n_tiles, V, d, k, inv_temp,
-                                                     static_cast<const float*>(lm_head), static_cast<const float*>(x),
-                                                     out_ids, out_logp, ctx.status);
+        e = launch_pdl(kern, dim3(n_rows), dim3(kThreads), smem, ctx.stream, partials, n_rows, n_tiles, V, d, k,
+                       inv_temp, static_cast<const float*>(lm_head), static_cast<const float*>(x), out_ids, out_logp,
+                       ctx.status);
+        if (e != cudaSuccess) return e;
     }
     return cudaGetLastError();
 }

@@ -17,6 +17,8 @@ __device__ __forceinline__ float silu_f(float g) { return g / (1.0f + __expf(-g)
 // partial [ks][rows][2I] (gate in columns [0, I), up in [I, 2I)) -> A [rows][I]
 __global__ void __launch_bounds__(256) swiglu_reduce_kernel(const float4* __restrict__ partial, int ks, int rows,
                                                             int I, __nv_bfloat162* __restrict__ A) {
+    pdl_trigger();
+    pdl_wait();
     const int i4 = I / 4;
     const size_t n = static_cast<size_t>(rows) * i4;
     const size_t split = static_cast<size_t>(rows) * 2 * i4;
@@ -38,6 +40,8 @@ __global__ void __launch_bounds__(256) swiglu_reduce_kernel(const float4* __rest
 __global__ void __launch_bounds__(256) down_reduce_kernel(const float4* __restrict__ partial, int ks, int rows, int d,
                                                           const __nv_bfloat162* __restrict__ hidden, int R, int M,
                                                           int gamma, __nv_bfloat162* __restrict__ hp) {
+    pdl_trigger();
+    pdl_wait();
     const int d4 = d / 4;
     const size_t n = static_cast<size_t>(rows) * d4;
     const size_t split = n;
@@ -66,18 +70,20 @@ int grid_for(size_t n, const Ctx& ctx) {
 cudaError_t launch_swiglu_reduce(const Ctx& ctx, const float* partial, int k_splits, int n_rows, int I,
                                  __nv_bfloat16* A) {
     const size_t n = static_cast<size_t>(n_rows) * (I / 4);
-    swiglu_reduce_kernel<<<grid_for(n, ctx), 256, 0, ctx.stream>>>(reinterpret_cast<const float4*>(partial), k_splits,
-                                                                   n_rows, I, reinterpret_cast<__nv_bfloat162*>(A));
-    return cudaGetLastError();
+    const cudaError_t e = launch_pdl(swiglu_reduce_kernel, dim3(grid_for(n, ctx)), dim3(256), 0, ctx.stream,
+                                     reinterpret_cast<const float4*>(partial), k_splits, n_rows, I,
+                                     reinterpret_cast<__nv_bfloat162*>(A));
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_down_reduce(const Ctx& ctx, const float* partial, int k_splits, int n_rows, int d,
                                const __nv_bfloat16* hidden, int R, int M, int gamma, __nv_bfloat16* h_prime) {
     const size_t n = static_cast<size_t>(n_rows) * (d / 4);
-    down_reduce_kernel<<<grid_for(n, ctx), 256, 0, ctx.stream>>>(
-        reinterpret_cast<const float4*>(partial), k_splits, n_rows, d,
-        reinterpret_cast<const __nv_bfloat162*>(hidden), R, M, gamma, reinterpret_cast<__nv_bfloat162*>(h_prime));
-    return cudaGetLastError();
+    const cudaError_t e = launch_pdl(down_reduce_kernel, dim3(grid_for(n, ctx)), dim3(256), 0, ctx.stream,
+                                     reinterpret_cast<const float4*>(partial), k_splits, n_rows, d,
+                                     reinterpret_cast<const __nv_bfloat162*>(hidden), R, M, gamma,
+                                     reinterpret_cast<__nv_bfloat162*>(h_prime));
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace tf

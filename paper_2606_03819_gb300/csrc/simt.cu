@@ -18,6 +18,8 @@ constexpr int kKChunk = 32;
 __global__ void __launch_bounds__(256) lmhead_simt_kernel(const float* __restrict__ W, const float* __restrict__ X,
                                                           int n_rows, int d, int V, float inv_temp,
                                                           Partials partials, int n_tiles) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float xs[kRowsPerCta][kKChunk + 1];
     __shared__ float ws[kBlockV][kKChunk + 1];
     const int vt = blockIdx.x;
@@ -117,6 +119,8 @@ __global__ void __launch_bounds__(256) swiglu_simt_kernel(const float* __restric
                                                           const float* __restrict__ W1, int n_rows, int K, int N,
                                                           float* __restrict__ out, const float* __restrict__ hidden,
                                                           int R, int M, int gamma) {
+    pdl_trigger();
+    pdl_wait();
     constexpr int T = 64, KC = 16;
     __shared__ float xs[KC][T + 4];
     __shared__ float w0s[KC][T + 4];
@@ -185,9 +189,10 @@ cudaError_t launch_lmhead_simt(const Ctx& ctx, int dtype, const void* lm_head, c
     if (n_rows <= 0) return cudaSuccess;
     const int n_tiles = (V + kBlockV - 1) / kBlockV;
     dim3 grid(n_tiles, (n_rows + kRowsPerCta - 1) / kRowsPerCta);
-    lmhead_simt_kernel<<<grid, 256, 0, ctx.stream>>>(static_cast<const float*>(lm_head), static_cast<const float*>(x),
-                                                     n_rows, d, V, inv_temp, partials, n_tiles);
-    return cudaGetLastError();
+    const cudaError_t e = launch_pdl(lmhead_simt_kernel, grid, dim3(256), 0, ctx.stream,
+                                     static_cast<const float*>(lm_head), static_cast<const float*>(x), n_rows, d, V,
+                                     inv_temp, partials, n_tiles);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_swiglu_simt(const Ctx& ctx, const void* X, const void* w_gate, const void* w_up,
@@ -195,16 +200,16 @@ cudaError_t launch_swiglu_simt(const Ctx& ctx, const void* X, const void* w_gate
                                int gamma, void* A, void* h_prime) {
     if (n_rows <= 0) return cudaSuccess;
     dim3 g1((I + 63) / 64, (n_rows + 63) / 64);
-    swiglu_simt_kernel<true><<<g1, 256, 0, ctx.stream>>>(
-        static_cast<const float*>(X), static_cast<const float*>(w_gate), static_cast<const float*>(w_up), n_rows,
-        2 * d, I, static_cast<float*>(A), nullptr, R, M, gamma);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_pdl(swiglu_simt_kernel<true>, g1, dim3(256), 0, ctx.stream, static_cast<const float*>(X),
+                               static_cast<const float*>(w_gate), static_cast<const float*>(w_up), n_rows, 2 * d, I,
+                               static_cast<float*>(A), static_cast<const float*>(nullptr), R, M, gamma);
+    if (e == cudaSuccess) e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     dim3 g2((d + 63) / 64, (n_rows + 63) / 64);
-    swiglu_simt_kernel<false><<<g2, 256, 0, ctx.stream>>>(
-        static_cast<const float*>(A), static_cast<const float*>(w_down), nullptr, n_rows, I, d,
-        static_cast<float*>(h_prime), static_cast<const float*>(hidden), R, M, gamma);
-    return cudaGetLastError();
+    e = launch_pdl(swiglu_simt_kernel<false>, g2, dim3(256), 0, ctx.stream, static_cast<const float*>(A),
+                   static_cast<const float*>(w_down), static_cast<const float*>(nullptr), n_rows, I, d,
+                   static_cast<float*>(h_prime), static_cast<const float*>(hidden), R, M, gamma);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace tf

@@ -143,6 +143,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                const __grid_constant__ CUtensorMap tmap_w1, int n_rows, int K, int n_ntiles,
                int n_mgroups, int k_splits, int w_stream_once, EpiParams ep, int* status) {
     using C = TileCfg<MT, NB, BN, STAGES>;
+    pdl_trigger();
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -180,6 +181,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    if (!(warp == 0 && lane == 0)) pdl_wait();   // the producer waits after its weight prefetch
 
     if (warp == 0) {
         // ------------------------------------------------------------------ TMA producer
@@ -189,29 +191,50 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             if (NB == 2) ptx::prefetch_tmap(&tmap_w1);
             const uint64_t pol_x = ptx::policy_evict_last();
             const uint64_t pol_w = w_stream_once ? ptx::policy_evict_first() : ptx::policy_evict_last();
+            // The weights are no kernel's output: the first unit's first weight tiles are
+            // requested before waiting for the previous kernel (which may be writing X).
+            int pre = 0;
+            if (blockIdx.x < n_units) {
+                const Unit w = decode_unit(blockIdx.x, n_mgroups, k_splits);
+                pre = nk < STAGES ? nk : STAGES;
+                for (int i = 0; i < pre; ++i) {
+                    const int kb = w.kx * nk + i;
+                    uint8_t* sp = smem + i * C::kStageBytes;
+                    ptx::mbar_arrive_expect_tx(&full[i], C::kStageBytes);
+                    ptx::tma_load_2d(sp + MT * C::kABytes, &tmap_w0, &full[i], kb * kBK, w.nt * BN, pol_w);
+                    if (NB == 2)
+                        ptx::tma_load_2d(sp + MT * C::kABytes + C::kBBytes, &tmap_w1, &full[i], kb * kBK,
+                                         w.nt * BN, pol_w);
+                }
+            }
+            pdl_wait();
             int stage = 0;
             uint32_t phase = 0;
             uint32_t issued_mask = 0;                 // stages that ever received a load
             uint32_t last_parity[STAGES > 0 ? STAGES : 1];
             bool ok = true;
+            int it = 0;                               // k-steps issued so far by this CTA
             for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
                 const Unit w = decode_unit(u, n_mgroups, k_splits);
                 const int nt = w.nt, mg = w.mg;
-                for (int kb = w.kx * nk; kb < (w.kx + 1) * nk; ++kb) {
+                for (int kb = w.kx * nk; kb < (w.kx + 1) * nk; ++kb, ++it) {
                     if (!ptx::mbar_wait(&empty[stage], phase ^ 1u, abort_flag, kWaitLimitNs)) {
                         ok = false;
                         break;
                     }
-                    ptx::mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
                     uint8_t* sp = smem + stage * C::kStageBytes;
+                    const bool w_done = it < pre;     // weight tiles already requested above
+                    if (!w_done) ptx::mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
 #pragma unroll
                     for (int j = 0; j < MT; ++j)
                         ptx::tma_load_2d(sp + j * C::kABytes, &tmap_x, &full[stage], kb * kBK,
                                          (mg * MT + j) * kBM, pol_x);
-                    ptx::tma_load_2d(sp + MT * C::kABytes, &tmap_w0, &full[stage], kb * kBK, nt * BN, pol_w);
-                    if (NB == 2)
-                        ptx::tma_load_2d(sp + MT * C::kABytes + C::kBBytes, &tmap_w1, &full[stage],
-                                         kb * kBK, nt * BN, pol_w);
+                    if (!w_done) {
+                        ptx::tma_load_2d(sp + MT * C::kABytes, &tmap_w0, &full[stage], kb * kBK, nt * BN, pol_w);
+                        if (NB == 2)
+                            ptx::tma_load_2d(sp + MT * C::kABytes + C::kBBytes, &tmap_w1, &full[stage],
+                                             kb * kBK, nt * BN, pol_w);
+                    }
                     issued_mask |= 1u << stage;
                     last_parity[stage] = phase;
                     if (++stage == STAGES) {
@@ -473,9 +496,9 @@ cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& t
     const int n_units = n_ntiles * n_mgroups * k_splits;
     const int grid = n_units < ctx.num_sms ? n_units : ctx.num_sms;
     const int stream_once = n_mgroups == 1 ? 1 : 0;
-    kern<<<grid, kThreads, C::kSmemBytes, ctx.stream>>>(tx, tw0, tw1, n_rows, K, n_ntiles, n_mgroups, k_splits,
-                                                       stream_once, ep, ctx.status);
-    return cudaGetLastError();
+    e = launch_pdl(kern, dim3(grid), dim3(kThreads), C::kSmemBytes, ctx.stream, tx, tw0, tw1, n_rows, K, n_ntiles,
+                   n_mgroups, k_splits, stream_once, ep, ctx.status);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace

@@ -19,6 +19,8 @@ __global__ void __launch_bounds__(256) gather_norm_kernel(const T* __restrict__ 
                                                           const int32_t* __restrict__ top_ids, int gamma, int M,
                                                           int K1, int R, int d, int V, float eps, T* __restrict__ X,
                                                           int* status) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float red[2][8];
     const int row = blockIdx.x;
     const int sq = row / R, r = row - sq * R;
@@ -215,6 +217,8 @@ __device__ __forceinline__ void write_nodes(const TreeArgs& a, int s, const Tree
 
 // General builder (any B): the queue in shared memory.
 __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, int stage_lists) {
+    pdl_trigger();
+    pdl_wait();
     extern __shared__ __align__(16) uint8_t smem_raw[];
     const TreeSmem t = tree_smem(smem_raw, a);
     unsigned long long* qkey = t.qkey;
@@ -356,6 +360,8 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
 // of build_tree_kernel.
 template <int S>
 __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a, int stage_lists) {
+    pdl_trigger();
+    pdl_wait();
     extern __shared__ __align__(16) uint8_t smem_raw[];
     const TreeSmem t = tree_smem(smem_raw, a);
     const int n_out = a.B + 1;
@@ -502,6 +508,8 @@ __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __
                                                         const int32_t* __restrict__ node_depth,
                                                         const int32_t* __restrict__ root_pos,
                                                         uint8_t* __restrict__ mask, int32_t* __restrict__ pos_ids) {
+    pdl_trigger();
+    pdl_wait();
     extern __shared__ uint32_t sm[];
     const int W = (n + 31) / 32;
     int* par = reinterpret_cast<int*>(sm);
@@ -589,6 +597,8 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
     const uint4* __restrict__ hidden, const uint4* __restrict__ embed, const uint4* __restrict__ norm_h,
     const uint4* __restrict__ norm_e, const int32_t* __restrict__ root_tok, const int32_t* __restrict__ top_ids,
     int gamma, int M, int K1, int R, int d, int V, float eps, uint4* __restrict__ X, int* status) {
+    pdl_trigger();
+    pdl_wait();
     constexpr int kMaxPerThread = 4;          // d <= 256 * 8 * 4 = 8192
     __shared__ double red[2][8];
     __shared__ float scale[4];                // hi, lo of the hidden half; hi, lo of the embedding half
@@ -682,23 +692,24 @@ cudaError_t launch_gather_norm(const Ctx& ctx, int dtype, const void* hidden, co
                                int M, int K1, int d, int V, float eps, void* X) {
     const int R = 1 + M * (gamma - 1);
     const int rows = b * R;
+    cudaError_t e;
     if (dtype == TF_BF16 && d % 8 == 0 && d <= 8192) {
-        gather_norm_bf16x8_kernel<<<rows, 256, 0, ctx.stream>>>(
-            static_cast<const uint4*>(hidden), static_cast<const uint4*>(embed), static_cast<const uint4*>(norm_h),
-            static_cast<const uint4*>(norm_e), root_tok, top_ids, gamma, M, K1, R, d, V, eps, static_cast<uint4*>(X),
-            ctx.status);
+        e = launch_pdl(gather_norm_bf16x8_kernel, dim3(rows), dim3(256), 0, ctx.stream,
+                       static_cast<const uint4*>(hidden), static_cast<const uint4*>(embed),
+                       static_cast<const uint4*>(norm_h), static_cast<const uint4*>(norm_e), root_tok, top_ids, gamma,
+                       M, K1, R, d, V, eps, static_cast<uint4*>(X), ctx.status);
     } else if (dtype == TF_BF16) {
-        gather_norm_kernel<__nv_bfloat16><<<rows, 256, 0, ctx.stream>>>(
-            static_cast<const __nv_bfloat16*>(hidden), static_cast<const __nv_bfloat16*>(embed),
-            static_cast<const __nv_bfloat16*>(norm_h), static_cast<const __nv_bfloat16*>(norm_e), root_tok, top_ids,
-            gamma, M, K1, R, d, V, eps, static_cast<__nv_bfloat16*>(X), ctx.status);
+        e = launch_pdl(gather_norm_kernel<__nv_bfloat16>, dim3(rows), dim3(256), 0, ctx.stream,
+                       static_cast<const __nv_bfloat16*>(hidden), static_cast<const __nv_bfloat16*>(embed),
+                       static_cast<const __nv_bfloat16*>(norm_h), static_cast<const __nv_bfloat16*>(norm_e), root_tok,
+                       top_ids, gamma, M, K1, R, d, V, eps, static_cast<__nv_bfloat16*>(X), ctx.status);
     } else {
-        gather_norm_kernel<float><<<rows, 256, 0, ctx.stream>>>(
-            static_cast<const float*>(hidden), static_cast<const float*>(embed), static_cast<const float*>(norm_h),
-            static_cast<const float*>(norm_e), root_tok, top_ids, gamma, M, K1, R, d, V, eps,
-            static_cast<float*>(X), ctx.status);
+        e = launch_pdl(gather_norm_kernel<float>, dim3(rows), dim3(256), 0, ctx.stream,
+                       static_cast<const float*>(hidden), static_cast<const float*>(embed),
+                       static_cast<const float*>(norm_h), static_cast<const float*>(norm_e), root_tok, top_ids, gamma, M,
+                       K1, R, d, V, eps, static_cast<float*>(X), ctx.status);
     }
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_build_tree(const Ctx& ctx, int b, int gamma, int M, int K1, int K2, int B, int V, int mode, int R,
@@ -719,8 +730,8 @@ cudaError_t launch_build_tree(const Ctx& ctx, int b, int gamma, int M, int K1, i
                                                  : build_tree_kernel;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    kern<<<b, kTreeThreads, smem, ctx.stream>>>(a, stage);
-    return cudaGetLastError();
+    e = launch_pdl(kern, dim3(b), dim3(kTreeThreads), smem, ctx.stream, a, stage);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_tree_mask(const Ctx& ctx, int b, int B, const int32_t* node_parent, const int32_t* node_depth,
@@ -731,8 +742,9 @@ cudaError_t launch_tree_mask(const Ctx& ctx, int b, int B, const int32_t* node_p
     cudaError_t e = cudaFuncSetAttribute(tree_mask_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    tree_mask_kernel<<<b, 256, smem, ctx.stream>>>(n, node_parent, node_depth, root_pos, mask, pos_ids);
-    return cudaGetLastError();
+    e = launch_pdl(tree_mask_kernel, dim3(b), dim3(256), smem, ctx.stream, n, node_parent, node_depth, root_pos, mask,
+                   pos_ids);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace tf

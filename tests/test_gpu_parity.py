@@ -144,7 +144,8 @@ def test_bf16_batch_equals_single_sequences():
 
 def test_bf16_recompute_path_is_exact():
     # 80 vocabulary rows of one 256-block aligned with every hidden state: the top-64 of each row
-    # all sit in that block, so its 8-entry list is certified incomplete and recomputed
+    # all sit in that block, so its 32-column chunks each hold more members of the top 64 than
+    # their two kept candidates; certification must flag and recompute them
     cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=1, V=4096, K2=64, B=64, M=4)
     inp = synth.make_inputs(cfg)
     g = torch.Generator().manual_seed(5)
@@ -231,3 +232,19 @@ def test_full_size_batch32_sampled_sequences():
 def test_full_size_wide_sampled_sequence(name):
     cfg = synth.get_config(name)
     check(cfg, orc_seqs=[3], emulate_also=False)
+
+
+def test_kernel_launch_counter_counts_each_kernel():
+    # tf_stage1_marginals is one LM-head pass and one merge: two kernels per call
+    from paper_2606_03819_gb300 import binding as Bn
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=2, V=2000)
+    d = parity.device_inputs(synth.make_inputs(cfg))
+    dims = Bn.Dims.from_config(cfg)
+    ws = Bn.alloc_workspace(dims)
+    ids = torch.empty(cfg.batch, cfg.gamma, dims.K1, dtype=torch.int32, device="cuda")
+    lp = torch.empty(cfg.batch, cfg.gamma, dims.K1, dtype=torch.float32, device="cuda")
+    n0 = Bn.tf_kernel_launches()
+    for _ in range(3):
+        Bn.tf_stage1_marginals(dims, d, d["hidden"], ids, lp, ws)
+    torch.cuda.synchronize()
+    assert Bn.tf_kernel_launches() - n0 == 6
