@@ -20,7 +20,10 @@
 //               the two warps of a group on the same lanes split the columns in halves.
 // A work unit is (N tile, group of MT M-tiles). With MT = 2 both slots hold one unit (M-tile j
 // in slot j); with MT = 1 consecutive units alternate slots so the epilogue of one overlaps the
-// MMAs of the next. Every wait is bounded: after a time limit the kernel raises TF_DEV_TIMEOUT,
+// MMAs of the next. With clusters of CL = 2 CTAs (the LM head over more than 128 rows), units
+// are dealt to clusters, CTA r of a cluster takes M-tile r of the unit's pair, and each CTA
+// loads half of the unit's weight tile and multicasts it to both; a stage is free again once
+// both CTAs' MMAs have consumed it. Every wait is bounded: after a time limit the kernel raises TF_DEV_TIMEOUT,
 // drains its in-flight copies and MMAs, frees TMEM and returns.
 #include <cuda.h>
 #include <math.h>
@@ -137,12 +140,14 @@ __device__ __forceinline__ ChunkNode chunk_tree(const uint32_t (&r)[32], int v0,
     }
 }
 
-template <int EPI, int MT, int NB, int BN, int STAGES>
+template <int EPI, int MT, int NB, int BN, int STAGES, int CL>
 __global__ void __launch_bounds__(kThreads, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_w0,
                const __grid_constant__ CUtensorMap tmap_w1, int n_rows, int K, int n_ntiles,
                int n_mgroups, int k_splits, int w_stream_once, EpiParams ep, int* status) {
     using C = TileCfg<MT, NB, BN, STAGES>;
+    static_assert(CL == 1 || (CL == 2 && NB == 1), "clusters of two share one weight operand");
+    constexpr uint16_t kClusterMask = static_cast<uint16_t>((1u << CL) - 1u);
     pdl_trigger();
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -158,12 +163,17 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int n_units = n_ntiles * n_mgroups * k_splits;
+    // Units are dealt to clusters; CTA `crank` of a cluster takes M-tile group member crank of
+    // every unit (with CL = 1 a cluster is one CTA).
+    const int crank = CL > 1 ? static_cast<int>(ptx::cluster_ctarank()) : 0;
+    const int cid = CL > 1 ? static_cast<int>(ptx::cluster_id_x()) : static_cast<int>(blockIdx.x);
+    const int ncl = CL > 1 ? static_cast<int>(ptx::cluster_count_x()) : static_cast<int>(gridDim.x);
     const int nk = K / kBK / k_splits;      // K-steps per unit (K % (64 * k_splits) == 0)
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             ptx::mbar_init(&full[s], 1);
-            ptx::mbar_init(&empty[s], 1);
+            ptx::mbar_init(&empty[s], CL);   // freed once every CTA of the cluster has consumed it
         }
         for (int g = 0; g < 2; ++g) {
             ptx::mbar_init(&tfull[g], 1);
@@ -179,6 +189,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     }
     ptx::tc_fence_before();
     __syncthreads();
+    if constexpr (CL > 1) ptx::cluster_sync();   // the peers' barriers exist before any multicast
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
     if (!(warp == 0 && lane == 0)) pdl_wait();   // the producer waits after its weight prefetch
@@ -191,20 +202,27 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             if (NB == 2) ptx::prefetch_tmap(&tmap_w1);
             const uint64_t pol_x = ptx::policy_evict_last();
             const uint64_t pol_w = w_stream_once ? ptx::policy_evict_first() : ptx::policy_evict_last();
+            // Weight tiles of one stage. In a cluster each CTA fetches its share of the rows and
+            // multicasts it to every CTA of the cluster (tmap_w0's box is BN / CL rows high).
+            auto load_w = [&](uint8_t* sp, uint64_t* bar, int kb, int nt) {
+                if constexpr (CL > 1) {
+                    ptx::tma_load_2d_multicast(sp + MT * C::kABytes + crank * (C::kBBytes / CL), &tmap_w0, bar,
+                                               kb * kBK, nt * BN + crank * (BN / CL), kClusterMask, pol_w);
+                } else {
+                    ptx::tma_load_2d(sp + MT * C::kABytes, &tmap_w0, bar, kb * kBK, nt * BN, pol_w);
+                    if (NB == 2)
+                        ptx::tma_load_2d(sp + MT * C::kABytes + C::kBBytes, &tmap_w1, bar, kb * kBK, nt * BN, pol_w);
+                }
+            };
             // The weights are no kernel's output: the first unit's first weight tiles are
             // requested before waiting for the previous kernel (which may be writing X).
             int pre = 0;
-            if (blockIdx.x < n_units) {
-                const Unit w = decode_unit(blockIdx.x, n_mgroups, k_splits);
+            if (cid < n_units) {
+                const Unit w = decode_unit(cid, n_mgroups, k_splits);
                 pre = nk < STAGES ? nk : STAGES;
                 for (int i = 0; i < pre; ++i) {
-                    const int kb = w.kx * nk + i;
-                    uint8_t* sp = smem + i * C::kStageBytes;
                     ptx::mbar_arrive_expect_tx(&full[i], C::kStageBytes);
-                    ptx::tma_load_2d(sp + MT * C::kABytes, &tmap_w0, &full[i], kb * kBK, w.nt * BN, pol_w);
-                    if (NB == 2)
-                        ptx::tma_load_2d(sp + MT * C::kABytes + C::kBBytes, &tmap_w1, &full[i], kb * kBK,
-                                         w.nt * BN, pol_w);
+                    load_w(smem + i * C::kStageBytes, &full[i], w.kx * nk + i, w.nt);
                 }
             }
             pdl_wait();
@@ -214,9 +232,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             uint32_t last_parity[STAGES > 0 ? STAGES : 1];
             bool ok = true;
             int it = 0;                               // k-steps issued so far by this CTA
-            for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+            for (int u = cid; u < n_units && ok; u += ncl) {
                 const Unit w = decode_unit(u, n_mgroups, k_splits);
-                const int nt = w.nt, mg = w.mg;
+                const int nt = w.nt, mt0 = (w.mg * CL + crank) * MT;
                 for (int kb = w.kx * nk; kb < (w.kx + 1) * nk; ++kb, ++it) {
                     if (!ptx::mbar_wait(&empty[stage], phase ^ 1u, abort_flag, kWaitLimitNs)) {
                         ok = false;
@@ -227,14 +245,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                     if (!w_done) ptx::mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
 #pragma unroll
                     for (int j = 0; j < MT; ++j)
-                        ptx::tma_load_2d(sp + j * C::kABytes, &tmap_x, &full[stage], kb * kBK,
-                                         (mg * MT + j) * kBM, pol_x);
-                    if (!w_done) {
-                        ptx::tma_load_2d(sp + MT * C::kABytes, &tmap_w0, &full[stage], kb * kBK, nt * BN, pol_w);
-                        if (NB == 2)
-                            ptx::tma_load_2d(sp + MT * C::kABytes + C::kBBytes, &tmap_w1, &full[stage],
-                                             kb * kBK, nt * BN, pol_w);
-                    }
+                        ptx::tma_load_2d(sp + j * C::kABytes, &tmap_x, &full[stage], kb * kBK, (mt0 + j) * kBM,
+                                         pol_x);
+                    if (!w_done) load_w(sp, &full[stage], kb, nt);
                     issued_mask |= 1u << stage;
                     last_parity[stage] = phase;
                     if (++stage == STAGES) {
@@ -261,7 +274,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             uint32_t use[2] = {0u, 0u};
             bool ok = true;
             int kl = 0;
-            for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++kl) {
+            for (int u = cid; u < n_units && ok; u += ncl, ++kl) {
                 const int g0 = (MT == 2) ? 0 : (kl & 1);
                 for (int j = 0; j < MT && ok; ++j)
                     ok = ptx::mbar_wait(&tempty[g0 + j], (use[g0 + j] & 1u) ^ 1u, abort_flag, kWaitLimitNs);
@@ -288,7 +301,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                             }
                         }
                     }
-                    ptx::mma_commit(&empty[stage]);   // frees the stage once these MMAs finish
+                    // frees the stage (in every CTA of the cluster) once these MMAs finish
+                    if constexpr (CL > 1)
+                        ptx::mma_commit_multicast(&empty[stage], kClusterMask);
+                    else
+                        ptx::mma_commit(&empty[stage]);
                     if (++stage == STAGES) {
                         stage = 0;
                         phase ^= 1u;
@@ -316,7 +333,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         const int half = (e % (kEpiWarps / 2)) / 4; // which half of the columns this warp takes
         uint32_t use = 0;
         int kl = 0;
-        for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++kl) {
+        for (int u = cid; u < n_units; u += ncl, ++kl) {
             if (MT == 1 && (kl & 1) != g) continue;
             if (!ptx::mbar_wait(&tfull[g], use & 1u, abort_flag, kWaitLimitNs)) {
                 *abort_flag = 1;
@@ -326,8 +343,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             ++use;
             ptx::tc_fence_after();
             const Unit w = decode_unit(u, n_mgroups, k_splits);
-            const int nt = w.nt, mg = w.mg;
-            const int row = (mg * MT + (MT == 2 ? g : 0)) * kBM + q * 32 + lane;
+            const int nt = w.nt;
+            const int row = ((w.mg * CL + crank) * MT + (MT == 2 ? g : 0)) * kBM + q * 32 + lane;
             const uint32_t tb = tmem_base + 256u * g + (static_cast<uint32_t>(q * 32) << 16);
 
             if constexpr (EPI == EPI_LMHEAD) {
@@ -445,6 +462,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
 
     ptx::tc_fence_before();
     __syncthreads();
+    // no CTA of the cluster may still write into this CTA's shared memory or barriers
+    if constexpr (CL > 1) ptx::cluster_sync();
     if (warp == 1) {
         __syncwarp();
         ptx::tc_fence_after();
@@ -486,18 +505,49 @@ cudaError_t make_tmap(CUtensorMap* map, const void* base, uint64_t inner, uint64
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-template <int EPI, int MT, int NB, int BN, int STAGES>
+// Clusters of CL CTAs that can be resident at once for this kernel (at most num_sms / CL).
+template <typename K>
+int resident_clusters(K kern, int smem, int cl, int num_sms) {
+    int cap = num_sms / cl;
+    if (cl == 1) return cap;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cl * cap);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cl;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n < 1) {
+        (void)cudaGetLastError();
+        return cap;
+    }
+    return n < cap ? n : cap;
+}
+
+template <int EPI, int MT, int NB, int BN, int STAGES, int CL = 1>
 cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& tw0, const CUtensorMap& tw1,
                      int n_rows, int K, int n_ntiles, int n_mgroups, const EpiParams& ep, int k_splits = 1) {
     using C = TileCfg<MT, NB, BN, STAGES>;
-    auto kern = tc_gemm_kernel<EPI, MT, NB, BN, STAGES>;
+    auto kern = tc_gemm_kernel<EPI, MT, NB, BN, STAGES, CL>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (e != cudaSuccess) return e;
     const int n_units = n_ntiles * n_mgroups * k_splits;
-    const int grid = n_units < ctx.num_sms ? n_units : ctx.num_sms;
     const int stream_once = n_mgroups == 1 ? 1 : 0;
-    e = launch_pdl(kern, dim3(grid), dim3(kThreads), C::kSmemBytes, ctx.stream, tx, tw0, tw1, n_rows, K, n_ntiles,
-                   n_mgroups, k_splits, stream_once, ep, ctx.status);
+    if constexpr (CL == 1) {
+        const int grid = n_units < ctx.num_sms ? n_units : ctx.num_sms;
+        e = launch_pdl(kern, dim3(grid), dim3(kThreads), C::kSmemBytes, ctx.stream, tx, tw0, tw1, n_rows, K,
+                       n_ntiles, n_mgroups, k_splits, stream_once, ep, ctx.status);
+    } else {
+        static const int max_cl = resident_clusters(kern, C::kSmemBytes, CL, ctx.num_sms);
+        const int n_cl = n_units < max_cl ? n_units : max_cl;
+        e = launch_pdl_cluster(kern, dim3(CL * n_cl), dim3(kThreads), C::kSmemBytes, ctx.stream, CL, tx, tw0, tw1,
+                               n_rows, K, n_ntiles, n_mgroups, k_splits, stream_once, ep, ctx.status);
+    }
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -506,19 +556,22 @@ cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& t
 cudaError_t launch_lmhead_tc(const Ctx& ctx, const void* lm_head, const void* x, int n_rows, int d, int V,
                              float inv_temp, Partials partials) {
     if (n_rows <= 0) return cudaSuccess;
+    const int n_tiles = (V + kBlockV - 1) / kBlockV;
+    const int m_tiles = (n_rows + kBM - 1) / kBM;
+    // More than one M-tile: clusters of two CTAs, one M-tile each, share every weight tile (each
+    // fetches half of its rows and multicasts them), so W_lm is read once while each CTA keeps
+    // one TMEM slot per unit and overlaps its epilogue with the next unit's MMAs.
+    const int cl = m_tiles == 1 ? 1 : 2;
     CUtensorMap tx, tw;
     cudaError_t e = make_tmap(&tx, x, d, n_rows, kBK, kBM);
-    if (e == cudaSuccess) e = make_tmap(&tw, lm_head, d, V, kBK, kBlockV);
+    if (e == cudaSuccess) e = make_tmap(&tw, lm_head, d, V, kBK, kBlockV / cl);
     if (e != cudaSuccess) return e;
     EpiParams ep{};
     ep.partials = partials;
     ep.V = V;
     ep.inv_temp = inv_temp;
-    const int n_tiles = (V + kBlockV - 1) / kBlockV;
-    const int m_tiles = (n_rows + kBM - 1) / kBM;
-    if (m_tiles == 1)
-        return run_gemm<EPI_LMHEAD, 1, 1, kBlockV, 4>(ctx, tx, tw, tw, n_rows, d, n_tiles, 1, ep);
-    return run_gemm<EPI_LMHEAD, 2, 1, kBlockV, 3>(ctx, tx, tw, tw, n_rows, d, n_tiles, (m_tiles + 1) / 2, ep);
+    if (m_tiles == 1) return run_gemm<EPI_LMHEAD, 1, 1, kBlockV, 4>(ctx, tx, tw, tw, n_rows, d, n_tiles, 1, ep);
+    return run_gemm<EPI_LMHEAD, 1, 1, kBlockV, 4, 2>(ctx, tx, tw, tw, n_rows, d, n_tiles, (m_tiles + 1) / 2, ep);
 }
 
 // Split-K factor for a GEMM with `base_units` (N tiles x M-tile groups) and nk K-steps: enough
