@@ -500,9 +500,12 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
 }
 
 // ------------------------------------------------------------------------------------------
-// mask[i][j] = 1 iff node j is node i or one of its ancestors. Ancestor sets are bitsets built
-// level by level (a node's set is its parent's set plus itself); pos = root_pos + depth.
-// Nodes with an invalid parent link (missing nodes) get empty rows and columns and pos -1.
+// mask[i][j] = 1 iff node j is node i or one of its ancestors; pos = root_pos + depth. Each
+// node walks its own parent chain (at most kMaxGamma links) and sets the bits of its row, so no
+// thread waits for another level. A node is present iff every link of its chain goes to a
+// smaller index exactly one level up and the chain ends at the root (node 0, depth 0); absent
+// nodes (missing from an underfull tree, or behind a broken link) get an empty row and
+// column and pos -1.
 // ------------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __restrict__ node_parent,
                                                         const int32_t* __restrict__ node_depth,
@@ -514,46 +517,39 @@ __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __
     const int W = (n + 31) / 32;
     int* par = reinterpret_cast<int*>(sm);
     int* dep = par + n;
-    uint32_t* anc = reinterpret_cast<uint32_t*>(dep + n);
-    __shared__ int max_dep;
+    uint32_t* anc = reinterpret_cast<uint32_t*>(dep + n);   // [n][W] ancestor-or-self bits
     const int s = blockIdx.x;
     const int32_t* P = node_parent + static_cast<size_t>(s) * n;
     const int32_t* D = node_depth + static_cast<size_t>(s) * n;
-    if (threadIdx.x == 0) max_dep = 0;
-    for (int i = threadIdx.x; i < n * W; i += blockDim.x) anc[i] = 0u;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        par[i] = P[i];
+        dep[i] = D[i];
+    }
     __syncthreads();
     for (int i = threadIdx.x; i < n; i += blockDim.x) {
-        int p = P[i], d = D[i];
-        const bool ok = (i == 0) ? (d == 0) : (p >= 0 && p < i && d >= 1 && d <= kMaxGamma);
-        par[i] = ok ? p : -1;
-        dep[i] = ok ? d : -1;
-        if (ok) atomicMax(&max_dep, d);
+        uint32_t* row = anc + static_cast<size_t>(i) * W;
+        for (int w = 0; w < W; ++w) row[w] = 0u;
+        bool ok = true;
+        int j = i;
+        for (int steps = 0; ok && j != 0; ++steps) {
+            const int p = par[j];
+            ok = steps < kMaxGamma && dep[j] >= 1 && dep[j] <= kMaxGamma && p >= 0 && p < j && dep[p] == dep[j] - 1;
+            row[j >> 5] |= 1u << (j & 31);
+            j = p;
+        }
+        ok = ok && dep[0] == 0;
+        if (ok) {
+            row[0] |= 1u;                                  // the root
+        } else {
+            for (int w = 0; w < W; ++w) row[w] = 0u;       // absent: empty row
+        }
+        pos_ids[static_cast<size_t>(s) * n + i] = ok ? root_pos[s] + dep[i] : -1;
     }
     __syncthreads();
-    for (int L = 0; L <= max_dep; ++L) {
-        for (int idx = threadIdx.x; idx < n * W; idx += blockDim.x) {
-            const int i = idx / W, w = idx - (idx / W) * W;
-            if (dep[i] != L) continue;
-            uint32_t v = 0u;
-            if (L > 0) {
-                const int p = par[i];
-                // the parent must sit one level up and be present (its own bit set)
-                if (dep[p] != L - 1 || !((anc[p * W + p / 32] >> (p & 31)) & 1u)) continue;
-                v = anc[p * W + w];
-            }
-            if (w == i / 32) v |= 1u << (i & 31);
-            anc[i * W + w] = v;
-        }
-        __syncthreads();
-    }
     uint8_t* out = mask + static_cast<size_t>(s) * n * n;
     for (int idx = threadIdx.x; idx < n * n; idx += blockDim.x) {
         const int i = idx / n, j = idx - (idx / n) * n;
-        out[idx] = static_cast<uint8_t>((anc[i * W + j / 32] >> (j & 31)) & 1u);
-    }
-    for (int i = threadIdx.x; i < n; i += blockDim.x) {
-        const bool present = (anc[i * W + i / 32] >> (i & 31)) & 1u;
-        pos_ids[static_cast<size_t>(s) * n + i] = present ? root_pos[s] + dep[i] : -1;
+        out[idx] = static_cast<uint8_t>((anc[i * W + (j >> 5)] >> (j & 31)) & 1u);
     }
 }
 
