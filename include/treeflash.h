@@ -202,17 +202,18 @@ tf_status tf_draft_tree_host(const tf_dims* dims, const tf_weights* w, const voi
 
 /* The LM-head pass fused with log-softmax bookkeeping (Alg. 1 "LMHead" and "TopM"):
  * streams W_lm once and, for every row r of x [n_rows, d] (dtype) and every block of 256
- * vocabulary entries, leaves in the workspace the block's max logit, its sum of
- * exp(logit - max) and its 8 largest (logit, id). Logits never reach memory.
+ * vocabulary entries, leaves in the workspace per half block its max logit, sum of
+ * exp(logit - max) and best (logit, id), and per 32-entry chunk its three largest logits with
+ * the ids of the first two (TF_VIEW_HALVES, TF_VIEW_CHUNKS). Logits never reach memory.
  * n_rows <= the larger of b*gamma and b*R. */
 tf_status tf_lmhead_partials(const tf_dims* dims, const void* lm_head, const void* x,
                              int32_t n_rows, void* ws, size_t ws_bytes, tf_stream_t stream);
 
-/* Merge the per-block partials of tf_lmhead_partials into each row's log-sum-exp and exact
- * top-k (k <= 64): out_ids [n_rows, k] int32, out_logp [n_rows, k] float = logit - LSE. A
- * block whose 8 kept entries could hide a member of the top-k has its logits recomputed
- * exactly from lm_head and x (sets TF_DEV_RECOMPUTED), so the result never depends on the
- * 8-entry truncation. */
+/* Merge the partials of tf_lmhead_partials (same n_rows) into each row's log-sum-exp and exact
+ * top-k (k <= 64): out_ids [n_rows, k] int32, out_logp [n_rows, k] float = logit - LSE. A chunk
+ * whose third-largest logit could still be a member of the top-k has its 32 logits recomputed
+ * exactly from lm_head and x (sets TF_DEV_RECOMPUTED), so the result never depends on keeping
+ * only two entries per chunk. */
 tf_status tf_lmhead_merge(const tf_dims* dims, const void* lm_head, const void* x,
                           int32_t n_rows, int32_t k, int32_t* out_ids, float* out_logp,
                           void* ws, size_t ws_bytes, tf_stream_t stream);
@@ -230,13 +231,30 @@ tf_status tf_ar_approx(const tf_dims* dims, const tf_weights* w, const void* hid
  * as separate calls without a copy. */
 tf_status tf_workspace_h_prime(const tf_dims* dims, void* ws, size_t ws_bytes, void** h_prime);
 
-/* Intermediates of Eq. 1 left in the workspace by the last tf_ar_approx / tf_stage2_ar_approx
- * (for inspection and testing; host only, no GPU work):
+/* Regions of a workspace laid out for `dims` (for inspection, testing and for exchanging
+ * LM-head partials between vocabulary shards; host only, no GPU work). *ptr receives the device
+ * address and *bytes the region's size.
+ * Intermediates of Eq. 1 left by the last tf_ar_approx / tf_stage2_ar_approx (TF_MODE_AR only):
  *   TF_VIEW_X        x = [RMSNorm(h)*w_h ; RMSNorm(Embd(prev))*w_e]   [b*R, 2d] dtype
  *   TF_VIEW_A        SiLU(W_gate x) * (W_up x)                         [b*R, I]  dtype
  *   TF_VIEW_H_PRIME  h' = h + W_down A                                 [b*R, d]  dtype
- * *ptr receives the device address and *bytes the view's size. */
-typedef enum { TF_VIEW_X = 0, TF_VIEW_A = 1, TF_VIEW_H_PRIME = 2 } tf_view;
+ * The partials of the last tf_lmhead_partials over n_rows rows, n_tiles = ceil(V / 256), both
+ * float4 tables indexed [block][part][row] with the call's n_rows as the row count:
+ *   TF_VIEW_HALVES   [n_tiles][2][n_rows] per half block (128 entries): (max logit m,
+ *                    sum of exp(z - m), best logit, best token id as int32 bits)
+ *   TF_VIEW_CHUNKS   [n_tiles][8][n_rows] per 32-entry chunk: (largest, second, third largest
+ *                    logit, offsets in the chunk of the first two in bits 0-7 and 8-15)
+ * Logits are W_lm x / T; empty entries hold -inf, sum 0 and id -1. The merge reads token ids
+ * of chunk entries from the block index, so partials of a vocabulary shard starting at token
+ * v0 (a multiple of 256) join an unsharded table at block v0 / 256 once v0 is added to their
+ * half-block ids. */
+typedef enum {
+    TF_VIEW_X = 0,
+    TF_VIEW_A = 1,
+    TF_VIEW_H_PRIME = 2,
+    TF_VIEW_HALVES = 3,
+    TF_VIEW_CHUNKS = 4
+} tf_view;
 tf_status tf_workspace_view(const tf_dims* dims, void* ws, size_t ws_bytes, int32_t view, void** ptr,
                             size_t* bytes);
 

@@ -256,15 +256,22 @@ def tf_workspace_h_prime(dims: Dims, ws) -> torch.Tensor:
     return ws[off:off + n].view(dims.torch_dtype).view(dims.batch, dims.R, dims.d)
 
 
-TF_VIEW_X, TF_VIEW_A, TF_VIEW_H_PRIME = 0, 1, 2
+TF_VIEW_X, TF_VIEW_A, TF_VIEW_H_PRIME, TF_VIEW_HALVES, TF_VIEW_CHUNKS = 0, 1, 2, 3, 4
 
 
-def tf_workspace_view(dims: Dims, ws, view: int) -> torch.Tensor:
-    """x [b*R, 2d], A [b*R, I] or h' [b*R, d] as a tensor view of the workspace (no copy)."""
+def tf_workspace_view(dims: Dims, ws, view: int, n_rows: Optional[int] = None) -> torch.Tensor:
+    """x [b*R, 2d], A [b*R, I] or h' [b*R, d] as a tensor view of the workspace (no copy); for
+    TF_VIEW_HALVES / TF_VIEW_CHUNKS the partials of the last LM-head pass over n_rows rows as
+    float32 [n_tiles, 2 or 8, n_rows, 4]."""
     p, n = ctypes.c_void_p(), ctypes.c_size_t()
     _check("tf_workspace_view", load_library().tf_workspace_view(
         ctypes.byref(dims.c()), _ptr(ws), ws.numel(), view, ctypes.byref(p), ctypes.byref(n)))
     off = p.value - ws.data_ptr()
+    if view in (TF_VIEW_HALVES, TF_VIEW_CHUNKS):
+        n_tiles = (dims.V + 255) // 256
+        parts = 2 if view == TF_VIEW_HALVES else 8
+        nb = n_tiles * parts * n_rows * 16
+        return ws[off:off + nb].view(torch.float32).view(n_tiles, parts, n_rows, 4)
     cols = {TF_VIEW_X: 2 * dims.d, TF_VIEW_A: dims.I, TF_VIEW_H_PRIME: dims.d}[view]
     return ws[off:off + n.value].view(dims.torch_dtype).view(dims.batch * dims.R, cols)
 

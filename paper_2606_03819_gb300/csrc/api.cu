@@ -362,14 +362,26 @@ tf_status tf_workspace_view(const tf_dims* dims, void* ws, size_t ws_bytes, int3
     if (!ptr || !bytes) return TF_ERR_INVALID_ARG;
     Dims D;
     TF_TRY(check_dims(dims, &D));
-    if (D.mode != TF_MODE_AR) return TF_ERR_INVALID_ARG;
     const Layout L = layout(D);
     TF_TRY(check_ws(L, ws, ws_bytes));
-    const size_t rows = static_cast<size_t>(D.b) * D.R;
+    const size_t rows2 = static_cast<size_t>(D.b) * D.R;
+    const size_t rows1 = static_cast<size_t>(D.b) * D.gamma;
+    const size_t rows_lm = D.mode == TF_MODE_AR && rows2 > rows1 ? rows2 : rows1;
     switch (view) {
-        case TF_VIEW_X: *ptr = at<void>(ws, L.X); *bytes = rows * 2 * D.d * D.esize; return TF_OK;
-        case TF_VIEW_A: *ptr = at<void>(ws, L.A); *bytes = rows * D.I * D.esize; return TF_OK;
-        case TF_VIEW_H_PRIME: *ptr = at<void>(ws, L.hp); *bytes = rows * D.d * D.esize; return TF_OK;
+        case TF_VIEW_HALVES:
+            *ptr = at<void>(ws, L.halves);
+            *bytes = rows_lm * D.n_tiles * kHalfBytesPerRowBlock;
+            return TF_OK;
+        case TF_VIEW_CHUNKS:
+            *ptr = at<void>(ws, L.chunks);
+            *bytes = rows_lm * D.n_tiles * kChunkBytesPerRowBlock;
+            return TF_OK;
+    }
+    if (D.mode != TF_MODE_AR) return TF_ERR_INVALID_ARG;
+    switch (view) {
+        case TF_VIEW_X: *ptr = at<void>(ws, L.X); *bytes = rows2 * 2 * D.d * D.esize; return TF_OK;
+        case TF_VIEW_A: *ptr = at<void>(ws, L.A); *bytes = rows2 * D.I * D.esize; return TF_OK;
+        case TF_VIEW_H_PRIME: *ptr = at<void>(ws, L.hp); *bytes = rows2 * D.d * D.esize; return TF_OK;
     }
     return TF_ERR_INVALID_ARG;
 }

@@ -430,29 +430,22 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
             const int dep = 127 - static_cast<int>(wlo >> 24);
             const int par = 0xFFFFFF - static_cast<int>(wlo & 0xFFFFFFu);
             const int node = count++;
+            // next sibling of the popped entry (the same shared-memory words for every lane),
+            // read before the expandability test so that both latencies overlap
+            const bool sibling = rank + 1 < list_len;
+            const size_t sat = static_cast<size_t>(row) * stride + rank + 1;
+            const int sib_tok = sibling ? ids_base[sat] : 0;
+            const float sib_lp = sibling ? lp_base[sat] : 0.0f;
+            // expandable? (depth cap; M-ary rule via one compare per lane)
+            const bool deep_ok = dep < a.gamma;
+            const bool hit = deep_ok && lane < a.M && t.topm[(dep - 1) * a.M + lane] == tok;
+            const unsigned bal = __ballot_sync(kFull, hit);
+            const int crow = !deep_ok ? -1
+                             : a.mode == TF_MODE_MARGINAL ? dep
+                             : bal ? (ar ? 1 + (dep - 1) * a.M + (__ffs(bal) - 1) : dep) : -1;
             if (tok < 0 || tok >= a.V) flags |= TF_DEV_BAD_TOKEN;
             if (!isfinite(sc)) flags |= TF_DEV_NONFINITE;
-            // expandable? (depth cap; M-ary rule via one compare per lane)
-            int crow = -1;
-            if (dep < a.gamma) {
-                if (a.mode == TF_MODE_MARGINAL) {
-                    crow = dep;
-                } else {
-                    const bool hit = lane < a.M && t.topm[(dep - 1) * a.M + lane] == tok;
-                    const unsigned bal = __ballot_sync(kFull, hit);
-                    if (bal) crow = ar ? 1 + (dep - 1) * a.M + (__ffs(bal) - 1) : dep;
-                }
-            }
-            // next sibling of the popped entry, and the first child of the new node (the same
-            // shared-memory words for every lane)
-            const bool sibling = rank + 1 < list_len;
-            unsigned long long sib_key = 0ull;
-            int sib_tok = 0;
-            if (sibling) {
-                const size_t at = static_cast<size_t>(row) * stride + rank + 1;
-                sib_tok = ids_base[at];
-                sib_key = queue_key(psc + lp_base[at], dep, par);
-            }
+            const unsigned long long sib_key = sibling ? queue_key(psc + sib_lp, dep, par) : 0ull;
             if (lane == wl) {
                 // the winner's best slot is the one holding its best key (keys are unique)
 #pragma unroll
