@@ -162,11 +162,12 @@ Partials partials_of(const Layout& L, void* ws, int n_rows) {
 }
 
 tf_status do_partials(const Ctx& ctx, const Dims& D, const Layout& L, void* ws, const void* lm_head, const void* x,
-                      int n_rows) {
+                      int n_rows, bool reset_status = false) {
     const Partials partials = partials_of(L, ws, n_rows);
     if (D.dtype == TF_BF16)
-        return cuda_status(launch_lmhead_tc(ctx, lm_head, x, n_rows, D.d, D.V, D.inv_temp, partials));
-    return cuda_status(launch_lmhead_simt(ctx, D.dtype, lm_head, x, n_rows, D.d, D.V, D.inv_temp, partials));
+        return cuda_status(launch_lmhead_tc(ctx, lm_head, x, n_rows, D.d, D.V, D.inv_temp, partials, reset_status));
+    return cuda_status(
+        launch_lmhead_simt(ctx, D.dtype, lm_head, x, n_rows, D.d, D.V, D.inv_temp, partials, reset_status));
 }
 
 tf_status do_merge(const Ctx& ctx, const Dims& D, const Layout& L, void* ws, const void* lm_head, const void* x,
@@ -286,9 +287,8 @@ tf_status tf_stage1_marginals(const tf_dims* dims, const tf_weights* w, const vo
     TF_TRY(prepare(dims, ws, ws_bytes, stream, &p));
     TF_TRY(check_weights(p.D, w, false));
     if (!aligned16(hidden) || !top_ids || !top_logp) return TF_ERR_INVALID_ARG;
-    TF_TRY(cuda_status(cudaMemsetAsync(p.ctx.status, 0, sizeof(int32_t), p.ctx.stream)));
     const int rows = p.D.b * p.D.gamma;
-    TF_TRY(do_partials(p.ctx, p.D, p.L, ws, w->lm_head, hidden, rows));
+    TF_TRY(do_partials(p.ctx, p.D, p.L, ws, w->lm_head, hidden, rows, /*reset_status=*/true));
     return do_merge(p.ctx, p.D, p.L, ws, w->lm_head, hidden, rows, p.D.K1, top_ids, top_logp);
 }
 

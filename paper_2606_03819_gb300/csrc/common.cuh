@@ -150,11 +150,13 @@ struct Ctx {
     int* status;  // device status word in the workspace
 };
 
-// LM-head pass (tensor-core path for bf16, CUDA-core path for f32)
+// LM-head pass (tensor-core path for bf16, CUDA-core path for f32); reset_status: the kernel
+// zeroes ctx.status once every earlier kernel on the stream has finished
 cudaError_t launch_lmhead_tc(const Ctx&, const void* lm_head, const void* x, int n_rows, int d,
-                             int V, float inv_temp, Partials partials);
+                             int V, float inv_temp, Partials partials, bool reset_status = false);
 cudaError_t launch_lmhead_simt(const Ctx&, int dtype, const void* lm_head, const void* x,
-                               int n_rows, int d, int V, float inv_temp, Partials partials);
+                               int n_rows, int d, int V, float inv_temp, Partials partials,
+                               bool reset_status = false);
 cudaError_t launch_lmhead_merge(const Ctx&, int dtype, Partials partials, int n_rows, int V,
                                 int d, int k, float inv_temp, const void* lm_head, const void* x,
                                 int32_t* out_ids, float* out_logp);

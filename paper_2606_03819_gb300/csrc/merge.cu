@@ -105,6 +105,144 @@ __device__ unsigned long long block_kth_largest(const unsigned long long* keys, 
     return prefix;
 }
 
+// Shared state of block_kth_largest_fast.
+constexpr int kBuckets = 256;
+constexpr int kCollectCap = 256;
+struct SelectSmem {
+    int hist[kBuckets];
+    unsigned long long coll[kCollectCap];
+    float wmax[kThreads / 32], wmin[kThreads / 32];
+    int wcnt[kThreads / 32];
+    float vmin, scale;
+    int total, bucket, rem, count, n_coll;
+    unsigned long long found;
+};
+
+// The k-th largest non-zero key of keys[0..n) (zero keys are empty slots and rank below all),
+// or 0 when fewer than k keys are non-zero. One histogram pass over 256 equal-width buckets of
+// the key values (a monotone map, so the k-th largest key lies in the bucket where the count from
+// the top reaches k), then an exact rank among the few keys of that bucket. Falls back to the
+// byte-wise radix select when the values are all equal, not finite, or crowd one bucket.
+__device__ unsigned long long block_kth_largest_fast(const unsigned long long* keys, int n, int k, SelectSmem& B,
+                                                     int* hist, int* sel, unsigned long long* found) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    float vmax = -INFINITY, vmin = INFINITY;
+    int cnt = 0;
+    for (int i = tid; i < n; i += kThreads) {
+        const unsigned long long key = keys[i];
+        if (key != 0ull) {
+            const float v = key_value(key);
+            vmax = fmaxf(vmax, v);
+            vmin = fminf(vmin, v);
+            ++cnt;
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
+        vmin = fminf(vmin, __shfl_xor_sync(0xffffffffu, vmin, o));
+        cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+    }
+    if (lane == 0) {
+        B.wmax[warp] = vmax;
+        B.wmin[warp] = vmin;
+        B.wcnt[warp] = cnt;
+    }
+    for (int i = tid; i < kBuckets; i += kThreads) B.hist[i] = 0;
+    __syncthreads();
+    if (tid == 0) {
+        float mx = -INFINITY, mn = INFINITY;
+        int c = 0;
+        for (int w = 0; w < kThreads / 32; ++w) {
+            mx = fmaxf(mx, B.wmax[w]);
+            mn = fminf(mn, B.wmin[w]);
+            c += B.wcnt[w];
+        }
+        B.total = c;
+        B.vmin = mn;
+        const float range = mx - mn;
+        B.scale = (range > 0.0f && isfinite(range)) ? static_cast<float>(kBuckets) / range : 0.0f;
+        B.n_coll = 0;
+    }
+    __syncthreads();
+    const int total = B.total;
+    const float scale = B.scale, vlo = B.vmin;
+    if (total < k) {
+        __syncthreads();
+        return 0ull;
+    }
+    if (scale == 0.0f) {
+        __syncthreads();
+        return block_kth_largest(keys, n, k, hist, sel, found);
+    }
+    auto bucket_of = [&](unsigned long long key) {
+        const int b = static_cast<int>((key_value(key) - vlo) * scale);
+        return b < 0 ? 0 : (b >= kBuckets ? kBuckets - 1 : b);
+    };
+    const int n_pad = (n + kThreads - 1) / kThreads * kThreads;
+    for (int i = tid; i < n_pad; i += kThreads) {
+        int b = kBuckets;
+        if (i < n) {
+            const unsigned long long key = keys[i];
+            if (key != 0ull) b = bucket_of(key);
+        }
+        const unsigned peers = __match_any_sync(0xffffffffu, b);
+        if (b < kBuckets && lane == __ffs(peers) - 1) atomicAdd(&B.hist[b], __popc(peers));
+    }
+    __syncthreads();
+    if (warp == 0) {
+        // lane l holds buckets 8l .. 8l+7; inclusive suffix sums over lanes (high buckets first)
+        int local[8];
+        int sum = 0;
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+            local[b] = B.hist[lane * 8 + b];
+            sum += local[b];
+        }
+        int incl = sum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_down_sync(0xffffffffu, incl, o);
+            if (lane + o < 32) incl += v;
+        }
+        const int excl = incl - sum;
+        if (excl < k && k <= incl) {
+            int c = excl;
+            for (int b = 7; b >= 0; --b) {
+                if (c + local[b] >= k) {
+                    B.bucket = lane * 8 + b;
+                    B.rem = k - c;
+                    B.count = local[b];
+                    break;
+                }
+                c += local[b];
+            }
+        }
+    }
+    __syncthreads();
+    const int bk = B.bucket, rem = B.rem, cb = B.count;
+    if (cb > kCollectCap) {
+        __syncthreads();
+        return block_kth_largest(keys, n, k, hist, sel, found);
+    }
+    for (int i = tid; i < n; i += kThreads) {
+        const unsigned long long key = keys[i];
+        if (key != 0ull && bucket_of(key) == bk) B.coll[atomicAdd(&B.n_coll, 1)] = key;
+    }
+    __syncthreads();
+    // keys are distinct: exactly one has rem - 1 larger keys in the bucket
+    for (int i = tid; i < cb; i += kThreads) {
+        const unsigned long long key = B.coll[i];
+        int rank = 0;
+        for (int j = 0; j < cb; ++j) rank += B.coll[j] > key ? 1 : 0;
+        if (rank == rem - 1) B.found = key;
+    }
+    __syncthreads();
+    const unsigned long long r = B.found;
+    __syncthreads();   // every thread has read the shared results before they are reused
+    return r;
+}
+
 // <w, x> for one weight row (d elements) and x in shared memory (fp32), by one warp: lanes take
 // 8-element slices; all of a lane's 16-byte loads are issued before the multiply-adds.
 __device__ __forceinline__ float dot_row(const __nv_bfloat16* w, const float* xs, int d, int lane) {
@@ -188,6 +326,7 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
     MergeSmem S;
     merge_layout(n_tiles, d, dsm, &S);
     __shared__ int hist[256];
+    __shared__ SelectSmem SB;
     __shared__ float red_m[kThreads / 32], red_s[kThreads / 32];
     __shared__ int sel_info[3], n_flag, flag_list[kMergeExpandChunks], n_cand, n_sel, n_valid, n_chalf;
     __shared__ int chalf[kMaxK];
@@ -257,7 +396,7 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
 
     // 2. theta0 and the halves at or above it (at most k: the keys are distinct)
     const unsigned long long theta0 =
-        n_valid >= k ? block_kth_largest(S.hkey, nh, k, hist, sel_info, &found) : 0ull;
+        n_valid >= k ? block_kth_largest_fast(S.hkey, nh, k, SB, hist, sel_info, &found) : 0ull;
     for (int i = tid; i < nh; i += kThreads) {
         const unsigned long long key = S.hkey[i];
         if (key != 0ull && key >= theta0) {
@@ -294,7 +433,7 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
     unsigned long long theta = 0;
     for (;;) {
         const int nc = n_cand;
-        theta = nc >= k ? block_kth_largest(S.cand, nc, k, hist, sel_info, &found) : 0ull;
+        theta = nc >= k ? block_kth_largest_fast(S.cand, nc, k, SB, hist, sel_info, &found) : 0ull;
         const float tval = key_value(theta);
         if (tid == 0) n_flag = 0;
         __syncthreads();

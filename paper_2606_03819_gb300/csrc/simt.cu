@@ -17,9 +17,10 @@ constexpr int kKChunk = 32;
 // two) and the per-half max, sum of exp and best entry.
 __global__ void __launch_bounds__(256) lmhead_simt_kernel(const float* __restrict__ W, const float* __restrict__ X,
                                                           int n_rows, int d, int V, float inv_temp,
-                                                          Partials partials, int n_tiles) {
+                                                          Partials partials, int n_tiles, int* reset_status) {
     pdl_trigger();
     pdl_wait();
+    if (reset_status && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *reset_status = 0;
     __shared__ float xs[kRowsPerCta][kKChunk + 1];
     __shared__ float ws[kBlockV][kKChunk + 1];
     const int vt = blockIdx.x;
@@ -184,14 +185,14 @@ __global__ void __launch_bounds__(256) swiglu_simt_kernel(const float* __restric
 }  // namespace
 
 cudaError_t launch_lmhead_simt(const Ctx& ctx, int dtype, const void* lm_head, const void* x, int n_rows, int d,
-                               int V, float inv_temp, Partials partials) {
+                               int V, float inv_temp, Partials partials, bool reset_status) {
     if (dtype != TF_F32) return cudaErrorNotSupported;
     if (n_rows <= 0) return cudaSuccess;
     const int n_tiles = (V + kBlockV - 1) / kBlockV;
     dim3 grid(n_tiles, (n_rows + kRowsPerCta - 1) / kRowsPerCta);
     const cudaError_t e = launch_pdl(lmhead_simt_kernel, grid, dim3(256), 0, ctx.stream,
                                      static_cast<const float*>(lm_head), static_cast<const float*>(x), n_rows, d, V,
-                                     inv_temp, partials, n_tiles);
+                                     inv_temp, partials, n_tiles, reset_status ? ctx.status : static_cast<int*>(nullptr));
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 

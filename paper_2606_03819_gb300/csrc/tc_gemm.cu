@@ -54,6 +54,7 @@ struct EpiParams {
     int ld_partial;              //          columns nb * n_total + n
     size_t partial_split_stride; // elements between consecutive k-splits
     int n_total;                 // N of the whole GEMM (n_ntiles * BN)
+    int reset_status;            // LMHEAD: zero *status first (the first kernel of a stage-1 call)
 };
 
 // Work unit u -> (N tile, M-tile group, K split); consecutive units share the N tile and K split
@@ -193,6 +194,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
     if (!(warp == 0 && lane == 0)) pdl_wait();   // the producer waits after its weight prefetch
+    // a call's status word starts at zero; cleared here, after every earlier kernel has finished,
+    // instead of by a separate memset that would end the overlap with the previous kernel
+    if (EPI == EPI_LMHEAD && ep.reset_status && blockIdx.x == 0 && threadIdx.x == 64 && status) *status = 0;
 
     if (warp == 0) {
         // ------------------------------------------------------------------ TMA producer
@@ -554,7 +558,7 @@ cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& t
 }  // namespace
 
 cudaError_t launch_lmhead_tc(const Ctx& ctx, const void* lm_head, const void* x, int n_rows, int d, int V,
-                             float inv_temp, Partials partials) {
+                             float inv_temp, Partials partials, bool reset_status) {
     if (n_rows <= 0) return cudaSuccess;
     const int n_tiles = (V + kBlockV - 1) / kBlockV;
     const int m_tiles = (n_rows + kBM - 1) / kBM;
@@ -570,6 +574,7 @@ cudaError_t launch_lmhead_tc(const Ctx& ctx, const void* lm_head, const void* x,
     ep.partials = partials;
     ep.V = V;
     ep.inv_temp = inv_temp;
+    ep.reset_status = reset_status ? 1 : 0;
     if (m_tiles == 1) return run_gemm<EPI_LMHEAD, 1, 1, kBlockV, 4>(ctx, tx, tw, tw, n_rows, d, n_tiles, 1, ep);
     return run_gemm<EPI_LMHEAD, 1, 1, kBlockV, 4, 2>(ctx, tx, tw, tw, n_rows, d, n_tiles, (m_tiles + 1) / 2, ep);
 }
