@@ -587,29 +587,34 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
     const uint4* __restrict__ norm_e, const int32_t* __restrict__ root_tok, const int32_t* __restrict__ top_ids,
     int gamma, int M, int K1, int R, int d, int V, float eps, uint4* __restrict__ X, int* status) {
     pdl_trigger();
-    pdl_wait();
     constexpr int kMaxPerThread = 4;          // d <= 256 * 8 * 4 = 8192
     __shared__ double red[2][8];
     __shared__ float scale[4];                // hi, lo of the hidden half; hi, lo of the embedding half
     const int row = blockIdx.x;
     const int sq = row / R, r = row - sq * R;
     const int hid = sq * gamma + stage2_hidden_index(r, M);
+
+    const int dv = d / 8;
+    // the hidden state is a step input (no kernel writes it): read before waiting for the
+    // previous kernel, which produces the candidate tokens
+    const uint4* h = hidden + static_cast<size_t>(hid) * dv;
+    uint4 hv[kMaxPerThread], ev[kMaxPerThread];
+#pragma unroll
+    for (int i = 0; i < kMaxPerThread; ++i) {
+        const int c = threadIdx.x + i * 256;
+        if (c < dv) hv[i] = h[c];
+    }
+    pdl_wait();
     int tok = (r == 0) ? root_tok[sq] : top_ids[(static_cast<size_t>(sq) * gamma + (r - 1) / M) * K1 + (r - 1) % M];
     if (tok < 0 || tok >= V) {
         if (threadIdx.x == 0) set_status(status, TF_DEV_BAD_TOKEN);
         tok = 0;
     }
-    const int dv = d / 8;
-    const uint4* h = hidden + static_cast<size_t>(hid) * dv;
     const uint4* e = embed + static_cast<size_t>(tok) * dv;
-    uint4 hv[kMaxPerThread], ev[kMaxPerThread];
 #pragma unroll
     for (int i = 0; i < kMaxPerThread; ++i) {
         const int c = threadIdx.x + i * 256;
-        if (c < dv) {
-            hv[i] = h[c];
-            ev[i] = e[c];
-        }
+        if (c < dv) ev[i] = e[c];
     }
     float sh = 0.0f, ch = 0.0f, se = 0.0f, ce = 0.0f;
 #pragma unroll
