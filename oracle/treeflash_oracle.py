@@ -19,6 +19,8 @@ What it computes (TreeFlash, "Parallel AR-Approximation for Faster Speculative D
   candidate m of depth i gets the children distribution q'^(m)_{t+i+1}.
 * The verifier's tree-attention mask and position ids for the B+1 nodes (the tree is
   verified in one parallel forward pass, Sec. 1 and Sec. 3).
+* The verification walk over a drafted tree: acceptance by an equality check with the
+  verifier's tokens (Sec. 3) and the step's block efficiency tau (Sec. 4).
 
 Everything is float64 (numpy). Library primitives used as steps: matrix products, sorting,
 exp/log. Readings of points the paper leaves open (each also listed in the design notes):
@@ -295,6 +297,37 @@ def tree_mask(parent: np.ndarray, depth: np.ndarray, root_pos: int):
             j = parent[j] if j > 0 else -1
     pos = np.where(present, root_pos + depth, -1).astype(np.int64)
     return mask, pos
+
+def accept_walk(tok: np.ndarray, parent: np.ndarray, verifier_tok: np.ndarray):
+    """Verification of a drafted tree by an equality check, and the step's block efficiency.
+
+    Sec. 3: token selection is deterministic, so a drafted token is accepted exactly when it
+    equals the verifier's own next token at that position. verifier_tok[i] is the verifier's
+    next token at the position of node i (its choice after the path root..i). Starting at the
+    root, the walk moves to the child of the current node whose token equals the verifier's
+    token there, while such a child exists (children of one node carry distinct tokens; if an
+    invalid tree repeats one, the smallest node index is taken). Sec. 4: block efficiency tau
+    counts the accepted tokens plus the verifier's residual token.
+
+    Returns (path, bonus): path = accepted node indices, root first (the tree rows whose KV
+    entries the verifier keeps); bonus = verifier_tok at the last accepted node. The step
+    accepts len(path) - 1 drafted tokens and gains tau = len(path) tokens. Missing nodes
+    (parent -1 beyond the root) are never children.
+    """
+    n = len(tok)
+    children = [[] for _ in range(n)]
+    for c in range(1, n):
+        if parent[c] >= 0:
+            children[int(parent[c])].append(c)
+    path = [0]
+    cur = 0
+    while True:
+        match = [c for c in children[cur] if tok[c] == verifier_tok[cur]]
+        if not match:
+            break
+        cur = match[0]
+        path.append(cur)
+    return path, int(verifier_tok[cur])
 
 
 # ---------------------------------------------------------------------------------------

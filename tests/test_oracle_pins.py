@@ -426,3 +426,62 @@ def test_oracle_matches_frozen_golden():
         assert res.tree.tok.tolist() == g["tok"]
         assert res.tree.parent.tolist() == g["parent"]
         np.testing.assert_allclose(res.tree.score, g["score"], rtol=1e-12)
+
+
+# ------------------------------------------------------------------ verification walk
+
+
+def test_accept_walk_hand_worked():
+    # root 0 -> 1 (5), 2 (7); 1 -> 3 (9), 4 (11); 3 -> 5 (2); node 6 missing
+    tok = np.array([100, 5, 7, 9, 11, 2, -1])
+    par = np.array([-1, 0, 0, 1, 1, 3, -1])
+    # the verifier continues 5, 9, 2 and then proposes 42: three drafted tokens accepted, tau 4
+    path, bonus = O.accept_walk(tok, par, np.array([5, 9, 0, 2, 0, 42, 0]))
+    assert path == [0, 1, 3, 5] and bonus == 42
+    # the verifier's first token is not drafted: nothing accepted, the step gains one token
+    path, bonus = O.accept_walk(tok, par, np.array([8, 9, 0, 2, 0, 42, 0]))
+    assert path == [0] and bonus == 8
+    # the second branch, stopping where no child matches (node 4 has none)
+    path, bonus = O.accept_walk(tok, par, np.array([5, 11, 0, 2, 17, 42, 0]))
+    assert path == [0, 1, 4] and bonus == 17
+    # a missing node is never accepted, even if its token matches
+    path, _ = O.accept_walk(tok, par, np.array([7, 0, -1, 0, 0, 0, 0]))
+    assert path == [0, 2]
+
+
+def _node_paths(par):
+    # every root path, as node indices, by walking parent links from each node
+    out = []
+    for i in range(len(par)):
+        if i > 0 and par[i] < 0:
+            continue
+        p, j = [], i
+        while j > 0:
+            p.append(j)
+            j = int(par[j])
+        out.append([0] + p[::-1])
+    return out
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_accept_walk_is_the_longest_consistent_root_path(seed):
+    # brute force over all root paths of an oracle tree: the accepted path is the longest path
+    # along which every drafted token equals the verifier's token at its parent, and the bonus
+    # is the verifier's token at its end
+    res = _run(seed=seed, B=12, M=3)
+    tok, par = res.tree.tok, res.tree.parent
+    n = len(tok)
+    rng = np.random.default_rng(100 + seed)
+    children = {i: [c for c in range(1, n) if par[c] == i] for i in range(n)}
+    ver = np.empty(n, dtype=np.int64)
+    for i in range(n):
+        if children[i] and rng.random() < 0.7:
+            ver[i] = tok[rng.choice(children[i])]    # the verifier agrees with one child
+        else:
+            ver[i] = 10_000 + i                      # a token no node carries
+    consistent = [p for p in _node_paths(par) if all(tok[b] == ver[a] for a, b in zip(p, p[1:]))]
+    best = max(consistent, key=len)
+    assert sum(1 for p in consistent if len(p) == len(best)) == 1
+    path, bonus = O.accept_walk(tok, par, ver)
+    assert path == best and bonus == ver[best[-1]]
+    assert 1 <= len(path) <= res.tree.depth.max() + 1
