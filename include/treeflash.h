@@ -194,6 +194,25 @@ tf_status tf_draft_tree_host(const tf_dims* dims, const tf_weights* w, const voi
                              float* node_score, uint8_t* mask, int32_t* pos_ids,
                              int32_t* dev_status, void* ws, size_t ws_bytes, tf_stream_t stream);
 
+/* The verification step that follows drafting (Sec. 3: token selection is deterministic, so
+ * the verifier accepts a drafted token exactly when it equals its own next token at that
+ * position; Sec. 4: block efficiency tau counts the accepted tokens plus the verifier's
+ * residual token). For every sequence, from the root, move to the child of the current node
+ * whose token equals the verifier's token at the current node, while one exists.
+ *  node_tok, node_parent [b, B+1] int32: a drafted tree (as tf_build_tree writes it; missing
+ *                nodes have parent -1 and are never accepted)
+ *  verifier_tok [b, B+1] int32: the verifier's next token at each node's position, i.e. its
+ *                choice after the path root..node (from the single parallel pass over the tree)
+ *  accept_len  [b] int32 out: drafted tokens accepted, 0..gamma; the step gains accept_len + 1
+ *  accept_path [b, gamma+1] int32 out: accepted node indices, root first, then -1: the tree rows
+ *                whose KV-cache entries the verifier keeps, in order
+ *  next_tok    [b] int32 out: the verifier's token at the last accepted node (the bonus token)
+ * Children of one node carry distinct tokens; if an invalid tree repeats one, the smallest node
+ * index is taken. At most gamma steps are taken, whatever the parent array holds. */
+tf_status tf_accept_walk(const tf_dims* dims, const int32_t* node_tok, const int32_t* node_parent,
+                         const int32_t* verifier_tok, int32_t* accept_len, int32_t* accept_path,
+                         int32_t* next_tok, tf_stream_t stream);
+
 /* ------------------------------------------------------------------------------------------
  * The pieces the stage calls are made of. tf_stage1_marginals is tf_lmhead_partials +
  * tf_lmhead_merge on the hidden states; tf_stage2_ar_approx is tf_ar_approx followed by the

@@ -46,7 +46,7 @@ class TfWeights(ctypes.Structure):
 EXPORTS = ("tf_status_string", "tf_version", "tf_kernel_launches", "tf_workspace_size", "tf_status_reset", "tf_status_read",
            "tf_stage1_marginals", "tf_stage2_ar_approx", "tf_build_tree", "tf_tree_mask",
            "tf_draft_tree_host", "tf_lmhead_partials", "tf_lmhead_merge", "tf_ar_approx",
-           "tf_workspace_h_prime", "tf_workspace_view", "tf_stage1_marginals_static")
+           "tf_workspace_h_prime", "tf_workspace_view", "tf_stage1_marginals_static", "tf_accept_walk")
 
 _lib = None
 
@@ -81,6 +81,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
         "tf_workspace_h_prime": (ctypes.c_int, [D, P, SZ, ctypes.POINTER(P)]),
         "tf_workspace_view": (ctypes.c_int, [D, P, SZ, I32, ctypes.POINTER(P), ctypes.POINTER(SZ)]),
         "tf_stage1_marginals_static": (ctypes.c_int, [D, W, P, P, P, P, P]),
+        "tf_accept_walk": (ctypes.c_int, [D, P, P, P, P, P, P, P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -226,6 +227,13 @@ def tf_draft_tree_host(dims: Dims, w: dict, hidden, root_tok, root_pos, node_tok
     if st not in (TF_OK, TF_ERR_DEVICE_STATUS):
         _check("tf_draft_tree_host", st)
     return st
+
+
+def tf_accept_walk(dims: Dims, node_tok, node_parent, verifier_tok, accept_len, accept_path, next_tok,
+                   stream=None):
+    _check("tf_accept_walk", load_library().tf_accept_walk(
+        ctypes.byref(dims.c()), _ptr(node_tok), _ptr(node_parent), _ptr(verifier_tok), _ptr(accept_len),
+        _ptr(accept_path), _ptr(next_tok), _stream(stream)))
 
 
 def tf_lmhead_partials(dims: Dims, lm_head, x, n_rows: int, ws, stream=None):

@@ -346,6 +346,18 @@ tf_status tf_tree_mask(const tf_dims* dims, const int32_t* node_parent, const in
     return cuda_status(launch_tree_mask(ctx, D.b, D.B, node_parent, node_depth, root_pos, mask, pos_ids));
 }
 
+tf_status tf_accept_walk(const tf_dims* dims, const int32_t* node_tok, const int32_t* node_parent,
+                         const int32_t* verifier_tok, int32_t* accept_len, int32_t* accept_path, int32_t* next_tok,
+                         tf_stream_t stream) {
+    Dims D;
+    TF_TRY(check_dims(dims, &D));
+    if (!node_tok || !node_parent || !verifier_tok || !accept_len || !accept_path || !next_tok)
+        return TF_ERR_INVALID_ARG;
+    Ctx ctx{reinterpret_cast<cudaStream_t>(stream), 0, nullptr};
+    return cuda_status(launch_accept_walk(ctx, D.b, D.B, D.gamma, node_tok, node_parent, verifier_tok, accept_len,
+                                          accept_path, next_tok));
+}
+
 tf_status tf_workspace_h_prime(const tf_dims* dims, void* ws, size_t ws_bytes, void** h_prime) {
     if (!h_prime) return TF_ERR_INVALID_ARG;
     Dims D;

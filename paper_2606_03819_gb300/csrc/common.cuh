@@ -183,6 +183,9 @@ cudaError_t launch_build_tree(const Ctx&, int b, int gamma, int M, int K1, int K
                               const float* top_logp, const int32_t* child_ids,
                               const float* child_logp, int32_t* node_tok, int32_t* node_parent,
                               int32_t* node_depth, float* node_score, int32_t* dev_status);
+cudaError_t launch_accept_walk(const Ctx&, int b, int B, int gamma, const int32_t* node_tok,
+                               const int32_t* node_parent, const int32_t* verifier_tok,
+                               int32_t* accept_len, int32_t* accept_path, int32_t* next_tok);
 cudaError_t launch_tree_mask(const Ctx&, int b, int B, const int32_t* node_parent,
                              const int32_t* node_depth, const int32_t* root_pos, uint8_t* mask,
                              int32_t* pos_ids);

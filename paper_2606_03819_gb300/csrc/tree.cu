@@ -546,6 +546,51 @@ __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __
     }
 }
 
+// ------------------------------------------------------------------------------------------
+// Verification walk (Sec. 3: a drafted token is accepted iff it equals the verifier's token at
+// its parent's position; Sec. 4: the step gains the accepted tokens plus the verifier's residual
+// token). One warp per sequence: from the root, each step finds the child of the current node
+// whose token equals the verifier's token there (a ballot over all nodes; the smallest index if
+// an invalid tree repeats a token) and moves to it. At most gamma steps (the depth cap), so a
+// corrupt parent array cannot loop.
+// ------------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(32) accept_walk_kernel(int n, int gamma, const int32_t* __restrict__ node_tok,
+                                                         const int32_t* __restrict__ node_parent,
+                                                         const int32_t* __restrict__ verifier_tok,
+                                                         int32_t* __restrict__ accept_len,
+                                                         int32_t* __restrict__ accept_path,
+                                                         int32_t* __restrict__ next_tok) {
+    pdl_trigger();
+    pdl_wait();
+    constexpr unsigned kFull = 0xffffffffu;
+    const int s = blockIdx.x, lane = threadIdx.x;
+    const int32_t* tok = node_tok + static_cast<size_t>(s) * n;
+    const int32_t* par = node_parent + static_cast<size_t>(s) * n;
+    const int32_t* ver = verifier_tok + static_cast<size_t>(s) * n;
+    int32_t* path = accept_path + static_cast<size_t>(s) * (gamma + 1);
+    int cur = 0, len = 0;
+    if (lane == 0) path[0] = 0;
+    for (int step = 0; step < gamma; ++step) {
+        const int want = ver[cur];
+        int found = -1;
+        for (int c0 = 1; c0 < n && found < 0; c0 += 32) {
+            const int c = c0 + lane;
+            const bool m = c < n && par[c] == cur && tok[c] == want;
+            const unsigned bal = __ballot_sync(kFull, m);
+            if (bal) found = c0 + __ffs(bal) - 1;
+        }
+        if (found < 0) break;
+        cur = found;
+        ++len;
+        if (lane == 0) path[len] = cur;
+    }
+    for (int i = len + 1 + lane; i <= gamma; i += 32) path[i] = -1;
+    if (lane == 0) {
+        accept_len[s] = len;
+        next_tok[s] = ver[cur];
+    }
+}
+
 }  // namespace
 
 // Error-free sum (Knuth's TwoSum): s + c tracks a running sum to about twice fp32 precision.
@@ -738,6 +783,14 @@ cudaError_t launch_tree_mask(const Ctx& ctx, int b, int B, const int32_t* node_p
     if (e != cudaSuccess) return e;
     e = launch_pdl(tree_mask_kernel, dim3(b), dim3(256), smem, ctx.stream, n, node_parent, node_depth, root_pos, mask,
                    pos_ids);
+    return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+cudaError_t launch_accept_walk(const Ctx& ctx, int b, int B, int gamma, const int32_t* node_tok,
+                               const int32_t* node_parent, const int32_t* verifier_tok, int32_t* accept_len,
+                               int32_t* accept_path, int32_t* next_tok) {
+    const cudaError_t e = launch_pdl(accept_walk_kernel, dim3(b), dim3(32), 0, ctx.stream, B + 1, gamma, node_tok,
+                                     node_parent, verifier_tok, accept_len, accept_path, next_tok);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
