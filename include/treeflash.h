@@ -83,8 +83,8 @@ typedef struct {
     int32_t V;            /* vocabulary size, K1 <= V < 2^31 */
     int32_t I;            /* approximator intermediate width; TF_BF16 needs I % 64 == 0 */
     int32_t gamma;        /* block size (max depth), 1..64 */
-    int32_t M;            /* stage-1 candidates per depth (M-ary branching), 1..32 */
-    int32_t K2;           /* children kept per distribution, 1..64; K2 >= B is exact */
+    int32_t M;            /* stage-1 candidates per depth (M-ary branching), 1..64 */
+    int32_t K2;           /* children kept per distribution, 1..512; K2 >= B is exact */
     int32_t B;            /* draft budget (nodes besides the root), 1..1023 */
     float temperature;    /* logits are W_lm x / temperature, temperature > 0 */
     float rms_eps;        /* RMSNorm epsilon of Eq. 1's normalisations */
@@ -229,7 +229,7 @@ tf_status tf_lmhead_partials(const tf_dims* dims, const void* lm_head, const voi
                              int32_t n_rows, void* ws, size_t ws_bytes, tf_stream_t stream);
 
 /* Merge the partials of tf_lmhead_partials (same n_rows) into each row's log-sum-exp and exact
- * top-k (k <= 64): out_ids [n_rows, k] int32, out_logp [n_rows, k] float = logit - LSE. A chunk
+ * top-k (k <= 512): out_ids [n_rows, k] int32, out_logp [n_rows, k] float = logit - LSE. A chunk
  * whose third-largest logit could still be a member of the top-k has its 32 logits recomputed
  * exactly from lm_head and x (sets TF_DEV_RECOMPUTED), so the result never depends on keeping
  * only two entries per chunk. */

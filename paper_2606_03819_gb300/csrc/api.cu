@@ -10,7 +10,7 @@
 #include "common.cuh"
 
 namespace tf {
-size_t merge_smem_bytes(int n_tiles, int d);
+size_t merge_smem_bytes(int n_tiles, int d, int k);
 
 namespace {
 std::atomic<unsigned long long> g_kernel_launches{0};
@@ -57,7 +57,7 @@ tf_status check_dims(const tf_dims* dims, Dims* o) {
     if (d.dtype == TF_BF16 && (d.d % 64 != 0 || (d.mode == TF_MODE_AR && d.I % 64 != 0)))
         return TF_ERR_UNSUPPORTED;
     const int n_tiles = (d.V + kBlockV - 1) / kBlockV;
-    if (merge_smem_bytes(n_tiles, d.d) > kMaxMergeSmem) return TF_ERR_UNSUPPORTED;
+    if (merge_smem_bytes(n_tiles, d.d, K1) > kMaxMergeSmem) return TF_ERR_UNSUPPORTED;
     const long long R = 1 + static_cast<long long>(d.M) * (d.gamma - 1);
     if (static_cast<long long>(d.batch) * R > (1ll << 30) || static_cast<long long>(d.batch) * d.gamma > (1ll << 30))
         return TF_ERR_UNSUPPORTED;

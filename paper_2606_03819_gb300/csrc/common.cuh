@@ -13,11 +13,11 @@ namespace tf {
 constexpr int kBlockV = 256;        // vocabulary entries per LM-head block (one MMA N-tile)
 constexpr int kChunk = 32;           // vocabulary columns per chunk (one TMEM load per row)
 constexpr int kChunks = kBlockV / kChunk;  // chunks per block
-constexpr int kMaxK = 64;           // largest top-k a merge can return
-constexpr int kMaxM = 32;           // largest M (the builder tests membership with one warp)
+constexpr int kMaxK = 512;          // largest top-k a merge can return
+constexpr int kMaxM = 64;           // largest M (the builder tests membership with two ballots)
 constexpr int kMaxB = 1023;         // largest draft budget
 constexpr int kMaxGamma = 64;
-constexpr int kMergeExpandChunks = kMaxK;  // chunks a merge may recompute exactly
+constexpr int kMergeExpandChunks = 64;     // chunks a merge may recompute exactly
 constexpr int kMaxKSplits = 4;        // split-K factor of the approximator GEMMs (workspace sized for it)
 
 // What the LM-head pass leaves per (row, vocabulary block of 256). Both arrays are indexed

@@ -10,7 +10,8 @@
 //      k-th largest candidate key comes from a radix select over 64-bit keys;
 //   3. certifies the result: a chunk whose third-largest value reaches the k-th candidate may
 //      hide further members of the top k. Those chunks' 32 logits are recomputed exactly from
-//      lm_head and x, replace the chunk's two candidates, and the selection is redone;
+//      lm_head and x (in rounds of at most 64 chunks), replace the chunk's two candidates, and
+//      the selection is redone;
 //   4. writes the k winners sorted, as (id, logit - LSE).
 // The result is the exact top-k of the full vocabulary whatever the input; a recompute needs
 // three members of the top k in one 32-column chunk (about one row in 500 on random data).
@@ -279,18 +280,20 @@ __device__ __forceinline__ float dot_row(const float* w, const float* xs, int d,
     return acc;
 }
 
-// Shared-memory layout of one merge CTA (dynamic part).
-constexpr int kDetailChunks = kMaxK * (kChunks / 2);           // chunks of the <= k halves kept
-constexpr int kCandCap = 2 * kDetailChunks + kMergeExpandChunks * kChunk;
+// Shared-memory layout of one merge CTA (dynamic part), for a top-k of k.
 struct MergeSmem {
     unsigned long long* hkey;   // [n_halves] best key of every half block (0 = empty)
-    unsigned long long* cand;   // [kCandCap]
-    float* c3;                  // [kDetailChunks] third value of each kept chunk (bound on the rest)
-    int* cbase;                 // [kDetailChunks] first vocabulary id of each kept chunk
-    uint8_t* expanded;          // [kDetailChunks] chunk recomputed
+    unsigned long long* cand;   // [2 * 4k + kMergeExpandChunks * kChunk]
+    unsigned long long* cand2;  // the same size: the compacted set of the next round
+    unsigned long long* sel;    // [k] the winners
+    float* c3;                  // [4k] third value of each kept chunk (bound on the rest)
+    int* cbase;                 // [4k] first vocabulary id of each kept chunk
+    int* chalf;                 // [k] the halves at or above theta0
+    uint8_t* expanded;          // [4k] chunk recomputed
     float* xs;                  // [d] x of the row in fp32, staged only for a recompute
 };
-__host__ __device__ inline size_t merge_layout(int n_tiles, int d, uint8_t* base, MergeSmem* m) {
+__host__ __device__ inline size_t merge_layout(int n_tiles, int d, int k, uint8_t* base, MergeSmem* m) {
+    const size_t detail = static_cast<size_t>(k) * (kChunks / 2);   // chunks of the k halves kept
     size_t off = 0;
     auto take = [&](size_t bytes) {
         uint8_t* p = base ? base + off : nullptr;
@@ -298,16 +301,22 @@ __host__ __device__ inline size_t merge_layout(int n_tiles, int d, uint8_t* base
         return p;
     };
     uint8_t* hk = take(static_cast<size_t>(2) * n_tiles * 8);
-    uint8_t* cd = take(static_cast<size_t>(kCandCap) * 8);
-    uint8_t* c3 = take(static_cast<size_t>(kDetailChunks) * 4);
-    uint8_t* cb = take(static_cast<size_t>(kDetailChunks) * 4);
-    uint8_t* ex = take(kDetailChunks);
+    uint8_t* cd = take((2 * detail + static_cast<size_t>(kMergeExpandChunks) * kChunk) * 8);
+    uint8_t* cd2 = take((2 * detail + static_cast<size_t>(kMergeExpandChunks) * kChunk) * 8);
+    uint8_t* se = take(static_cast<size_t>(k) * 8);
+    uint8_t* c3 = take(detail * 4);
+    uint8_t* cb = take(detail * 4);
+    uint8_t* ch = take(static_cast<size_t>(k) * 4);
+    uint8_t* ex = take(detail);
     uint8_t* xs = take(static_cast<size_t>(d) * 4);
     if (m) {
         m->hkey = reinterpret_cast<unsigned long long*>(hk);
         m->cand = reinterpret_cast<unsigned long long*>(cd);
+        m->cand2 = reinterpret_cast<unsigned long long*>(cd2);
+        m->sel = reinterpret_cast<unsigned long long*>(se);
         m->c3 = reinterpret_cast<float*>(c3);
         m->cbase = reinterpret_cast<int*>(cb);
+        m->chalf = reinterpret_cast<int*>(ch);
         m->expanded = ex;
         m->xs = reinterpret_cast<float*>(xs);
     }
@@ -324,13 +333,13 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
     pdl_wait();
     extern __shared__ __align__(16) uint8_t dsm[];
     MergeSmem S;
-    merge_layout(n_tiles, d, dsm, &S);
+    merge_layout(n_tiles, d, k, dsm, &S);
+    const int n_detail = k * (kChunks / 2);
     __shared__ int hist[256];
     __shared__ SelectSmem SB;
     __shared__ float red_m[kThreads / 32], red_s[kThreads / 32];
-    __shared__ int sel_info[3], n_flag, flag_list[kMergeExpandChunks], n_cand, n_sel, n_valid, n_chalf;
-    __shared__ int chalf[kMaxK];
-    __shared__ unsigned long long sel[kMaxK], found;
+    __shared__ int sel_info[3], n_flag, flag_list[kMergeExpandChunks], n_cand, n_next, n_sel, n_valid, n_chalf;
+    __shared__ unsigned long long found;
     __shared__ float zbuf[kMergeExpandChunks * kChunk];
     __shared__ float lse_s;
 
@@ -372,7 +381,7 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
             }
         }
     }
-    for (int i = tid; i < kDetailChunks; i += kThreads) S.expanded[i] = 0;
+    for (int i = tid; i < n_detail; i += kThreads) S.expanded[i] = 0;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
@@ -401,14 +410,14 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
         const unsigned long long key = S.hkey[i];
         if (key != 0ull && key >= theta0) {
             const int slot = atomicAdd(&n_chalf, 1);
-            if (slot < kMaxK) chalf[slot] = i;
+            if (slot < k) S.chalf[slot] = i;
         }
     }
     __syncthreads();
-    const int nch = min(n_chalf, kMaxK);
+    const int nch = min(n_chalf, k);
     // their chunks: the two largest entries at or above theta0 become candidates
     for (int i = tid; i < nch * (kChunks / 2); i += kThreads) {
-        const int h = chalf[i >> 2];
+        const int h = S.chalf[i >> 2];
         const int tile = h >> 1, chunk = (h & 1) * (kChunks / 2) + (i & 3);
         const float4 q = partials.chunks[partials.chunk_at(tile, chunk, row)];
         const int v0 = tile * kBlockV + chunk * kChunk;
@@ -427,13 +436,18 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
     __syncthreads();
 
     // 3. select; a kept chunk whose third value reaches the k-th candidate may hide members of
-    //    the top k, so its 32 logits are recomputed exactly and the selection is redone
-    int n_expanded = 0;
+    //    the top k, so its 32 logits are recomputed exactly and the selection is redone. Chunks
+    //    are recomputed in rounds of at most kMergeExpandChunks; after each round only keys at or
+    //    above the k-th candidate survive (the candidates are logits of the row, so every member
+    //    of the true top k is at or above it, and it only rises), which bounds the set by
+    //    k + kMergeExpandChunks * kChunk whatever the input.
     bool x_staged = false;
     unsigned long long theta = 0;
+    unsigned long long* cand = S.cand;
+    unsigned long long* spare = S.cand2;
     for (;;) {
         const int nc = n_cand;
-        theta = nc >= k ? block_kth_largest_fast(S.cand, nc, k, SB, hist, sel_info, &found) : 0ull;
+        theta = nc >= k ? block_kth_largest_fast(cand, nc, k, SB, hist, sel_info, &found) : 0ull;
         const float tval = key_value(theta);
         if (tid == 0) n_flag = 0;
         __syncthreads();
@@ -445,21 +459,19 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
             }
         }
         __syncthreads();
-        const int nf = n_flag;
+        const int nf = min(n_flag, kMergeExpandChunks);   // the rest wait for the next round
         if (nf == 0) break;
-        if (n_expanded + nf > kMergeExpandChunks) {
-            // more chunks in doubt than the recompute budget: keep the answer and say so
-            if (tid == 0) set_status(status, TF_DEV_NONFINITE);
-            break;
+        if (tid == 0) {
+            set_status(status, TF_DEV_RECOMPUTED);
+            n_next = 0;
         }
-        if (tid == 0) set_status(status, TF_DEV_RECOMPUTED);
-        // exact logits of every flagged chunk: x staged once in shared memory, then one warp per
+        // exact logits of this round's chunks: x staged once in shared memory, then one warp per
         // column with all of its 16-byte weight loads issued before the multiply-adds
         if (!x_staged) {
             for (int i = tid; i < d; i += kThreads) S.xs[i] = to_f32(x[static_cast<size_t>(row) * d + i]);
             x_staged = true;
-            __syncthreads();
         }
+        __syncthreads();
         for (int q = warp; q < nf * kChunk; q += kThreads / 32) {
             const int f = q / kChunk, cc = q - f * kChunk;
             const int v = S.cbase[flag_list[f]] + cc;
@@ -467,22 +479,32 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
             if (lane == 0) zbuf[q] = v < V ? acc * inv_temp : -INFINITY;
         }
         __syncthreads();
-        // the flagged chunks' two candidates leave the candidate set; all their logits enter it
-        for (int j = tid; j < n_cand; j += kThreads) {
-            const int id = key_id(S.cand[j]);
+        // the next set: surviving keys not from this round's chunks, then their exact logits
+        for (int j = tid; j < nc; j += kThreads) {
+            const unsigned long long key = cand[j];
+            if (key == 0ull || key < theta) continue;
+            const int id = key_id(key);
+            bool mine = false;
             for (int f = 0; f < nf; ++f) {
                 const int v0 = S.cbase[flag_list[f]];
-                if (id >= v0 && id < v0 + kChunk) S.cand[j] = 0ull;
+                mine = mine || (id >= v0 && id < v0 + kChunk);
             }
+            if (!mine) spare[atomicAdd(&n_next, 1)] = key;
         }
-        __syncthreads();
         for (int q = tid; q < nf * kChunk; q += kThreads) {
             const int f = q / kChunk, cc = q - f * kChunk;
             const int v = S.cbase[flag_list[f]] + cc;
-            if (v < V) S.cand[atomicAdd(&n_cand, 1)] = cand_key(zbuf[q], v);
+            if (v < V) {
+                const unsigned long long key = cand_key(zbuf[q], v);
+                if (key >= theta) spare[atomicAdd(&n_next, 1)] = key;
+            }
         }
         for (int f = tid; f < nf; f += kThreads) S.expanded[flag_list[f]] = 1;
-        n_expanded += nf;
+        __syncthreads();
+        if (tid == 0) n_cand = n_next;
+        unsigned long long* t = cand;
+        cand = spare;
+        spare = t;
         __syncthreads();
     }
 
@@ -491,19 +513,19 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
     __syncthreads();
     const int nc = n_cand;
     for (int i = tid; i < nc; i += kThreads) {
-        const unsigned long long key = S.cand[i];
+        const unsigned long long key = cand[i];
         if (key != 0ull && key >= theta) {
             const int slot = atomicAdd(&n_sel, 1);
-            if (slot < kMaxK) sel[slot] = key;
+            if (slot < k) S.sel[slot] = key;
         }
     }
     __syncthreads();
     const int ns = min(n_sel, k);
     const float lse = lse_s;
     for (int i = tid; i < ns; i += kThreads) {
-        const unsigned long long key = sel[i];
+        const unsigned long long key = S.sel[i];
         int rank = 0;
-        for (int j = 0; j < ns; ++j) rank += sel[j] > key ? 1 : 0;
+        for (int j = 0; j < ns; ++j) rank += S.sel[j] > key ? 1 : 0;
         out_ids[static_cast<size_t>(row) * k + rank] = key_id(key);
         out_logp[static_cast<size_t>(row) * k + rank] = key_value(key) - lse;
     }
@@ -516,14 +538,14 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
 
 }  // namespace
 
-size_t merge_smem_bytes(int n_tiles, int d) { return merge_layout(n_tiles, d, nullptr, nullptr); }
+size_t merge_smem_bytes(int n_tiles, int d, int k) { return merge_layout(n_tiles, d, k, nullptr, nullptr); }
 
 cudaError_t launch_lmhead_merge(const Ctx& ctx, int dtype, Partials partials, int n_rows, int V, int d, int k,
                                 float inv_temp, const void* lm_head, const void* x, int32_t* out_ids,
                                 float* out_logp) {
     if (n_rows <= 0) return cudaSuccess;
     const int n_tiles = (V + kBlockV - 1) / kBlockV;
-    const size_t smem = merge_smem_bytes(n_tiles, d);
+    const size_t smem = merge_smem_bytes(n_tiles, d, k);
     if (dtype == TF_BF16) {
         auto kern = lmhead_merge_kernel<__nv_bfloat16>;
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));

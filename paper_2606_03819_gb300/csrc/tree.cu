@@ -96,6 +96,17 @@ struct TreeArgs {
     int32_t* dev_status;
 };
 
+// Index m of `tok` among the M <= 64 stage-1 candidates of depth `dep` (the M-ary rule of
+// Algorithm 1 Part 2: the node is expandable iff its token is one of them), or -1; two warp
+// ballots, so every lane of the warp must call it (active = false gives -1).
+__device__ __forceinline__ int mary_index(const int* topm, int dep, int M, int tok, int lane, bool active) {
+    const int* t = topm + (dep - 1) * M;
+    const bool h0 = active && lane < M && t[lane] == tok;
+    const bool h1 = active && lane + 32 < M && t[lane + 32] == tok;
+    const unsigned b0 = __ballot_sync(0xffffffffu, h0), b1 = __ballot_sync(0xffffffffu, h1);
+    return b0 ? __ffs(b0) - 1 : (b1 ? 32 + __ffs(b1) - 1 : -1);
+}
+
 __device__ __forceinline__ unsigned long long queue_key(float score, int depth, int parent) {
     return (static_cast<unsigned long long>(float_key(score)) << 32) |
            (static_cast<unsigned long long>(127 - depth) << 24) | static_cast<unsigned long long>(0xFFFFFF - parent);
@@ -294,15 +305,14 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
             const int node = count++;
             if (tok < 0 || tok >= a.V) flags |= TF_DEV_BAD_TOKEN;
             if (!isfinite(sc)) flags |= TF_DEV_NONFINITE;
-            // expandable? (depth cap; M-ary rule via one compare per lane)
+            // expandable? (depth cap; M-ary rule)
             int crow = -1;
             if (dep < a.gamma) {
                 if (a.mode == TF_MODE_MARGINAL) {
                     crow = dep;
                 } else {
-                    const bool hit = lane < a.M && topm[(dep - 1) * a.M + lane] == tok;
-                    const unsigned bal = __ballot_sync(kFull, hit);
-                    if (bal) crow = ar ? 1 + (dep - 1) * a.M + (__ffs(bal) - 1) : dep;
+                    const int m = mary_index(topm, dep, a.M, tok, lane, true);
+                    if (m >= 0) crow = ar ? 1 + (dep - 1) * a.M + m : dep;
                 }
             }
             const bool sibling = rank + 1 < list_len;
@@ -436,13 +446,12 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
             const size_t sat = static_cast<size_t>(row) * stride + rank + 1;
             const int sib_tok = sibling ? ids_base[sat] : 0;
             const float sib_lp = sibling ? lp_base[sat] : 0.0f;
-            // expandable? (depth cap; M-ary rule via one compare per lane)
+            // expandable? (depth cap; M-ary rule)
             const bool deep_ok = dep < a.gamma;
-            const bool hit = deep_ok && lane < a.M && t.topm[(dep - 1) * a.M + lane] == tok;
-            const unsigned bal = __ballot_sync(kFull, hit);
+            const int m = mary_index(t.topm, dep, a.M, tok, lane, deep_ok && a.mode != TF_MODE_MARGINAL);
             const int crow = !deep_ok ? -1
                              : a.mode == TF_MODE_MARGINAL ? dep
-                             : bal ? (ar ? 1 + (dep - 1) * a.M + (__ffs(bal) - 1) : dep) : -1;
+                             : m >= 0 ? (ar ? 1 + (dep - 1) * a.M + m : dep) : -1;
             if (tok < 0 || tok >= a.V) flags |= TF_DEV_BAD_TOKEN;
             if (!isfinite(sc)) flags |= TF_DEV_NONFINITE;
             const unsigned long long sib_key = sibling ? queue_key(psc + sib_lp, dep, par) : 0ull;

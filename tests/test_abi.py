@@ -68,7 +68,7 @@ def test_workspace_size_and_validation(lib):
         with pytest.raises(Bn.TreeFlashError) as e:
             Bn.tf_workspace_size(_dims(**kw))
         assert e.value.status == Bn.TF_ERR_INVALID_ARG, kw
-    for kw in (dict(M=33), dict(K2=65), dict(B=2000), dict(gamma=65), dict(dtype="bf16", d=100),
+    for kw in (dict(M=65), dict(K2=513, V=4096), dict(B=2000), dict(gamma=65), dict(dtype="bf16", d=100),
                dict(dtype="bf16", I=100)):
         with pytest.raises(Bn.TreeFlashError) as e:
             Bn.tf_workspace_size(_dims(**kw))

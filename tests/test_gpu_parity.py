@@ -234,6 +234,57 @@ def test_full_size_wide_sampled_sequence(name):
     check(cfg, orc_seqs=[3], emulate_also=False)
 
 
+# ------------------------------------------------------------------ large budgets and branching
+# (Fig. 5: budgets up to 512; Fig. 6: M up to 64): K2 = B keeps the per-row lists exact, the
+# merge returns up to 512 entries, the builder tests membership among up to 64 candidates and
+# keeps its queue in shared memory beyond B = 127.
+
+
+def test_fp32_large_budget_and_branching():
+    cfg = synth.get_config("tiny_peaked", M=64, K2=256, B=256)
+    _, reps = check(cfg)
+    print(reps)
+
+
+def test_bf16_large_budget():
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", d=256, V=4096, M=48, K2=512, B=512)
+    _, reps = check(cfg)
+    print(reps)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_lmhead_top512_equals_topk_of_exact_logits(dtype):
+    # the merge's exact top-k at k = 512 against torch.topk of the fp64 logits (ties have
+    # probability zero for these continuous inputs)
+    from paper_2606_03819_gb300 import binding as Bn
+    V, d, rows, k = 8192, 256, 20, 512
+    dims = Bn.Dims(batch=rows, d=d, V=V, I=64, gamma=1, M=4, K2=k, B=k, dtype=dtype, mode="marginal")
+    g = torch.Generator().manual_seed(11)
+    dt = dims.torch_dtype
+    W = (torch.randn(V, d, generator=g) * 0.02).to(dt)
+    x = (torch.randn(rows, d, generator=g) * 4.0).to(dt)
+    ws = Bn.alloc_workspace(dims)
+    ids = torch.empty(rows, k, dtype=torch.int32, device="cuda")
+    lp = torch.empty(rows, k, dtype=torch.float32, device="cuda")
+    Bn.tf_status_reset(ws)
+    Bn.tf_lmhead_partials(dims, W.cuda(), x.cuda(), rows, ws)
+    Bn.tf_lmhead_merge(dims, W.cuda(), x.cuda(), rows, k, ids, lp, ws)
+    assert not (Bn.tf_status_read(ws) & ~16)
+    z = x.double() @ W.double().T
+    ref = torch.topk(z, k, dim=1)
+    lse = torch.logsumexp(z, dim=1, keepdim=True)
+    got = ids.cpu().long()
+    # the id sets must agree exactly wherever the k-th and (k+1)-th logits are apart by more
+    # than the arithmetic's error (bf16 inputs, fp32 accumulation)
+    tol = 1e-4 if dtype == "f32" else 2e-3
+    zs = torch.sort(z, dim=1, descending=True).values
+    for r in range(rows):
+        if zs[r, k - 1] - zs[r, k] > tol:
+            assert set(got[r].tolist()) == set(ref.indices[r].tolist()), f"row {r}"
+        np.testing.assert_allclose(lp[r].cpu().double().numpy(), (z[r, got[r]] - lse[r]).numpy(), atol=tol)
+    assert (lp[:, :-1] >= lp[:, 1:]).all()
+
+
 def test_kernel_launch_counter_counts_each_kernel():
     # tf_stage1_marginals is one LM-head pass and one merge: two kernels per call
     from paper_2606_03819_gb300 import binding as Bn
