@@ -113,6 +113,7 @@ __device__ __forceinline__ unsigned long long queue_key(float score, int depth, 
 }
 
 constexpr int kTreeThreads = 256;
+constexpr int kMaskRows = 128;    // mask rows per CTA
 
 // Shared-memory bytes of build_tree_kernel: queue, node arrays, stage-1 top-M, and (when they
 // fit) the sequence's child lists.
@@ -120,10 +121,26 @@ __host__ __device__ inline size_t tree_smem_fixed(int B, int gamma, int M) {
     return static_cast<size_t>(B + 2) * (8 + 4 * 4) + static_cast<size_t>(B + 1) * 4 * 4 +
            static_cast<size_t>(gamma) * M * 4 + 16;
 }
-__host__ __device__ inline size_t tree_smem_lists(int mode, int gamma, int R, int K1, int K2) {
-    return mode == TF_MODE_AR ? static_cast<size_t>(R) * K2 * 8 : static_cast<size_t>(gamma) * K1 * 8;
-}
+// Bytes of the staged list prefixes: the first sw entries of each of the rows child lists.
+__host__ __device__ inline size_t tree_smem_lists(int rows, int sw) { return static_cast<size_t>(rows) * sw * 8; }
 constexpr size_t kTreeSmemLimit = 200 * 1024;
+
+// The child lists of one sequence: the first sw entries of every row staged in shared memory,
+// the rest read from global memory. A list's entry of rank r is reached only after r pops of
+// that list, so sw = min(list length, B + 1) already covers every entry a tree can use.
+struct ListView {
+    const int32_t* s_ids;   // [rows][sw]
+    const float* s_lp;
+    const int32_t* g_ids;   // [rows][stride]
+    const float* g_lp;
+    int sw, stride;
+    __device__ __forceinline__ int tok(int row, int rank) const {
+        return rank < sw ? s_ids[row * sw + rank] : g_ids[static_cast<size_t>(row) * stride + rank];
+    }
+    __device__ __forceinline__ float lp(int row, int rank) const {
+        return rank < sw ? s_lp[row * sw + rank] : g_lp[static_cast<size_t>(row) * stride + rank];
+    }
+};
 
 // Shared memory of both builders: queue arrays (used by the general builder only), output nodes,
 // stage-1 top-M and the staged child lists.
@@ -134,7 +151,7 @@ struct TreeSmem {
     int *o_tok, *o_par, *o_dep;
     float* o_score;
     int* topm;        // [gamma, M]
-    uint8_t* lists;   // ids [rows][stride] int32, then log-probs [rows][stride] float
+    uint8_t* lists;   // staged prefixes: ids [rows][sw] int32, then log-probs [rows][sw] float
 };
 __device__ __forceinline__ TreeSmem tree_smem(uint8_t* base, const TreeArgs& a) {
     TreeSmem t;
@@ -154,37 +171,36 @@ __device__ __forceinline__ TreeSmem tree_smem(uint8_t* base, const TreeArgs& a) 
     return t;
 }
 
-// Stage sequence s's stage-1 top-M and, when stage_lists, its child lists (every pop then
-// touches shared memory only); returns where the lists are read from.
-__device__ __forceinline__ void stage_sequence(const TreeArgs& a, int s, const TreeSmem& t, int stage_lists,
-                                               const int32_t** ids_base, const float** lp_base) {
+// Stage sequence s's stage-1 top-M and the first sw entries of each of its child lists.
+__device__ __forceinline__ ListView stage_sequence(const TreeArgs& a, int s, const TreeSmem& t, int sw) {
     const int tid = threadIdx.x;
     const bool ar = a.mode == TF_MODE_AR;
     const int n_rows_l = ar ? a.R : a.gamma;
     const int stride = ar ? a.K2 : a.K1;
-    const int32_t* g_ids = ar ? a.child_ids + static_cast<size_t>(s) * a.R * a.K2
-                              : a.top_ids + static_cast<size_t>(s) * a.gamma * a.K1;
-    const float* g_lp = ar ? a.child_logp + static_cast<size_t>(s) * a.R * a.K2
-                           : a.top_logp + static_cast<size_t>(s) * a.gamma * a.K1;
-    *ids_base = g_ids;
-    *lp_base = g_lp;
+    ListView v;
+    v.g_ids = ar ? a.child_ids + static_cast<size_t>(s) * a.R * a.K2 : a.top_ids + static_cast<size_t>(s) * a.gamma * a.K1;
+    v.g_lp = ar ? a.child_logp + static_cast<size_t>(s) * a.R * a.K2 : a.top_logp + static_cast<size_t>(s) * a.gamma * a.K1;
+    v.stride = stride;
+    v.sw = sw;
     for (int i = tid; i < a.gamma * a.M; i += kTreeThreads)
         t.topm[i] = a.top_ids[(static_cast<size_t>(s) * a.gamma + i / a.M) * a.K1 + i % a.M];
-    if (!stage_lists) return;
-    const int n = n_rows_l * stride;
+    const int n = n_rows_l * sw;
     int32_t* si = reinterpret_cast<int32_t*>(t.lists);
     float* sl = reinterpret_cast<float*>(si + n);
-    const bool vec = ((reinterpret_cast<uintptr_t>(g_ids) | reinterpret_cast<uintptr_t>(g_lp) |
+    v.s_ids = si;
+    v.s_lp = sl;
+    const bool vec = sw == stride &&
+                     ((reinterpret_cast<uintptr_t>(v.g_ids) | reinterpret_cast<uintptr_t>(v.g_lp) |
                        reinterpret_cast<uintptr_t>(si) | reinterpret_cast<uintptr_t>(sl)) & 15) == 0 &&
                      (n & 3) == 0;
+    constexpr int T = kTreeThreads;
     if (vec) {
-        // 16-byte copies, sixteen per thread in flight before the first store
-        const int4* gi = reinterpret_cast<const int4*>(g_ids);
-        const float4* gl = reinterpret_cast<const float4*>(g_lp);
+        // whole lists: 16-byte copies, sixteen per thread in flight before the first store
+        const int4* gi = reinterpret_cast<const int4*>(v.g_ids);
+        const float4* gl = reinterpret_cast<const float4*>(v.g_lp);
         int4* di = reinterpret_cast<int4*>(si);
         float4* dl = reinterpret_cast<float4*>(sl);
         const int n4 = n >> 2;
-        constexpr int T = kTreeThreads;
         for (int base = tid; base < n4; base += 8 * T) {
             int4 va[8];
             float4 vb[8];
@@ -202,16 +218,30 @@ __device__ __forceinline__ void stage_sequence(const TreeArgs& a, int s, const T
                 }
         }
     } else {
-#pragma unroll 8
-        for (int i = tid; i < n; i += kTreeThreads) {
-            const int32_t v = g_ids[i];
-            const float w = g_lp[i];
-            si[i] = v;
-            sl[i] = w;
+        // prefixes of sw entries: element copies, eight per thread in flight
+        for (int base = tid; base < n; base += 8 * T) {
+            int32_t va[8];
+            float vb[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int i = base + j * T;
+                if (i < n) {
+                    const size_t g = static_cast<size_t>(i / sw) * stride + i % sw;
+                    va[j] = v.g_ids[g];
+                    vb[j] = v.g_lp[g];
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int i = base + j * T;
+                if (i < n) {
+                    si[i] = va[j];
+                    sl[i] = vb[j];
+                }
+            }
         }
     }
-    *ids_base = si;
-    *lp_base = sl;
+    return v;
 }
 
 // Nodes from shared memory to the outputs.
@@ -227,7 +257,7 @@ __device__ __forceinline__ void write_nodes(const TreeArgs& a, int s, const Tree
 }
 
 // General builder (any B): the queue in shared memory.
-__global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, int stage_lists) {
+__global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, int sw) {
     pdl_trigger();
     pdl_wait();
     extern __shared__ __align__(16) uint8_t smem_raw[];
@@ -246,10 +276,7 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
     const int s = blockIdx.x;
     const int tid = threadIdx.x;
     const bool ar = a.mode == TF_MODE_AR;
-    const int stride = ar ? a.K2 : a.K1;
-    const int32_t* ids_base;
-    const float* lp_base;
-    stage_sequence(a, s, t, stage_lists, &ids_base, &lp_base);
+    const ListView lv = stage_sequence(a, s, t, sw);
     __syncthreads();
 
     if (tid < 32) {
@@ -259,18 +286,16 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
         const int root = a.root_tok[s];
         if (root < 0 || root >= a.V) flags |= TF_DEV_BAD_TOKEN;
         const int list_len = a.K2;
-        auto ids_of = [&](int row) -> const int32_t* { return ids_base + static_cast<size_t>(row) * stride; };
-        auto lp_of = [&](int row) -> const float* { return lp_base + static_cast<size_t>(row) * stride; };
         if (lane == 0) {
             o_tok[0] = root;
             o_par[0] = -1;
             o_dep[0] = 0;
             o_score[0] = 0.0f;
-            qkey[0] = queue_key(lp_of(0)[0], 1, 0);
+            qkey[0] = queue_key(lv.lp(0, 0), 1, 0);
             qps[0] = 0.0f;
             qrow[0] = 0;
             qrank[0] = 0;
-            qtok[0] = ids_of(0)[0];
+            qtok[0] = lv.tok(0, 0);
         }
         int n_e = 1;
         int count = 1;
@@ -324,8 +349,8 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
                 o_score[node] = sc;
                 if (sibling) {                   // next sibling of the popped entry
                     qrank[best] = rank + 1;
-                    qtok[best] = ids_of(row)[rank + 1];
-                    qkey[best] = queue_key(psc + lp_of(row)[rank + 1], dep, par);
+                    qtok[best] = lv.tok(row, rank + 1);
+                    qkey[best] = queue_key(psc + lv.lp(row, rank + 1), dep, par);
                 } else if (best != last) {       // list exhausted: move the last entry here
                     qkey[best] = qkey[last];
                     qps[best] = qps[last];
@@ -339,11 +364,11 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
             if (crow >= 0) {
                 fresh = n_e;
                 if (lane == 0) {
-                    qkey[n_e] = queue_key(sc + lp_of(crow)[0], dep + 1, node);
+                    qkey[n_e] = queue_key(sc + lv.lp(crow, 0), dep + 1, node);
                     qps[n_e] = sc;
                     qrow[n_e] = crow;
                     qrank[n_e] = 0;
-                    qtok[n_e] = ids_of(crow)[0];
+                    qtok[n_e] = lv.tok(crow, 0);
                 }
                 ++n_e;
             }
@@ -368,8 +393,8 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
 // register j / 32). Slots are appended in pop order and an exhausted list leaves an empty slot
 // (key 0, below every real key), so no entry ever moves. Pops, tie rules and results are those
 // of build_tree_kernel.
-template <int S>
-__global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a, int stage_lists) {
+template <int S, bool FULL>
+__global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a, int sw) {
     pdl_trigger();
     pdl_wait();
     extern __shared__ __align__(16) uint8_t smem_raw[];
@@ -377,10 +402,10 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
     const int n_out = a.B + 1;
     const int s = blockIdx.x;
     const bool ar = a.mode == TF_MODE_AR;
-    const int stride = ar ? a.K2 : a.K1;
-    const int32_t* ids_base;
-    const float* lp_base;
-    stage_sequence(a, s, t, stage_lists, &ids_base, &lp_base);
+    const ListView lv = stage_sequence(a, s, t, sw);
+    // FULL: every rank a pop can reach is staged, so entries are read from shared memory only
+    auto ltok = [&](int row, int rank) { return FULL ? lv.s_ids[row * sw + rank] : lv.tok(row, rank); };
+    auto llp = [&](int row, int rank) { return FULL ? lv.s_lp[row * sw + rank] : lv.lp(row, rank); };
     __syncthreads();
     if (threadIdx.x < 32) {
         const int lane = threadIdx.x;
@@ -399,8 +424,8 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
             spsc[j] = 0.0f;
         }
         if (lane == 0) {
-            key[0] = queue_key(lp_base[0], 1, 0);
-            stok[0] = ids_base[0];
+            key[0] = queue_key(llp(0, 0), 1, 0);
+            stok[0] = ltok(0, 0);
             t.o_tok[0] = root;
             t.o_par[0] = -1;
             t.o_dep[0] = 0;
@@ -443,9 +468,8 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
             // next sibling of the popped entry (the same shared-memory words for every lane),
             // read before the expandability test so that both latencies overlap
             const bool sibling = rank + 1 < list_len;
-            const size_t sat = static_cast<size_t>(row) * stride + rank + 1;
-            const int sib_tok = sibling ? ids_base[sat] : 0;
-            const float sib_lp = sibling ? lp_base[sat] : 0.0f;
+            const int sib_tok = sibling ? ltok(row, rank + 1) : 0;
+            const float sib_lp = sibling ? llp(row, rank + 1) : 0.0f;
             // expandable? (depth cap; M-ary rule)
             const bool deep_ok = dep < a.gamma;
             const int m = mary_index(t.topm, dep, a.M, tok, lane, deep_ok && a.mode != TF_MODE_MARGINAL);
@@ -466,9 +490,8 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
                 }
             }
             if (crow >= 0) {
-                const size_t at = static_cast<size_t>(crow) * stride;
-                const int ctok = ids_base[at];
-                const unsigned long long ckey = queue_key(sc + lp_base[at], dep + 1, node);
+                const int ctok = ltok(crow, 0);
+                const unsigned long long ckey = queue_key(sc + llp(crow, 0), dep + 1, node);
                 const bool mine = lane == (n_e & 31);
 #pragma unroll
                 for (int j = 0; j < S; ++j) {
@@ -517,10 +540,11 @@ __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __
     pdl_wait();
     extern __shared__ uint32_t sm[];
     const int W = (n + 31) / 32;
+    const int s = blockIdx.x;
+    const int r0 = blockIdx.y * kMaskRows, r1 = min(n, r0 + kMaskRows);   // this CTA's rows
     int* par = reinterpret_cast<int*>(sm);
     int* dep = par + n;
-    uint32_t* anc = reinterpret_cast<uint32_t*>(dep + n);   // [n][W] ancestor-or-self bits
-    const int s = blockIdx.x;
+    uint32_t* anc = reinterpret_cast<uint32_t*>(dep + n);   // [kMaskRows][W] ancestor-or-self bits
     const int32_t* P = node_parent + static_cast<size_t>(s) * n;
     const int32_t* D = node_depth + static_cast<size_t>(s) * n;
     for (int i = threadIdx.x; i < n; i += blockDim.x) {
@@ -528,8 +552,8 @@ __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __
         dep[i] = D[i];
     }
     __syncthreads();
-    for (int i = threadIdx.x; i < n; i += blockDim.x) {
-        uint32_t* row = anc + static_cast<size_t>(i) * W;
+    for (int i = r0 + threadIdx.x; i < r1; i += blockDim.x) {
+        uint32_t* row = anc + static_cast<size_t>(i - r0) * W;
         for (int w = 0; w < W; ++w) row[w] = 0u;
         bool ok = true;
         int j = i;
@@ -549,9 +573,11 @@ __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __
     }
     __syncthreads();
     uint8_t* out = mask + static_cast<size_t>(s) * n * n;
-    for (int idx = threadIdx.x; idx < n * n; idx += blockDim.x) {
-        const int i = idx / n, j = idx - (idx / n) * n;
-        out[idx] = static_cast<uint8_t>((anc[i * W + (j >> 5)] >> (j & 31)) & 1u);
+    const int count = (r1 - r0) * n;
+    for (int idx = threadIdx.x; idx < count; idx += blockDim.x) {
+        const int i = idx / n, jcol = idx - (idx / n) * n;
+        out[static_cast<size_t>(r0 + i) * n + jcol] =
+            static_cast<uint8_t>((anc[i * W + (jcol >> 5)] >> (jcol & 31)) & 1u);
     }
 }
 
@@ -767,18 +793,28 @@ cudaError_t launch_build_tree(const Ctx& ctx, int b, int gamma, int M, int K1, i
     TreeArgs a{gamma, M, K1, K2, B, V, mode, R, root_tok, top_ids, top_logp, child_ids, child_logp,
                node_tok, node_parent, node_depth, node_score, dev_status};
     const size_t fixed = tree_smem_fixed(B, gamma, M);
-    const size_t lists = tree_smem_lists(mode, gamma, R, K1, K2);
-    const int stage = fixed + lists <= kTreeSmemLimit ? 1 : 0;
-    const size_t smem = fixed + (stage ? lists : 0);
+    const int rows_l = mode == TF_MODE_AR ? R : gamma;
+    const int stride = mode == TF_MODE_AR ? K2 : K1;
+    // stage the entries a tree can reach (rank <= B) when they fit, else a prefix that does
+    const int sw_full = stride < B + 1 ? stride : B + 1;
+    int sw = sw_full;
+    if (fixed + tree_smem_lists(rows_l, sw) > kTreeSmemLimit) {
+        const size_t room = kTreeSmemLimit > fixed ? kTreeSmemLimit - fixed : 0;
+        sw = static_cast<int>(room / (static_cast<size_t>(rows_l) * 8)) & ~3;
+        if (sw > sw_full) sw = sw_full;
+    }
+    const size_t smem = fixed + tree_smem_lists(rows_l, sw);
     // the register-queue builder whenever B + 1 slots fit in four registers per lane
-    void (*kern)(TreeArgs, int) = B + 1 <= 32 ? build_tree_reg_kernel<1>
-                                  : B + 1 <= 64 ? build_tree_reg_kernel<2>
-                                  : B + 1 <= 96 ? build_tree_reg_kernel<3>
-                                  : B + 1 <= 128 ? build_tree_reg_kernel<4>
-                                                 : build_tree_kernel;
+    const bool full = sw == sw_full;
+    void (*kern)(TreeArgs, int) =
+        B + 1 <= 32    ? (full ? build_tree_reg_kernel<1, true> : build_tree_reg_kernel<1, false>)
+        : B + 1 <= 64  ? (full ? build_tree_reg_kernel<2, true> : build_tree_reg_kernel<2, false>)
+        : B + 1 <= 96  ? (full ? build_tree_reg_kernel<3, true> : build_tree_reg_kernel<3, false>)
+        : B + 1 <= 128 ? (full ? build_tree_reg_kernel<4, true> : build_tree_reg_kernel<4, false>)
+                       : build_tree_kernel;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    e = launch_pdl(kern, dim3(b), dim3(kTreeThreads), smem, ctx.stream, a, stage);
+    e = launch_pdl(kern, dim3(b), dim3(kTreeThreads), smem, ctx.stream, a, sw);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -786,12 +822,12 @@ cudaError_t launch_tree_mask(const Ctx& ctx, int b, int B, const int32_t* node_p
                              const int32_t* root_pos, uint8_t* mask, int32_t* pos_ids) {
     const int n = B + 1;
     const int W = (n + 31) / 32;
-    const size_t smem = static_cast<size_t>(2 * n + n * W) * 4;
+    const size_t smem = static_cast<size_t>(2 * n + kMaskRows * W) * 4;
     cudaError_t e = cudaFuncSetAttribute(tree_mask_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    e = launch_pdl(tree_mask_kernel, dim3(b), dim3(256), smem, ctx.stream, n, node_parent, node_depth, root_pos, mask,
-                   pos_ids);
+    e = launch_pdl(tree_mask_kernel, dim3(b, (n + kMaskRows - 1) / kMaskRows), dim3(256), smem, ctx.stream, n,
+                   node_parent, node_depth, root_pos, mask, pos_ids);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 

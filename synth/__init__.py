@@ -89,6 +89,9 @@ CONFIGS = {
                           K2=64, B=64, h_entropy=(1.0, 1.0)),
     "wide_flat": Config("wide_flat", batch=8, d=5120, V=151936, I=5120, gamma=16, M=16,
                         K2=64, B=64, h_entropy=(5.0, 5.0)),
+    # large draft budget (Fig. 5) with exact per-row lists (K2 = B), and wide branching (Fig. 6)
+    "q8_b512": Config("q8_b512", batch=1, M=16, K2=512, B=512, **_Q8),
+    "q8_m64": Config("q8_m64", batch=1, M=64, K2=64, B=64, **_Q8),
     # the q8_b64 step with the vocabulary cut to 32768 (W_lm 268 MB, still twice the L2):
     # small enough for multi-pass profiler captures
     "prof_v32k": Config("prof_v32k", batch=1, M=16, K2=64, B=64, **dict(_Q8, V=32768)),

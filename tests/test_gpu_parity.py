@@ -223,6 +223,14 @@ def test_full_size_qwen3_8b_shape(name):
     assert gpu["node_depth"][0].max() >= 3
 
 
+@pytest.mark.parametrize("name", ["q8_b512", "q8_m64"])
+def test_full_size_large_budget_and_branching(name):
+    # Fig. 5 / Fig. 6 regimes at the full Qwen3-8B shape: B = K2 = 512 (exact lists), M = 64
+    # (961 stage-2 rows)
+    _, reps = check(synth.get_config(name), inp=_inputs(name))
+    print(name, reps)
+
+
 def test_full_size_batch32_sampled_sequences():
     cfg = synth.get_config("batch32")
     check(cfg, orc_seqs=[0, 17, 31], emulate_also=False)
@@ -248,6 +256,14 @@ def test_fp32_large_budget_and_branching():
 
 def test_bf16_large_budget():
     cfg = synth.get_config("tiny_peaked", dtype="bf16", d=256, V=4096, M=48, K2=512, B=512)
+    _, reps = check(cfg)
+    print(reps)
+
+
+def test_fp32_budget_near_the_limit_with_truncated_lists():
+    # B = 1000 (the shared-memory queue at 32 slots per lane) with K2 = 512 < B: the oracle
+    # truncates every list to 512 entries too
+    cfg = synth.get_config("tiny_peaked", V=4096, M=32, K2=512, B=1000)
     _, reps = check(cfg)
     print(reps)
 
