@@ -50,9 +50,8 @@ struct EpiParams {
     int ld_out;
     const __nv_bfloat16* hidden; // DOWN: residual rows, [b * gamma, ld_out]
     int R, M, gamma;
-    float* partial;              // PARTIAL: fp32 [k_splits][n_rows][ld_partial], accumulator nb at
-    int ld_partial;              //          columns nb * n_total + n
-    size_t partial_split_stride; // elements between consecutive k-splits
+    float* partial;              // PARTIAL: fp32 sums [k_splits][n_cols / 32][n_rows][32] (chunk-major),
+    int n_cols;                  //          accumulator nb of N tile nt at columns nb * n_total + nt * BN
     int n_total;                 // N of the whole GEMM (n_ntiles * BN)
     int reset_status;            // LMHEAD: zero *status first (the first kernel of a stage-1 call)
 };
@@ -272,7 +271,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     } else if (warp == 1) {
         // ------------------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kBM, BN);
+            // the NB weight tiles of a stage are adjacent in shared memory with the same swizzle, so
+            // one MMA of N = NB * BN covers them: A is read from shared memory once per k-step
+            constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kBM, NB * BN);
             int stage = 0;
             uint32_t phase = 0;
             uint32_t use[2] = {0u, 0u};
@@ -294,15 +295,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                     const uint32_t b0 = a0 + MT * C::kABytes;
 #pragma unroll
                     for (int kk = 0; kk < kBK / 16; ++kk) {
+                        const uint64_t bd = ptx::sw128_kmajor_desc(b0 + kk * 32);
 #pragma unroll
                         for (int j = 0; j < MT; ++j) {
                             const uint64_t ad = ptx::sw128_kmajor_desc(a0 + j * C::kABytes + kk * 32);
-#pragma unroll
-                            for (int nb = 0; nb < NB; ++nb) {
-                                const uint64_t bd = ptx::sw128_kmajor_desc(b0 + nb * C::kBBytes + kk * 32);
-                                ptx::mma_bf16(tmem_base + 256u * (g0 + j) + nb * BN, ad, bd, kIdesc,
-                                              (kb | kk) != 0 ? 1u : 0u);
-                            }
+                            ptx::mma_bf16(tmem_base + 256u * (g0 + j), ad, bd, kIdesc, (kb | kk) != 0 ? 1u : 0u);
                         }
                     }
                     // frees the stage (in every CTA of the cluster) once these MMAs finish
@@ -388,7 +385,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 ptx::tc_fence_before();
                 ptx::mbar_arrive(&tempty[g]);
             } else if constexpr (EPI == EPI_PARTIAL) {
-                float* base = ep.partial + w.kx * ep.partial_split_stride + static_cast<size_t>(row) * ep.ld_partial;
+                // chunk-major: a lane's 32 columns are 128 contiguous bytes and the warp's 32 rows
+                // one contiguous 4 KB block
+                float* split = ep.partial + static_cast<size_t>(w.kx) * ep.n_cols * n_rows;
 #pragma unroll 1
                 for (int nb = 0; nb < NB; ++nb) {
 #pragma unroll 1
@@ -396,7 +395,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                         uint32_t ra[32];
                         ptx::tmem_ld_32cols(tb + nb * BN + c, ra);
                         if (row < n_rows) {
-                            float4* dst = reinterpret_cast<float4*>(base + nb * ep.n_total + nt * BN + c);
+                            const int col = nb * ep.n_total + nt * BN + c;
+                            float4* dst = reinterpret_cast<float4*>(
+                                split + (static_cast<size_t>(col >> 5) * n_rows + row) * 32);
 #pragma unroll
                             for (int j = 0; j < 8; ++j)
                                 dst[j] = make_float4(__uint_as_float(ra[4 * j]), __uint_as_float(ra[4 * j + 1]),
@@ -464,6 +465,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         }
     }
 
+    // the producer and MMA lanes rejoin their warps first: the CTA-wide barrier below must wait
+    // for every thread, not only for each warp's first arrivals
+    __syncwarp();
     ptx::tc_fence_before();
     __syncthreads();
     // no CTA of the cluster may still write into this CTA's shared memory or barriers
@@ -611,8 +615,7 @@ cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, const void* w_gate, 
     ep.out = static_cast<__nv_bfloat16*>(A);
     ep.ld_out = I;
     ep.partial = partial;
-    ep.ld_partial = 2 * I;
-    ep.partial_split_stride = static_cast<size_t>(n_rows) * 2 * I;
+    ep.n_cols = 2 * I;
     ep.n_total = I;
     if (ks1 == 1) {
         if (bn_gu == BN)
@@ -644,8 +647,7 @@ cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, const void* w_gate, 
     ed.M = M;
     ed.gamma = gamma;
     ed.partial = partial;
-    ed.ld_partial = d;
-    ed.partial_split_stride = static_cast<size_t>(n_rows) * d;
+    ed.n_cols = d;
     ed.n_total = d;
     if (ks2 == 1) {
         if (bn_d == BN)
