@@ -40,7 +40,9 @@ constexpr int kEpiWarps = 16;  // two groups (one per TMEM slot) of eight warps
 constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
-enum { EPI_LMHEAD = 0, EPI_GATEUP = 1, EPI_DOWN = 2, EPI_PARTIAL = 3 };
+// EPI_CGATEUP / EPI_CDOWN: the GATEUP / DOWN results from split-K over the CTAs of a cluster, the
+// partial sums added in shared memory across the cluster instead of through global memory.
+enum { EPI_LMHEAD = 0, EPI_GATEUP = 1, EPI_DOWN = 2, EPI_PARTIAL = 3, EPI_CGATEUP = 4, EPI_CDOWN = 5 };
 
 struct EpiParams {
     Partials partials;           // LMHEAD: per (row, vocabulary block) summaries
@@ -146,7 +148,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                const __grid_constant__ CUtensorMap tmap_w1, int n_rows, int K, int n_ntiles,
                int n_mgroups, int k_splits, int w_stream_once, EpiParams ep, int* status) {
     using C = TileCfg<MT, NB, BN, STAGES>;
-    static_assert(CL == 1 || (CL == 2 && NB == 1), "clusters of two share one weight operand");
+    // Two kinds of cluster: kMulticast, two CTAs on two M-tiles sharing each weight tile by TMA
+    // multicast; kSplitK, CL CTAs on the CL K-ranges of one output tile (one tile per cluster),
+    // whose accumulators are summed through distributed shared memory.
+    constexpr bool kSplitK = EPI == EPI_CGATEUP || EPI == EPI_CDOWN;
+    constexpr bool kMulticast = CL > 1 && !kSplitK;
+    static_assert(CL == 1 || kSplitK || (CL == 2 && NB == 1), "clusters of two share one weight operand");
+    static_assert(!kSplitK || (CL == 4 && MT == 2 && BN == 128), "cluster split-K: 4 K-ranges of a 256 x 128 tile");
     constexpr uint16_t kClusterMask = static_cast<uint16_t>((1u << CL) - 1u);
     pdl_trigger();
     extern __shared__ uint8_t smem_raw[];
@@ -162,18 +170,24 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int n_units = n_ntiles * n_mgroups * k_splits;
-    // Units are dealt to clusters; CTA `crank` of a cluster takes M-tile group member crank of
-    // every unit (with CL = 1 a cluster is one CTA).
+    // Units are dealt to clusters. Multicast: CTA `crank` of a cluster takes M-tile group member
+    // crank of every unit. Split-K: a unit is an output tile and CTA crank takes K-range crank.
+    // With CL = 1 a cluster is one CTA.
+    const int n_units = kSplitK ? n_ntiles * n_mgroups : n_ntiles * n_mgroups * k_splits;
     const int crank = CL > 1 ? static_cast<int>(ptx::cluster_ctarank()) : 0;
+    const int m_cl = kMulticast ? CL : 1, m_rank = kMulticast ? crank : 0;   // M-tiles of a cluster, this CTA's
     const int cid = CL > 1 ? static_cast<int>(ptx::cluster_id_x()) : static_cast<int>(blockIdx.x);
     const int ncl = CL > 1 ? static_cast<int>(ptx::cluster_count_x()) : static_cast<int>(gridDim.x);
     const int nk = K / kBK / k_splits;      // K-steps per unit (K % (64 * k_splits) == 0)
+    auto unit_of = [&](int u) {
+        if constexpr (kSplitK) return Unit{u / n_mgroups, u % n_mgroups, crank};
+        return decode_unit(u, n_mgroups, k_splits);
+    };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             ptx::mbar_init(&full[s], 1);
-            ptx::mbar_init(&empty[s], CL);   // freed once every CTA of the cluster has consumed it
+            ptx::mbar_init(&empty[s], m_cl);   // freed once every CTA sharing the stage has consumed it
         }
         for (int g = 0; g < 2; ++g) {
             ptx::mbar_init(&tfull[g], 1);
@@ -208,7 +222,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             // Weight tiles of one stage. In a cluster each CTA fetches its share of the rows and
             // multicasts it to every CTA of the cluster (tmap_w0's box is BN / CL rows high).
             auto load_w = [&](uint8_t* sp, uint64_t* bar, int kb, int nt) {
-                if constexpr (CL > 1) {
+                if constexpr (kMulticast) {
                     ptx::tma_load_2d_multicast(sp + MT * C::kABytes + crank * (C::kBBytes / CL), &tmap_w0, bar,
                                                kb * kBK, nt * BN + crank * (BN / CL), kClusterMask, pol_w);
                 } else {
@@ -221,7 +235,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             // requested before waiting for the previous kernel (which may be writing X).
             int pre = 0;
             if (cid < n_units) {
-                const Unit w = decode_unit(cid, n_mgroups, k_splits);
+                const Unit w = unit_of(cid);
                 pre = nk < STAGES ? nk : STAGES;
                 for (int i = 0; i < pre; ++i) {
                     ptx::mbar_arrive_expect_tx(&full[i], C::kStageBytes);
@@ -236,8 +250,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             bool ok = true;
             int it = 0;                               // k-steps issued so far by this CTA
             for (int u = cid; u < n_units && ok; u += ncl) {
-                const Unit w = decode_unit(u, n_mgroups, k_splits);
-                const int nt = w.nt, mt0 = (w.mg * CL + crank) * MT;
+                const Unit w = unit_of(u);
+                const int nt = w.nt, mt0 = (w.mg * m_cl + m_rank) * MT;
                 for (int kb = w.kx * nk; kb < (w.kx + 1) * nk; ++kb, ++it) {
                     if (!ptx::mbar_wait(&empty[stage], phase ^ 1u, abort_flag, kWaitLimitNs)) {
                         ok = false;
@@ -303,7 +317,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                         }
                     }
                     // frees the stage (in every CTA of the cluster) once these MMAs finish
-                    if constexpr (CL > 1)
+                    if constexpr (kMulticast)
                         ptx::mma_commit_multicast(&empty[stage], kClusterMask);
                     else
                         ptx::mma_commit(&empty[stage]);
@@ -343,12 +357,14 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             }
             ++use;
             ptx::tc_fence_after();
-            const Unit w = decode_unit(u, n_mgroups, k_splits);
+            const Unit w = unit_of(u);
             const int nt = w.nt;
-            const int row = ((w.mg * CL + crank) * MT + (MT == 2 ? g : 0)) * kBM + q * 32 + lane;
+            const int row = ((w.mg * m_cl + m_rank) * MT + (MT == 2 ? g : 0)) * kBM + q * 32 + lane;
             const uint32_t tb = tmem_base + 256u * g + (static_cast<uint32_t>(q * 32) << 16);
 
-            if constexpr (EPI == EPI_LMHEAD) {
+            if constexpr (kSplitK) {
+                // the accumulators are summed across the cluster below, once every CTA has them
+            } else if constexpr (EPI == EPI_LMHEAD) {
                 static_assert(BN == kBlockV, "one LM-head N tile is one vocabulary block");
                 // this warp's half of the block: chunks [half * 4, half * 4 + 4)
                 constexpr int kHalf = kChunks / 2;
@@ -465,6 +481,111 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         }
     }
 
+    if constexpr (kSplitK) {
+        // ------------------------------------------------------------------ split-K sum
+        // The tile's output columns are owned in CL blocks of BN / CL: CTA o adds the CL partial
+        // sums of block o in K-range order (the order of the split-K reduction kernels) and
+        // applies the epilogue. Every CTA first writes the blocks it does not own into their
+        // owners' stage rings (idle once all MMAs of the cluster are done), row r's 16-byte units
+        // permuted by r % 8 so that the 32 rows of a warp spread over the banks.
+        constexpr int kOwn = BN / CL;                    // output columns per owner
+        constexpr int kRowF4 = NB * kOwn / 4;            // 16-byte units per row of a block
+        constexpr int kSlotBytes = MT * kBM * kRowF4 * 16;
+        static_assert(kOwn == 32, "one TMEM load per block and accumulator");
+        static_assert((CL - 1) * kSlotBytes <= STAGES * C::kStageBytes, "the received blocks fit the ring");
+        const bool has_unit = cid < n_units;
+        const int e = warp - 2;
+        const int g = e / (kEpiWarps / 2), q = warp & 3, half = (e % (kEpiWarps / 2)) / 4;
+        const int r = g * kBM + q * 32 + lane;           // tile row: TMEM slot g, lane q * 32 + lane
+        const uint32_t tb = tmem_base + 256u * g + (static_cast<uint32_t>(q * 32) << 16);
+        const uint32_t ring = ptx::smem_u32(smem);
+        __syncwarp();
+        ptx::tc_fence_before();
+        ptx::cluster_sync();   // all accumulators of the cluster are final; no copy or MMA uses a ring
+        ptx::tc_fence_after();
+        if (warp >= 2 && has_unit) {
+            // the warp's half of the columns holds the blocks of owners 2 half and 2 half + 1
+            for (int o = 2 * half; o < 2 * half + 2; ++o) {
+                if (o == crank) continue;
+                const int slot = crank < o ? crank : crank - 1;
+                const uint32_t dst = ptx::mapa_shared(ring + slot * kSlotBytes + r * kRowF4 * 16, o);
+#pragma unroll
+                for (int nb = 0; nb < NB; ++nb) {
+                    uint32_t ra[32];
+                    ptx::tmem_ld_32cols(tb + nb * BN + o * kOwn, ra);
+#pragma unroll
+                    for (int f = 0; f < 8; ++f)
+                        ptx::st_cluster_f4(dst + ((nb * 8 + f) ^ (r & 7)) * 16, __uint_as_float(ra[4 * f]),
+                                           __uint_as_float(ra[4 * f + 1]), __uint_as_float(ra[4 * f + 2]),
+                                           __uint_as_float(ra[4 * f + 3]));
+                }
+            }
+        }
+        __syncwarp();
+        ptx::cluster_sync();   // every block is in its owner's shared memory
+        if (warp >= 2 && has_unit) {
+            // this warp: 16 of the own block's columns, c0 .. c0 + 15 of the tile
+            const Unit w = unit_of(cid);
+            const int c0 = crank * kOwn + half * 16;
+            const int row = w.mg * MT * kBM + r;
+            float acc[NB][16];
+#pragma unroll
+            for (int kx = 0; kx < CL; ++kx) {
+#pragma unroll
+                for (int nb = 0; nb < NB; ++nb) {
+                    float v[16];
+                    if (kx == crank) {
+                        uint32_t ra[16];
+                        ptx::tmem_ld_16cols(tb + nb * BN + c0, ra);
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(ra[j]);
+                    } else {
+                        const int slot = kx < crank ? kx : kx - 1;
+                        const float4* src = reinterpret_cast<const float4*>(smem + slot * kSlotBytes + r * kRowF4 * 16);
+#pragma unroll
+                        for (int f = 0; f < 4; ++f) {
+                            const float4 t = src[(nb * 8 + half * 4 + f) ^ (r & 7)];
+                            v[4 * f] = t.x;
+                            v[4 * f + 1] = t.y;
+                            v[4 * f + 2] = t.z;
+                            v[4 * f + 3] = t.w;
+                        }
+                    }
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) acc[nb][j] = kx == 0 ? v[j] : acc[nb][j] + v[j];
+                }
+            }
+            if (row < n_rows) {
+                const size_t col = static_cast<size_t>(w.nt) * BN + c0;
+                uint32_t packed[8];
+                if constexpr (EPI == EPI_CGATEUP) {
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        packed[j] = pack_bf16x2(silu_f(acc[0][2 * j]) * acc[NB - 1][2 * j],
+                                                silu_f(acc[0][2 * j + 1]) * acc[NB - 1][2 * j + 1]);
+                } else {
+                    const int sq = row / ep.R, rr = row - sq * ep.R;
+                    const int hid_row = sq * ep.gamma + stage2_hidden_index(rr, ep.M);
+                    const uint4* res = reinterpret_cast<const uint4*>(ep.hidden + static_cast<size_t>(hid_row) * ep.ld_out + col);
+#pragma unroll
+                    for (int j = 0; j < 2; ++j) {
+                        const uint4 hv = res[j];
+                        const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w};
+#pragma unroll
+                        for (int t = 0; t < 4; ++t) {
+                            const __nv_bfloat162 h2 = *reinterpret_cast<const __nv_bfloat162*>(&hw[t]);
+                            packed[4 * j + t] = pack_bf16x2(__bfloat162float(h2.x) + acc[0][8 * j + 2 * t],
+                                                            __bfloat162float(h2.y) + acc[0][8 * j + 2 * t + 1]);
+                        }
+                    }
+                }
+                uint4* dst = reinterpret_cast<uint4*>(ep.out + static_cast<size_t>(row) * ep.ld_out + col);
+                dst[0] = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+                dst[1] = make_uint4(packed[4], packed[5], packed[6], packed[7]);
+            }
+        }
+    }
+
     // the producer and MMA lanes rejoin their warps first: the CTA-wide barrier below must wait
     // for every thread, not only for each warp's first arrivals
     __syncwarp();
@@ -546,7 +667,12 @@ cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& t
     if (e != cudaSuccess) return e;
     const int n_units = n_ntiles * n_mgroups * k_splits;
     const int stream_once = n_mgroups == 1 ? 1 : 0;
-    if constexpr (CL == 1) {
+    if constexpr (EPI == EPI_CGATEUP || EPI == EPI_CDOWN) {
+        // one output tile per cluster, its K-ranges on the cluster's CTAs; the caller has checked
+        // that all clusters are resident at once (splitk_clusters_fit)
+        e = launch_pdl_cluster(kern, dim3(CL * n_ntiles * n_mgroups), dim3(kThreads), C::kSmemBytes, ctx.stream, CL,
+                               tx, tw0, tw1, n_rows, K, n_ntiles, n_mgroups, CL, stream_once, ep, ctx.status);
+    } else if constexpr (CL == 1) {
         const int grid = n_units < ctx.num_sms ? n_units : ctx.num_sms;
         e = launch_pdl(kern, dim3(grid), dim3(kThreads), C::kSmemBytes, ctx.stream, tx, tw0, tw1, n_rows, K,
                        n_ntiles, n_mgroups, k_splits, stream_once, ep, ctx.status);
@@ -557,6 +683,38 @@ cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& t
                                n_rows, K, n_ntiles, n_mgroups, k_splits, stream_once, ep, ctx.status);
     }
     return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// Whether n_tiles clusters of the split-K kernel can all be resident at once (each cluster then
+// runs its one tile and the ring can take the partial sums; a second wave would serialise them).
+template <int EPI, int MT, int NB, int BN, int STAGES, int CL>
+bool splitk_clusters_fit(const Ctx& ctx, int n_tiles) {
+    using C = TileCfg<MT, NB, BN, STAGES>;
+    auto kern = tc_gemm_kernel<EPI, MT, NB, BN, STAGES, CL>;
+    static const int max_cl = [&] {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) != cudaSuccess) {
+            (void)cudaGetLastError();
+            return 0;
+        }
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(CL * (ctx.num_sms / CL));
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = C::kSmemBytes;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = CL;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+            (void)cudaGetLastError();
+            return 0;
+        }
+        return n;
+    }();
+    return n_tiles <= max_cl;
 }
 
 }  // namespace
@@ -625,6 +783,10 @@ cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, const void* w_gate, 
             e = m_tiles == 1 ? run_gemm<EPI_GATEUP, 1, 2, 64, 6>(ctx, tx, tg, tu, n_rows, 2 * d, I / 64, 1, ep)
                              : run_gemm<EPI_GATEUP, 2, 2, 64, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / 64, n_mg, ep);
         if (e != cudaSuccess) return e;
+    } else if (m_tiles == 2 && bn_gu == BN && ks1 == 4 &&
+               splitk_clusters_fit<EPI_CGATEUP, 2, 2, BN, 3, 4>(ctx, I / BN)) {
+        e = run_gemm<EPI_CGATEUP, 2, 2, BN, 3, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, 1, ep, 4);
+        if (e != cudaSuccess) return e;
     } else {
         if (bn_gu == BN)
             e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 2, BN, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, 1, ep, ks1)
@@ -656,6 +818,8 @@ cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, const void* w_gate, 
         return m_tiles == 1 ? run_gemm<EPI_DOWN, 1, 1, 64, 8>(ctx, ta, td, td, n_rows, I, d / 64, 1, ed)
                             : run_gemm<EPI_DOWN, 2, 1, 64, 5>(ctx, ta, td, td, n_rows, I, d / 64, n_mg, ed);
     }
+    if (m_tiles == 2 && bn_d == BN && ks2 == 4 && splitk_clusters_fit<EPI_CDOWN, 2, 1, BN, 4, 4>(ctx, d / BN))
+        return run_gemm<EPI_CDOWN, 2, 1, BN, 4, 4>(ctx, ta, td, td, n_rows, I, d / BN, 1, ed, 4);
     if (bn_d == BN)
         e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 1, BN, 6>(ctx, ta, td, td, n_rows, I, d / BN, 1, ed, ks2)
                          : run_gemm<EPI_PARTIAL, 2, 1, BN, 4>(ctx, ta, td, td, n_rows, I, d / BN, n_mg, ed, ks2);

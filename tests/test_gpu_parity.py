@@ -108,6 +108,14 @@ def test_bf16_d_and_I_several_k_blocks():
     check(cfg)
 
 
+def test_bf16_two_m_tiles_cluster_split_k():
+    # 1 + M(gamma - 1) = 241 stage-2 rows (two 128-row tiles) with d = I = 512: both approximator
+    # GEMMs split K over 4-CTA clusters and add the partial sums in distributed shared memory
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=1, d=512, I=512, V=3000, gamma=16, M=16,
+                           K2=16, B=32)
+    check(cfg)
+
+
 @pytest.mark.parametrize("mode", ["marginal", "marginal_mary"])
 def test_bf16_marginal_modes(mode):
     check(synth.get_config("tiny_peaked", dtype="bf16", batch=3, V=2000, mode=mode))
