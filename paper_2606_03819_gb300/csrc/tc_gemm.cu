@@ -373,14 +373,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 if (row - lane < n_rows) {
                     float hm = -INFINITY, hsum = 0.0f, hbv = -INFINITY;
                     int hbid = -1;
-#pragma unroll
-                    for (int j = 0; j < kHalf; ++j) {
-                        const int ci = half * kHalf + j;
-                        const int v0 = nt * BN + ci * kChunk;
-                        uint32_t ra[32];
-                        ptx::tmem_ld_32cols(tb + ci * kChunk, ra);
-                        const ChunkNode c = chunk_tree<0, 32>(ra, v0, ep.V, ep.inv_temp);
-                        // half summary; chunks arrive in id order, so strict > keeps the smaller id
+                    // half summary; chunks arrive in id order, so strict > keeps the smaller id
+                    auto fold = [&](const ChunkNode& c, int ci, int v0) {
                         if (c.a1 > hbv) {
                             hbv = c.a1;
                             hbid = v0 + c.i1;
@@ -393,7 +387,35 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                         if (row < n_rows)
                             P.chunks[P.chunk_at(nt, ci, row)] =
                                 make_float4(c.a1, c.a2, c.a3, __int_as_float(c.i1 | (c.i2 << 8)));
-                        __syncwarp();   // reconverge before the next warp-collective TMEM load
+                    };
+                    // Chunks in pairs: both TMEM loads in flight together, the two trees independent
+                    // of each other (so their instructions interleave), and the next pair's loads
+                    // issued before this pair is folded and stored.
+                    const int cb = half * kHalf;
+                    uint32_t ra[32], rb[32];
+                    ptx::tmem_ld_32cols_nowait(tb + cb * kChunk, ra);
+                    ptx::tmem_ld_32cols_nowait(tb + (cb + 1) * kChunk, rb);
+                    ptx::tmem_wait_ld_regs(ra);
+                    ptx::tmem_wait_ld_regs(rb);
+#pragma unroll
+                    for (int pr = 0; pr < kHalf / 2; ++pr) {
+                        const int ci = cb + 2 * pr;
+                        const int v0 = nt * BN + ci * kChunk;
+                        const ChunkNode c0 = chunk_tree<0, 32>(ra, v0, ep.V, ep.inv_temp);
+                        const ChunkNode c1 = chunk_tree<0, 32>(rb, v0 + kChunk, ep.V, ep.inv_temp);
+                        const bool more = pr + 1 < kHalf / 2;
+                        if (more) {
+                            __syncwarp();   // converged for the warp-collective TMEM loads
+                            ptx::tmem_ld_32cols_nowait(tb + (ci + 2) * kChunk, ra);
+                            ptx::tmem_ld_32cols_nowait(tb + (ci + 3) * kChunk, rb);
+                        }
+                        fold(c0, ci, v0);
+                        fold(c1, ci + 1, v0 + kChunk);
+                        if (more) {
+                            __syncwarp();
+                            ptx::tmem_wait_ld_regs(ra);
+                            ptx::tmem_wait_ld_regs(rb);
+                        }
                     }
                     if (row < n_rows)
                         P.halves[P.half_at(nt, half, row)] = make_float4(hm, hsum, hbv, __int_as_float(hbid));
@@ -486,8 +508,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         // The tile's output columns are owned in CL blocks of BN / CL: CTA o adds the CL partial
         // sums of block o in K-range order (the order of the split-K reduction kernels) and
         // applies the epilogue. Every CTA first writes the blocks it does not own into their
-        // owners' stage rings (idle once all MMAs of the cluster are done), row r's 16-byte units
-        // permuted by r % 8 so that the 32 rows of a warp spread over the banks.
+        // owners' stage rings (idle once all MMAs of the cluster are done), laid out
+        // [16-byte unit][row] so that the 32 lanes (rows) of a warp store 512 contiguous bytes.
         constexpr int kOwn = BN / CL;                    // output columns per owner
         constexpr int kRowF4 = NB * kOwn / 4;            // 16-byte units per row of a block
         constexpr int kSlotBytes = MT * kBM * kRowF4 * 16;
@@ -508,14 +530,14 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             for (int o = 2 * half; o < 2 * half + 2; ++o) {
                 if (o == crank) continue;
                 const int slot = crank < o ? crank : crank - 1;
-                const uint32_t dst = ptx::mapa_shared(ring + slot * kSlotBytes + r * kRowF4 * 16, o);
+                const uint32_t dst = ptx::mapa_shared(ring + slot * kSlotBytes + r * 16, o);
 #pragma unroll
                 for (int nb = 0; nb < NB; ++nb) {
                     uint32_t ra[32];
                     ptx::tmem_ld_32cols(tb + nb * BN + o * kOwn, ra);
 #pragma unroll
                     for (int f = 0; f < 8; ++f)
-                        ptx::st_cluster_f4(dst + ((nb * 8 + f) ^ (r & 7)) * 16, __uint_as_float(ra[4 * f]),
+                        ptx::st_cluster_f4(dst + (nb * 8 + f) * (MT * kBM * 16), __uint_as_float(ra[4 * f]),
                                            __uint_as_float(ra[4 * f + 1]), __uint_as_float(ra[4 * f + 2]),
                                            __uint_as_float(ra[4 * f + 3]));
                 }
@@ -541,10 +563,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                         for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(ra[j]);
                     } else {
                         const int slot = kx < crank ? kx : kx - 1;
-                        const float4* src = reinterpret_cast<const float4*>(smem + slot * kSlotBytes + r * kRowF4 * 16);
+                        const float4* src = reinterpret_cast<const float4*>(smem + slot * kSlotBytes) + r;
 #pragma unroll
                         for (int f = 0; f < 4; ++f) {
-                            const float4 t = src[(nb * 8 + half * 4 + f) ^ (r & 7)];
+                            const float4 t = src[(nb * 8 + half * 4 + f) * (MT * kBM)];
                             v[4 * f] = t.x;
                             v[4 * f + 1] = t.y;
                             v[4 * f + 2] = t.z;
