@@ -98,7 +98,7 @@ Layout layout(const Dims& D) {
     L.X = take(rows2 * 2 * D.d * D.esize);
     L.A = take(rows2 * D.I * D.esize);
     L.hp = take(rows2 * D.d * D.esize);
-    // split-K partial sums of the bf16 approximator GEMMs: [k_splits][max(2I, d) / 32][rows][32] fp32
+    // split-K partial sums of the bf16 approximator GEMMs: [k_splits][max(2I, d) / 4][rows][4] fp32
     L.kpart = D.dtype == TF_BF16 ? take(static_cast<size_t>(kMaxKSplits) * rows2 *
                                         (2 * static_cast<size_t>(D.I) > static_cast<size_t>(D.d) ? 2 * D.I : D.d) * 4)
                                  : take(0);

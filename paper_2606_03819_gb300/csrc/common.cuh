@@ -168,7 +168,7 @@ cudaError_t launch_gather_norm(const Ctx&, int dtype, const void* hidden, const 
 cudaError_t launch_swiglu_tc(const Ctx&, const void* X, const void* w_gate, const void* w_up,
                              const void* w_down, const void* hidden, int n_rows, int d, int I,
                              int R, int M, int gamma, void* A, void* h_prime, float* partial);
-// split-K reductions of the approximator GEMMs (partial sums in fp32, [k_splits][N / 32][rows][32])
+// split-K reductions of the approximator GEMMs (partial sums in fp32, [k_splits][N / 4][rows][4])
 cudaError_t launch_swiglu_reduce(const Ctx&, const float* partial, int k_splits, int n_rows, int I,
                                  __nv_bfloat16* A);
 cudaError_t launch_down_reduce(const Ctx&, const float* partial, int k_splits, int n_rows, int d,

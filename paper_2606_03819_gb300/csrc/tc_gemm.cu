@@ -52,7 +52,7 @@ struct EpiParams {
     int ld_out;
     const __nv_bfloat16* hidden; // DOWN: residual rows, [b * gamma, ld_out]
     int R, M, gamma;
-    float* partial;              // PARTIAL: fp32 sums [k_splits][n_cols / 32][n_rows][32] (chunk-major),
+    float* partial;              // PARTIAL: fp32 sums [k_splits][n_cols / 4][n_rows][4] (float4-major),
     int n_cols;                  //          accumulator nb of N tile nt at columns nb * n_total + nt * BN
     int n_total;                 // N of the whole GEMM (n_ntiles * BN)
     int reset_status;            // LMHEAD: zero *status first (the first kernel of a stage-1 call)
@@ -423,9 +423,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 ptx::tc_fence_before();
                 ptx::mbar_arrive(&tempty[g]);
             } else if constexpr (EPI == EPI_PARTIAL) {
-                // chunk-major: a lane's 32 columns are 128 contiguous bytes and the warp's 32 rows
-                // one contiguous 4 KB block
-                float* split = ep.partial + static_cast<size_t>(w.kx) * ep.n_cols * n_rows;
+                // float4-major: each store instruction writes the warp's 32 rows of 4 columns, 512
+                // contiguous bytes
+                float4* split = reinterpret_cast<float4*>(ep.partial + static_cast<size_t>(w.kx) * ep.n_cols * n_rows);
 #pragma unroll 1
                 for (int nb = 0; nb < NB; ++nb) {
 #pragma unroll 1
@@ -434,11 +434,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                         ptx::tmem_ld_32cols(tb + nb * BN + c, ra);
                         if (row < n_rows) {
                             const int col = nb * ep.n_total + nt * BN + c;
-                            float4* dst = reinterpret_cast<float4*>(
-                                split + (static_cast<size_t>(col >> 5) * n_rows + row) * 32);
+                            float4* dst = split + static_cast<size_t>(col >> 2) * n_rows + row;
 #pragma unroll
                             for (int j = 0; j < 8; ++j)
-                                dst[j] = make_float4(__uint_as_float(ra[4 * j]), __uint_as_float(ra[4 * j + 1]),
+                                dst[static_cast<size_t>(j) * n_rows] = make_float4(__uint_as_float(ra[4 * j]), __uint_as_float(ra[4 * j + 1]),
                                                      __uint_as_float(ra[4 * j + 2]), __uint_as_float(ra[4 * j + 3]));
                         }
                     }
