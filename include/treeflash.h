@@ -13,6 +13,7 @@
  *                                           "Inference"), the M-ary rule for non-leaves.
  *   verification     (tf_tree_mask)         ancestor mask and position ids for the verifier's
  *                                           single parallel pass over the tree (Sec. 1, Sec. 3).
+ *   Part 2 + mask    (tf_build_tree_mask)   both of the above; one launch for B + 1 <= 128.
  *
  * Conventions shared by every call:
  *  - Pointers are DEVICE pointers owned by the caller unless a parameter says "host". The
@@ -179,9 +180,22 @@ tf_status tf_tree_mask(const tf_dims* dims, const int32_t* node_parent, const in
                        const int32_t* root_pos, uint8_t* mask, int32_t* pos_ids,
                        tf_stream_t stream);
 
+/* tf_build_tree followed by tf_tree_mask, with the same arguments and results: the two outputs
+ * of both calls, bit for bit. When B + 1 <= 128 the mask and position ids are written by the
+ * builder itself from the tree it holds (one launch instead of two); larger trees run both
+ * launches. root_pos [b] int32; mask [b, B+1, B+1] uint8 and pos_ids [b, B+1] int32 out, as in
+ * tf_tree_mask. */
+tf_status tf_build_tree_mask(const tf_dims* dims, const int32_t* root_tok, const int32_t* root_pos,
+                             const int32_t* top_ids, const float* top_logp,
+                             const int32_t* child_ids, const float* child_logp,
+                             int32_t* node_tok, int32_t* node_parent, int32_t* node_depth,
+                             float* node_score, uint8_t* mask, int32_t* pos_ids,
+                             int32_t* dev_status, tf_stream_t stream);
+
 /* The whole drafting step for callers holding the step's inputs in HOST memory (pinned memory
- * makes the copies asynchronous): copies hidden/root_tok/root_pos to the device, runs the four
- * calls above, copies the tree, mask and status back, and synchronises `stream`.
+ * makes the copies asynchronous): copies hidden/root_tok/root_pos to the device, runs stage 1,
+ * stage 2 (TF_MODE_AR) and tf_build_tree_mask, copies the tree, mask and status back, and
+ * synchronises `stream`.
  * Host inputs: hidden [b, gamma, d] dtype, root_tok [b], root_pos [b]. Host outputs:
  * node_tok, node_parent, node_depth [b, B+1] int32, node_score [b, B+1] float,
  * mask [b, B+1, B+1] uint8, pos_ids [b, B+1] int32, dev_status [b] int32 (per-sequence bits

@@ -44,7 +44,7 @@ class TfWeights(ctypes.Structure):
 
 
 EXPORTS = ("tf_status_string", "tf_version", "tf_kernel_launches", "tf_workspace_size", "tf_status_reset", "tf_status_read",
-           "tf_stage1_marginals", "tf_stage2_ar_approx", "tf_build_tree", "tf_tree_mask",
+           "tf_stage1_marginals", "tf_stage2_ar_approx", "tf_build_tree", "tf_tree_mask", "tf_build_tree_mask",
            "tf_draft_tree_host", "tf_lmhead_partials", "tf_lmhead_merge", "tf_ar_approx",
            "tf_workspace_h_prime", "tf_workspace_view", "tf_stage1_marginals_static", "tf_accept_walk")
 
@@ -74,6 +74,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
         "tf_stage2_ar_approx": (ctypes.c_int, [D, W, P, P, P, P, P, P, SZ, P]),
         "tf_build_tree": (ctypes.c_int, [D, P, P, P, P, P, P, P, P, P, P, P]),
         "tf_tree_mask": (ctypes.c_int, [D, P, P, P, P, P, P]),
+        "tf_build_tree_mask": (ctypes.c_int, [D, P, P, P, P, P, P, P, P, P, P, P, P, P, P]),
         "tf_draft_tree_host": (ctypes.c_int, [D, W, P, P, P, P, P, P, P, P, P, P, P, SZ, P]),
         "tf_lmhead_partials": (ctypes.c_int, [D, P, P, I32, P, SZ, P]),
         "tf_lmhead_merge": (ctypes.c_int, [D, P, P, I32, I32, P, P, P, SZ, P]),
@@ -215,6 +216,14 @@ def tf_tree_mask(dims: Dims, node_parent, node_depth, root_pos, mask, pos_ids, s
     _check("tf_tree_mask", load_library().tf_tree_mask(
         ctypes.byref(dims.c()), _ptr(node_parent), _ptr(node_depth), _ptr(root_pos), _ptr(mask),
         _ptr(pos_ids), _stream(stream)))
+
+
+def tf_build_tree_mask(dims: Dims, root_tok, root_pos, top_ids, top_logp, child_ids, child_logp, node_tok,
+                       node_parent, node_depth, node_score, mask, pos_ids, dev_status, stream=None):
+    _check("tf_build_tree_mask", load_library().tf_build_tree_mask(
+        ctypes.byref(dims.c()), _ptr(root_tok), _ptr(root_pos), _ptr(top_ids), _ptr(top_logp), _ptr(child_ids),
+        _ptr(child_logp), _ptr(node_tok), _ptr(node_parent), _ptr(node_depth), _ptr(node_score), _ptr(mask),
+        _ptr(pos_ids), _ptr(dev_status), _stream(stream)))
 
 
 def tf_draft_tree_host(dims: Dims, w: dict, hidden, root_tok, root_pos, node_tok, node_parent, node_depth,

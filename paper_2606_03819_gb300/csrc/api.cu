@@ -346,6 +346,27 @@ tf_status tf_tree_mask(const tf_dims* dims, const int32_t* node_parent, const in
     return cuda_status(launch_tree_mask(ctx, D.b, D.B, node_parent, node_depth, root_pos, mask, pos_ids));
 }
 
+tf_status tf_build_tree_mask(const tf_dims* dims, const int32_t* root_tok, const int32_t* root_pos,
+                             const int32_t* top_ids, const float* top_logp, const int32_t* child_ids,
+                             const float* child_logp, int32_t* node_tok, int32_t* node_parent, int32_t* node_depth,
+                             float* node_score, uint8_t* mask, int32_t* pos_ids, int32_t* dev_status,
+                             tf_stream_t stream) {
+    Dims D;
+    TF_TRY(check_dims(dims, &D));
+    if (!root_tok || !root_pos || !top_ids || !top_logp || !node_tok || !node_parent || !node_depth || !node_score ||
+        !mask || !pos_ids || !dev_status)
+        return TF_ERR_INVALID_ARG;
+    if (D.mode == TF_MODE_AR && (!child_ids || !child_logp)) return TF_ERR_INVALID_ARG;
+    Ctx ctx{reinterpret_cast<cudaStream_t>(stream), 0, nullptr};
+    const bool fused = D.B + 1 <= kFusedMaskMaxNodes;   // the builder CTA writes the mask of its tree
+    TF_TRY(cuda_status(launch_build_tree(ctx, D.b, D.gamma, D.M, D.K1, D.K2, D.B, D.V, D.mode, D.R, root_tok, top_ids,
+                                         top_logp, child_ids, child_logp, node_tok, node_parent, node_depth,
+                                         node_score, dev_status, fused ? root_pos : nullptr,
+                                         fused ? mask : nullptr, fused ? pos_ids : nullptr)));
+    if (fused) return TF_OK;
+    return cuda_status(launch_tree_mask(ctx, D.b, D.B, node_parent, node_depth, root_pos, mask, pos_ids));
+}
+
 tf_status tf_accept_walk(const tf_dims* dims, const int32_t* node_tok, const int32_t* node_parent,
                          const int32_t* verifier_tok, int32_t* accept_len, int32_t* accept_path, int32_t* next_tok,
                          tf_stream_t stream) {
@@ -432,9 +453,9 @@ tf_status tf_draft_tree_host(const tf_dims* dims, const tf_weights* w, const voi
     uint8_t* d_mask = at<uint8_t>(ws, L.n_mask);
     int32_t* d_posid = at<int32_t>(ws, L.n_pos);
     int32_t* d_stat = at<int32_t>(ws, L.n_stat);
-    TF_TRY(tf_build_tree(dims, d_root, top_ids, top_logp, D.mode == TF_MODE_AR ? child_ids : nullptr,
-                         D.mode == TF_MODE_AR ? child_logp : nullptr, d_tok, d_par, d_dep, d_score, d_stat, stream));
-    TF_TRY(tf_tree_mask(dims, d_par, d_dep, d_pos, d_mask, d_posid, stream));
+    TF_TRY(tf_build_tree_mask(dims, d_root, d_pos, top_ids, top_logp, D.mode == TF_MODE_AR ? child_ids : nullptr,
+                              D.mode == TF_MODE_AR ? child_logp : nullptr, d_tok, d_par, d_dep, d_score, d_mask,
+                              d_posid, d_stat, stream));
     TF_TRY(cuda_status(cudaMemcpyAsync(node_tok, d_tok, nn * 4, cudaMemcpyDeviceToHost, st)));
     TF_TRY(cuda_status(cudaMemcpyAsync(node_parent, d_par, nn * 4, cudaMemcpyDeviceToHost, st)));
     TF_TRY(cuda_status(cudaMemcpyAsync(node_depth, d_dep, nn * 4, cudaMemcpyDeviceToHost, st)));

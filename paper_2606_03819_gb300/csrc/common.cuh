@@ -182,7 +182,11 @@ cudaError_t launch_build_tree(const Ctx&, int b, int gamma, int M, int K1, int K
                               int mode, int R, const int32_t* root_tok, const int32_t* top_ids,
                               const float* top_logp, const int32_t* child_ids,
                               const float* child_logp, int32_t* node_tok, int32_t* node_parent,
-                              int32_t* node_depth, float* node_score, int32_t* dev_status);
+                              int32_t* node_depth, float* node_score, int32_t* dev_status,
+                              const int32_t* root_pos = nullptr, uint8_t* mask = nullptr,
+                              int32_t* pos_ids = nullptr);
+// the largest tree (B + 1 nodes) whose mask launch_build_tree can write from the builder itself
+constexpr int kFusedMaskMaxNodes = 128;
 cudaError_t launch_accept_walk(const Ctx&, int b, int B, int gamma, const int32_t* node_tok,
                                const int32_t* node_parent, const int32_t* verifier_tok,
                                int32_t* accept_len, int32_t* accept_path, int32_t* next_tok);

@@ -94,6 +94,11 @@ struct TreeArgs {
     int32_t* node_depth;
     float* node_score;
     int32_t* dev_status;
+    // optional, with B + 1 <= kMaskRows: the builder also writes the verification mask and
+    // position ids (tf_tree_mask's outputs) from the tree it holds in shared memory
+    const int32_t* root_pos;
+    uint8_t* mask;
+    int32_t* pos_ids;
 };
 
 // Index m of `tok` among the M <= 64 stage-1 candidates of depth `dep` (the M-ary rule of
@@ -113,13 +118,14 @@ __device__ __forceinline__ unsigned long long queue_key(float score, int depth, 
 }
 
 constexpr int kTreeThreads = 256;
-constexpr int kMaskRows = 128;    // mask rows per CTA
+constexpr int kMaskRows = kFusedMaskMaxNodes;    // mask rows per CTA (the fused mask is one block)
 
 // Shared-memory bytes of build_tree_kernel: queue, node arrays, stage-1 top-M, and (when they
 // fit) the sequence's child lists.
-__host__ __device__ inline size_t tree_smem_fixed(int B, int gamma, int M) {
+__host__ __device__ inline size_t tree_mask_words(int n) { return static_cast<size_t>(n) * ((n + 31) / 32); }
+__host__ __device__ inline size_t tree_smem_fixed(int B, int gamma, int M, bool with_mask) {
     return static_cast<size_t>(B + 2) * (8 + 4 * 4) + static_cast<size_t>(B + 1) * 4 * 4 +
-           static_cast<size_t>(gamma) * M * 4 + 16;
+           static_cast<size_t>(gamma) * M * 4 + 16 + (with_mask ? tree_mask_words(B + 1) * 4 + 16 : 0);
 }
 // Bytes of the staged list prefixes: the first sw entries of each of the rows child lists.
 __host__ __device__ inline size_t tree_smem_lists(int rows, int sw) { return static_cast<size_t>(rows) * sw * 8; }
@@ -151,6 +157,7 @@ struct TreeSmem {
     int *o_tok, *o_par, *o_dep;
     float* o_score;
     int* topm;        // [gamma, M]
+    uint32_t* anc;    // with the fused mask: [B + 1][(B + 32) / 32] ancestor-or-self bits
     uint8_t* lists;   // staged prefixes: ids [rows][sw] int32, then log-probs [rows][sw] float
 };
 __device__ __forceinline__ TreeSmem tree_smem(uint8_t* base, const TreeArgs& a) {
@@ -166,8 +173,13 @@ __device__ __forceinline__ TreeSmem tree_smem(uint8_t* base, const TreeArgs& a) 
     t.o_dep = t.o_par + n_out;
     t.o_score = reinterpret_cast<float*>(t.o_dep + n_out);
     t.topm = reinterpret_cast<int*>(t.o_score + n_out);
-    t.lists = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(t.topm + a.gamma * a.M) + 15) &
-                                         ~static_cast<uintptr_t>(15));
+    uint8_t* next = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(t.topm + a.gamma * a.M) + 15) &
+                                               ~static_cast<uintptr_t>(15));
+    t.anc = reinterpret_cast<uint32_t*>(next);
+    if (a.mask)
+        next = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(t.anc + tree_mask_words(n_out)) + 15) &
+                                          ~static_cast<uintptr_t>(15));
+    t.lists = next;
     return t;
 }
 
@@ -254,6 +266,52 @@ __device__ __forceinline__ void write_nodes(const TreeArgs& a, int s, const Tree
         a.node_depth[o] = t.o_dep[i];
         a.node_score[o] = t.o_score[i];
     }
+}
+
+// Rows r0 .. r1-1 of one sequence's tree-attention mask and their position ids. mask[i][j] = 1
+// iff node j is node i or one of its ancestors; pos = root_pos + depth. Each node walks its own
+// parent chain (at most kMaxGamma links) and sets the bits of its row, so no thread waits for
+// another level. A node is present iff every link of its chain goes to a smaller index exactly
+// one level up and the chain ends at the root (node 0, depth 0); absent nodes (missing from an
+// underfull tree, or behind a broken link) get an empty row and column and pos -1.
+// par, dep: the tree's n parents and depths (shared memory); anc: (r1 - r0) x W words of shared
+// scratch; mask_s [n][n] and pos_s [n]: this sequence's outputs.
+__device__ __forceinline__ void mask_rows(int n, const int* par, const int* dep, int root_pos, int r0, int r1,
+                                          uint32_t* anc, uint8_t* mask_s, int32_t* pos_s) {
+    const int W = (n + 31) / 32;
+    for (int i = r0 + static_cast<int>(threadIdx.x); i < r1; i += blockDim.x) {
+        uint32_t* row = anc + static_cast<size_t>(i - r0) * W;
+        for (int w = 0; w < W; ++w) row[w] = 0u;
+        bool ok = true;
+        int j = i;
+        for (int steps = 0; ok && j != 0; ++steps) {
+            const int p = par[j];
+            ok = steps < kMaxGamma && dep[j] >= 1 && dep[j] <= kMaxGamma && p >= 0 && p < j && dep[p] == dep[j] - 1;
+            row[j >> 5] |= 1u << (j & 31);
+            j = p;
+        }
+        ok = ok && dep[0] == 0;
+        if (ok) {
+            row[0] |= 1u;                                  // the root
+        } else {
+            for (int w = 0; w < W; ++w) row[w] = 0u;       // absent: empty row
+        }
+        pos_s[i] = ok ? root_pos + dep[i] : -1;
+    }
+    __syncthreads();
+    const int count = (r1 - r0) * n;
+    for (int idx = threadIdx.x; idx < count; idx += blockDim.x) {
+        const int i = idx / n, jcol = idx - (idx / n) * n;
+        mask_s[static_cast<size_t>(r0 + i) * n + jcol] = static_cast<uint8_t>((anc[i * W + (jcol >> 5)] >> (jcol & 31)) & 1u);
+    }
+}
+
+// The fused mask of a builder CTA, once its tree is complete in shared memory.
+__device__ __forceinline__ void fused_mask(const TreeArgs& a, int s, const TreeSmem& t) {
+    if (!a.mask) return;
+    const int n = a.B + 1;
+    mask_rows(n, t.o_par, t.o_dep, a.root_pos[s], 0, n, t.anc, a.mask + static_cast<size_t>(s) * n * n,
+              a.pos_ids + static_cast<size_t>(s) * n);
 }
 
 // General builder (any B): the queue in shared memory.
@@ -387,6 +445,7 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
     }
     __syncthreads();
     write_nodes(a, s, t);
+    fused_mask(a, s, t);
 }
 
 // Builder for B + 1 <= 32 S: the queue in registers, S slots per lane (slot j on lane j % 32,
@@ -522,15 +581,12 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
     }
     __syncthreads();
     write_nodes(a, s, t);
+    fused_mask(a, s, t);
 }
 
 // ------------------------------------------------------------------------------------------
-// mask[i][j] = 1 iff node j is node i or one of its ancestors; pos = root_pos + depth. Each
-// node walks its own parent chain (at most kMaxGamma links) and sets the bits of its row, so no
-// thread waits for another level. A node is present iff every link of its chain goes to a
-// smaller index exactly one level up and the chain ends at the root (node 0, depth 0); absent
-// nodes (missing from an underfull tree, or behind a broken link) get an empty row and
-// column and pos -1.
+// The tree-attention mask and position ids (mask_rows) of a drafted tree in global memory: one
+// CTA per sequence and block of kMaskRows rows.
 // ------------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __restrict__ node_parent,
                                                         const int32_t* __restrict__ node_depth,
@@ -539,12 +595,11 @@ __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __
     pdl_trigger();
     pdl_wait();
     extern __shared__ uint32_t sm[];
-    const int W = (n + 31) / 32;
     const int s = blockIdx.x;
     const int r0 = blockIdx.y * kMaskRows, r1 = min(n, r0 + kMaskRows);   // this CTA's rows
     int* par = reinterpret_cast<int*>(sm);
     int* dep = par + n;
-    uint32_t* anc = reinterpret_cast<uint32_t*>(dep + n);   // [kMaskRows][W] ancestor-or-self bits
+    uint32_t* anc = reinterpret_cast<uint32_t*>(dep + n);   // [kMaskRows][(n + 31) / 32] ancestor-or-self bits
     const int32_t* P = node_parent + static_cast<size_t>(s) * n;
     const int32_t* D = node_depth + static_cast<size_t>(s) * n;
     for (int i = threadIdx.x; i < n; i += blockDim.x) {
@@ -552,33 +607,8 @@ __global__ void __launch_bounds__(256) tree_mask_kernel(int n, const int32_t* __
         dep[i] = D[i];
     }
     __syncthreads();
-    for (int i = r0 + threadIdx.x; i < r1; i += blockDim.x) {
-        uint32_t* row = anc + static_cast<size_t>(i - r0) * W;
-        for (int w = 0; w < W; ++w) row[w] = 0u;
-        bool ok = true;
-        int j = i;
-        for (int steps = 0; ok && j != 0; ++steps) {
-            const int p = par[j];
-            ok = steps < kMaxGamma && dep[j] >= 1 && dep[j] <= kMaxGamma && p >= 0 && p < j && dep[p] == dep[j] - 1;
-            row[j >> 5] |= 1u << (j & 31);
-            j = p;
-        }
-        ok = ok && dep[0] == 0;
-        if (ok) {
-            row[0] |= 1u;                                  // the root
-        } else {
-            for (int w = 0; w < W; ++w) row[w] = 0u;       // absent: empty row
-        }
-        pos_ids[static_cast<size_t>(s) * n + i] = ok ? root_pos[s] + dep[i] : -1;
-    }
-    __syncthreads();
-    uint8_t* out = mask + static_cast<size_t>(s) * n * n;
-    const int count = (r1 - r0) * n;
-    for (int idx = threadIdx.x; idx < count; idx += blockDim.x) {
-        const int i = idx / n, jcol = idx - (idx / n) * n;
-        out[static_cast<size_t>(r0 + i) * n + jcol] =
-            static_cast<uint8_t>((anc[i * W + (jcol >> 5)] >> (jcol & 31)) & 1u);
-    }
+    mask_rows(n, par, dep, root_pos[s], r0, r1, anc, mask + static_cast<size_t>(s) * n * n,
+              pos_ids + static_cast<size_t>(s) * n);
 }
 
 // ------------------------------------------------------------------------------------------
@@ -789,10 +819,12 @@ cudaError_t launch_gather_norm(const Ctx& ctx, int dtype, const void* hidden, co
 cudaError_t launch_build_tree(const Ctx& ctx, int b, int gamma, int M, int K1, int K2, int B, int V, int mode, int R,
                               const int32_t* root_tok, const int32_t* top_ids, const float* top_logp,
                               const int32_t* child_ids, const float* child_logp, int32_t* node_tok,
-                              int32_t* node_parent, int32_t* node_depth, float* node_score, int32_t* dev_status) {
+                              int32_t* node_parent, int32_t* node_depth, float* node_score, int32_t* dev_status,
+                              const int32_t* root_pos, uint8_t* mask, int32_t* pos_ids) {
+    if (mask && B + 1 > kFusedMaskMaxNodes) return cudaErrorInvalidValue;
     TreeArgs a{gamma, M, K1, K2, B, V, mode, R, root_tok, top_ids, top_logp, child_ids, child_logp,
-               node_tok, node_parent, node_depth, node_score, dev_status};
-    const size_t fixed = tree_smem_fixed(B, gamma, M);
+               node_tok, node_parent, node_depth, node_score, dev_status, root_pos, mask, pos_ids};
+    const size_t fixed = tree_smem_fixed(B, gamma, M, mask != nullptr);
     const int rows_l = mode == TF_MODE_AR ? R : gamma;
     const int stride = mode == TF_MODE_AR ? K2 : K1;
     // stage the entries a tree can reach (rank <= B) when they fit, else a prefix that does

@@ -2,8 +2,8 @@
 
 The Drafter allocates, once, the workspace and every output tensor with torch on the target
 device, then each `draft` call queues tf_stage1_marginals -> tf_stage2_ar_approx (TreeFlash
-mode only) -> tf_build_tree -> tf_tree_mask on the current stream. Returned tensors are views
-of the Drafter's buffers and are overwritten by the next call.
+mode only) -> tf_build_tree_mask (the tree, then its verifier mask) on the current stream.
+Returned tensors are views of the Drafter's buffers and are overwritten by the next call.
 """
 from __future__ import annotations
 
@@ -45,10 +45,9 @@ class Drafter:
         return self.child_ids, self.child_logp
 
     def build(self, root_tok, root_pos, stream=None):
-        B.tf_build_tree(self.dims, root_tok, self.top_ids, self.top_logp, self.child_ids, self.child_logp,
-                        self.node_tok, self.node_parent, self.node_depth, self.node_score, self.dev_status,
-                        stream)
-        B.tf_tree_mask(self.dims, self.node_parent, self.node_depth, root_pos, self.mask, self.pos_ids, stream)
+        B.tf_build_tree_mask(self.dims, root_tok, root_pos, self.top_ids, self.top_logp, self.child_ids,
+                             self.child_logp, self.node_tok, self.node_parent, self.node_depth, self.node_score,
+                             self.mask, self.pos_ids, self.dev_status, stream)
 
     def draft(self, hidden, root_tok, root_pos, stream=None) -> dict:
         self.stage1(hidden, stream)
