@@ -13,7 +13,8 @@ What it computes (TreeFlash, "Parallel AR-Approximation for Faster Speculative D
   - stage 2: the AR-approximator of Eq. 1, h' = h + SwiGLU(h~ :: e), evaluated on one row
     for depth 1 (conditioned on the root token x_t) and on M rows for every depth
     i = 2..gamma (conditioned on the stage-1 candidates of depth i-1), each projected
-    through the LM head into q'.
+    through the LM head into q'; optionally with the "w/ Linear" ablation's linear layer in
+    place of the SwiGLU (reading R12).
 * Part 2 of Algorithm 1: OPT-Tree best-first selection (Sec. 3, "Inference") of B nodes by
   cumulative path log-probability; a popped node at depth i whose token is the stage-1
   candidate m of depth i gets the children distribution q'^(m)_{t+i+1}.
@@ -42,6 +43,11 @@ exp/log. Readings of points the paper leaves open (each also listed in the desig
   R10 Marginal baselines: "marginal" is DDTree (OPT-Tree on the stage-1 marginals, every
       node expandable, Sec. 4 "Baselines"); "marginal_mary" is the same search restricted
       by the M-ary rule of Sec. 3 (what TreeFlash reduces to with a zeroed approximator).
+  R12 The "w/ Linear" ablation (Sec. 4 "Model Design", Table 3) replaces the SwiGLU of
+      Eq. 1 by one linear layer on the same input: h' = h + W_lin (h~ :: e), W_lin [d, 2d],
+      no bias term. The token-dependent part of h' is then W_lin's embedding half applied
+      to e, the same for every hidden state: the "bias conditioned on the previous token"
+      the paper describes.
 
 Optional bf16 emulation (`emulate_bf16=True`) rounds to bfloat16 (round to nearest even)
 exactly where a bf16 implementation stores intermediates: the RMSNorm outputs, SiLU(G)*U,
@@ -138,13 +144,29 @@ def ar_approximator(h: np.ndarray, e_raw: np.ndarray, norm_h: np.ndarray, norm_e
     return rnd(h + a @ w_down.T)
 
 
+def linear_approximator(h: np.ndarray, e_raw: np.ndarray, norm_h: np.ndarray, norm_e: np.ndarray,
+                        w_lin: np.ndarray, eps: float, emulate_bf16: bool = False) -> np.ndarray:
+    """The "w/ Linear" ablation (reading R12): h' = h + W_lin (h~ :: e) with the same
+    normalised input as Eq. 1. h, e_raw: [rows, d]; w_lin: [d, 2d]."""
+    rnd = bf16_round if emulate_bf16 else (lambda a: a)
+    x = np.concatenate([rnd(rmsnorm(h, norm_h, eps)), rnd(rmsnorm(e_raw, norm_e, eps))], axis=1)
+    return rnd(h + x @ w_lin.T)
+
+
 def stage2(H: np.ndarray, root_tok: int, top_ids: np.ndarray, W: dict, M: int,
-           temperature: float, eps: float, emulate_bf16: bool = False):
-    """Stage 2 for one sequence: returns (h_prime [R, d], logp [R, V])."""
+           temperature: float, eps: float, emulate_bf16: bool = False, approx: str = "swiglu"):
+    """Stage 2 for one sequence: returns (h_prime [R, d], logp [R, V]). approx: "swiglu"
+    (Eq. 1) or "linear" (reading R12)."""
     gamma = H.shape[0]
     hid, prev = stage2_conditioning(gamma, M, root_tok, top_ids)
-    hp = ar_approximator(H[hid], W["embed"][prev], W["norm_h"], W["norm_e"],
-                         W["w_gate"], W["w_up"], W["w_down"], eps, emulate_bf16)
+    if approx == "swiglu":
+        hp = ar_approximator(H[hid], W["embed"][prev], W["norm_h"], W["norm_e"],
+                             W["w_gate"], W["w_up"], W["w_down"], eps, emulate_bf16)
+    elif approx == "linear":
+        hp = linear_approximator(H[hid], W["embed"][prev], W["norm_h"], W["norm_e"],
+                                 W["w_lin"], eps, emulate_bf16)
+    else:
+        raise ValueError(approx)
     return hp, log_softmax(lm_head(hp, W["lm_head"], temperature))
 
 
@@ -352,17 +374,17 @@ class SeqResult:
 def draft_sequence(H: np.ndarray, root_tok: int, root_pos: int, W: dict, *, M: int, K2: int,
                    B: int, temperature: float = 1.0, eps: float = 1e-6, mode: str = "ar",
                    emulate_bf16: bool = False, keep: Optional[int] = None,
-                   literal: bool = False) -> SeqResult:
+                   literal: bool = False, approx: str = "swiglu") -> SeqResult:
     """One sequence through Algorithm 1 (both parts) and the mask. W holds float64 arrays
     lm_head [V,d], embed [V,d], norm_h [d], norm_e [d], w_gate [I,2d], w_up [I,2d],
-    w_down [d,I]. `keep` truncates every child list (reading R5); None = whole
-    distributions."""
+    w_down [d,I] (approx "swiglu") or w_lin [d,2d] (approx "linear", reading R12). `keep`
+    truncates every child list (reading R5); None = whole distributions."""
     gamma = H.shape[0]
     K1 = max(M, K2)
     s1_logp, top_ids, top_logp = stage1(H, W["lm_head"], temperature, K1)
     hp = s2 = cids = clp = None
     if mode == "ar":
-        hp, s2 = stage2(H, root_tok, top_ids, W, M, temperature, eps, emulate_bf16)
+        hp, s2 = stage2(H, root_tok, top_ids, W, M, temperature, eps, emulate_bf16, approx)
         cids = np.stack([ranked(r, K2) for r in s2])
         clp = np.take_along_axis(s2, cids, axis=1)
     src = ChildSource(mode, gamma, M, top_ids, s1_logp, s2)
@@ -373,8 +395,8 @@ def draft_sequence(H: np.ndarray, root_tok: int, root_pos: int, W: dict, *, M: i
 
 
 def weights_f64(inputs: dict, to_f64) -> dict:
-    keys = ("lm_head", "embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down")
-    return {k: to_f64(inputs[k]) for k in keys}
+    keys = ("lm_head", "embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down", "w_lin")
+    return {k: to_f64(inputs[k]) for k in keys if inputs.get(k) is not None}
 
 
 # ---------------------------------------------------------------------------------------

@@ -45,11 +45,12 @@ class Config:
     B: int
     dtype: str = "bf16"            # "bf16" or "f32": storage and input type of every tensor
     mode: str = "ar"               # "ar" (TreeFlash), "marginal" (DDTree), "marginal_mary"
+    approx: str = "swiglu"         # stage-2 approximator: "swiglu" (Eq. 1) or "linear" (ablation)
     temperature: float = 1.0
     rms_eps: float = 1e-6
     seed: int = 0
     w_std: float = 0.02            # W_lm, E, W_gate, W_up
-    wd_std: float = 0.02           # W_down
+    wd_std: float = 0.02           # W_down, and W_lin of the linear approximator
     h_std: float = 1.0             # used when h_entropy is None: h ~ N(0, h_std^2)
     h_entropy: Optional[Tuple[float, float]] = None  # (nats at depth 1, nats at depth gamma)
 
@@ -92,6 +93,8 @@ CONFIGS = {
     # large draft budget (Fig. 5) with exact per-row lists (K2 = B), and wide branching (Fig. 6)
     "q8_b512": Config("q8_b512", batch=1, M=16, K2=512, B=512, **_Q8),
     "q8_m64": Config("q8_m64", batch=1, M=64, K2=64, B=64, **_Q8),
+    # the q8_b64 step with the "w/ Linear" ablation's approximator (Sec. 4, Table 3)
+    "q8_b64_linear": Config("q8_b64_linear", batch=1, M=16, K2=64, B=64, approx="linear", **_Q8),
     # the q8_b64 step with the vocabulary cut to 32768 (W_lm 268 MB, still twice the L2):
     # small enough for multi-pass profiler captures
     "prof_v32k": Config("prof_v32k", batch=1, M=16, K2=64, B=64, **dict(_Q8, V=32768)),
@@ -158,7 +161,9 @@ def make_inputs(cfg: Config, seed: Optional[int] = None) -> dict:
 
     Keys: hidden [b, gamma, d], lm_head [V, d], embed [V, d], norm_h [d], norm_e [d],
     w_gate [I, 2d], w_up [I, 2d], w_down [d, I], root_tok [b] int32, root_pos [b] int32,
-    h_scale [gamma] float64 (the per-depth hidden-state std that was used).
+    h_scale [gamma] float64 (the per-depth hidden-state std that was used), and for the linear
+    approximator w_lin [d, 2d] ~ N(0, wd_std^2), drawn last so that every other tensor is the
+    same as for the SwiGLU configuration of the same shape and seed.
     """
     seed = cfg.seed if seed is None else seed
     dt = torch.float32 if cfg.dtype == "f32" else torch.bfloat16
@@ -175,10 +180,13 @@ def make_inputs(cfg: Config, seed: Optional[int] = None) -> dict:
     hidden = base.to(dt)
     root_tok = torch.randint(0, V, (cfg.batch,), generator=g, dtype=torch.int64).to(torch.int32)
     root_pos = (torch.arange(cfg.batch, dtype=torch.int32) * 7 + 1000).to(torch.int32)
-    return dict(hidden=hidden, lm_head=lm_head, embed=embed,
-                norm_h=torch.ones(d, dtype=dt), norm_e=torch.ones(d, dtype=dt),
-                w_gate=w_gate, w_up=w_up, w_down=w_down,
-                root_tok=root_tok, root_pos=root_pos, h_scale=scales)
+    out = dict(hidden=hidden, lm_head=lm_head, embed=embed,
+               norm_h=torch.ones(d, dtype=dt), norm_e=torch.ones(d, dtype=dt),
+               w_gate=w_gate, w_up=w_up, w_down=w_down,
+               root_tok=root_tok, root_pos=root_pos, h_scale=scales)
+    if cfg.approx == "linear":
+        out["w_lin"] = _randn(g, (d, 2 * d), cfg.wd_std, dt)
+    return out
 
 
 def to_f64(t: torch.Tensor) -> np.ndarray:

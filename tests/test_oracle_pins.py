@@ -177,6 +177,70 @@ def test_concat_order_hidden_first():
                 np.testing.assert_allclose(delta[a], delta[b], atol=1e-12)
 
 
+def test_linear_approximator_hand_computed():
+    # "w/ Linear" ablation (Sec. 4, Table 3; reading R12): h' = h + W_lin [h~ ; e].
+    # d = 2, norm weights 1, eps = 0; h = (3, 4): RMS sqrt(12.5); e = (1, -1): RMS 1.
+    h = np.array([[3.0, 4.0]])
+    e = np.array([[1.0, -1.0]])
+    w_lin = np.array([[1.0, 0.0, 2.0, 0.0],     # out0 = x0 + 2 x2
+                      [0.0, -1.0, 0.0, 3.0]])   # out1 = -x1 + 3 x3
+    x0, x1 = 3 / math.sqrt(12.5), 4 / math.sqrt(12.5)
+    expect = np.array([[3 + x0 + 2.0, 4 - x1 - 3.0]])
+    got = O.linear_approximator(h, e, np.ones(2), np.ones(2), w_lin, 0.0)
+    np.testing.assert_allclose(got, expect, rtol=1e-14)
+
+
+def test_linear_approximator_identity_blocks():
+    # W_lin = [I | 0] adds the normalised hidden state, [0 | I] the normalised embedding:
+    # pins which half of the input is which (h~ first) against rmsnorm's closed form.
+    rng = np.random.default_rng(9)
+    d = 6
+    h, e = rng.normal(0, 2, (3, d)), rng.normal(0, 1, (3, d))
+    wh, we = rng.uniform(0.5, 1.5, d), rng.uniform(0.5, 1.5, d)
+    eye, zero = np.eye(d), np.zeros((d, d))
+    eps = 1e-6
+    rms = lambda a: np.sqrt((a * a).mean(axis=1, keepdims=True) + eps)
+    got_h = O.linear_approximator(h, e, wh, we, np.hstack([eye, zero]), eps)
+    got_e = O.linear_approximator(h, e, wh, we, np.hstack([zero, eye]), eps)
+    np.testing.assert_allclose(got_h, h + h / rms(h) * wh, rtol=1e-13)
+    np.testing.assert_allclose(got_e, h + e / rms(e) * we, rtol=1e-13)
+
+
+def test_linear_approximator_is_a_token_conditioned_bias():
+    # The paper describes the linear variant as a bias on the hidden state conditioned on the
+    # previous token: for a fixed previous token the shift h' - h - W_lin^h h~ is the same for
+    # every hidden state, and the difference between two previous tokens' h' is the same for
+    # every hidden state.
+    H, root, W = small_problem(seed=8, gamma=3)
+    d = H.shape[1]
+    W["w_lin"] = np.random.default_rng(10).normal(0, 0.3, (d, 2 * d))
+    _, ids, _ = O.stage1(H, W["lm_head"], 1.0, 4)
+    hp, lp = O.stage2(H, root, ids, W, 3, 1.0, 1e-6, approx="linear")
+    hid, prev = O.stage2_conditioning(3, 3, root, ids)
+    h_part = O.rmsnorm(H[hid], W["norm_h"], 1e-6) @ W["w_lin"][:, :d].T
+    bias = hp - H[hid] - h_part
+    e_part = O.rmsnorm(W["embed"][prev], W["norm_e"], 1e-6) @ W["w_lin"][:, d:].T
+    np.testing.assert_allclose(bias, e_part, atol=1e-12)
+    # rows of one depth share h, so they differ by their tokens' embedding terms alone
+    for a, b in ((1, 2), (2, 3), (4, 6)):
+        np.testing.assert_allclose(hp[a] - hp[b], e_part[a] - e_part[b], atol=1e-12)
+    np.testing.assert_allclose(np.exp(lp).sum(1), 1.0, rtol=1e-13)
+
+
+def test_zero_linear_approximator_reduces_to_marginal_tree():
+    # W_lin = 0 gives h' = h, so the linear variant's tree is the M-ary marginal tree
+    for seed in range(3):
+        H, root, W = small_problem(V=32, gamma=4, seed=seed)
+        W["w_lin"] = np.zeros((H.shape[1], 2 * H.shape[1]))
+        a = O.draft_sequence(H, root, 1000, W, M=3, K2=10, B=10, approx="linear")
+        b = O.draft_sequence(H, root, 1000, W, M=3, K2=10, B=10, mode="marginal_mary")
+        hid, _ = O.stage2_conditioning(4, 3, root, a.top_ids)
+        np.testing.assert_array_equal(a.h_prime, H[hid])
+        np.testing.assert_array_equal(a.tree.tok, b.tree.tok)
+        np.testing.assert_array_equal(a.tree.parent, b.tree.parent)
+        np.testing.assert_allclose(a.tree.score, b.tree.score, atol=1e-12)
+
+
 # ------------------------------------------------------------------ Part 2: tree search
 
 
