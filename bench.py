@@ -162,11 +162,14 @@ def profiled_traffic():
 
 def algorithmic_bytes(cfg):
     """Bytes a tree build must move at least: W_lm twice (stage 2 needs the global stage-1
-    top-M first, and W_lm is ~10x the L2), the three approximator matrices, the gathered
-    embedding rows and the hidden states. Outputs are ignored."""
+    top-M first, and W_lm is ~10x the L2), the approximator's matrices (the linear variant's
+    W_lin alone), the gathered embedding rows and the hidden states. Outputs are ignored."""
     e = 2 if cfg.dtype == "bf16" else 4
     lm = cfg.V * cfg.d * e
-    mlp = (2 * cfg.I * 2 * cfg.d + cfg.d * cfg.I) * e   # W_gate, W_up [I, 2d]; W_down [d, I]
+    if cfg.approx == "linear":
+        mlp = cfg.d * 2 * cfg.d * e                    # W_lin [d, 2d]
+    else:
+        mlp = (2 * cfg.I * 2 * cfg.d + cfg.d * cfg.I) * e   # W_gate, W_up [I, 2d]; W_down [d, I]
     rows = cfg.batch * cfg.R
     gathered = rows * cfg.d * e
     hidden = cfg.batch * cfg.gamma * cfg.d * e
@@ -183,7 +186,8 @@ class OracleSample:
     def __init__(self, cfg, inp):
         import synth
         self.cfg = cfg
-        self.W = {k: synth.to_f64(inp[k]) for k in ("embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down")}
+        keys = ("embed", "norm_h", "norm_e") + (("w_lin",) if cfg.approx == "linear" else ("w_gate", "w_up", "w_down"))
+        self.W = {k: synth.to_f64(inp[k]) for k in keys}
         self.lm = synth.to_f64(inp["lm_head"])
         self.H = synth.to_f64(inp["hidden"][0])
         self.root = int(inp["root_tok"][0])
@@ -198,12 +202,15 @@ class OracleSample:
         root = self.root % Vs
         hid, prev = O.stage2_conditioning(cfg.gamma, cfg.M, root, np.zeros((cfg.gamma, cfg.M), dtype=np.int64))
         t0 = time.perf_counter()
-        O.ar_approximator(self.H[hid], W["embed"][prev], W["norm_h"], W["norm_e"], W["w_gate"], W["w_up"],
-                          W["w_down"], cfg.rms_eps)
+        if cfg.approx == "linear":
+            O.linear_approximator(self.H[hid], W["embed"][prev], W["norm_h"], W["norm_e"], W["w_lin"], cfg.rms_eps)
+        else:
+            O.ar_approximator(self.H[hid], W["embed"][prev], W["norm_h"], W["norm_e"], W["w_gate"], W["w_up"],
+                              W["w_down"], cfg.rms_eps)
         t_mlp = time.perf_counter() - t0
         t0 = time.perf_counter()
         O.draft_sequence(self.H, root, 0, W, M=cfg.M, K2=cfg.K2, B=cfg.B, temperature=cfg.temperature,
-                         eps=cfg.rms_eps, mode=cfg.mode)
+                         eps=cfg.rms_eps, mode=cfg.mode, approx=cfg.approx)
         t = time.perf_counter() - t0
         full = t_mlp + max(t - t_mlp, 0.0) * cfg.V / Vs
         return t, full, Vs
@@ -246,7 +253,7 @@ def run_reference(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_tree * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": cfg.name, "batch": cfg.batch, "d": cfg.d, "V": cfg.V, "I": cfg.I,
-                       "gamma": cfg.gamma, "M": cfg.M, "K2": cfg.K2, "B": cfg.B},
+                       "gamma": cfg.gamma, "M": cfg.M, "K2": cfg.K2, "B": cfg.B, "approx": cfg.approx},
             "cpu_baseline": {"value": value, "unit": "trees/s", "cores": cores, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "trees/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -401,7 +408,7 @@ def run_gpu(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,0.02) weights, hidden states scaled to 2-4 nat marginals)",
         "config": {"workload": cfg.name, "batch": cfg.batch, "d": cfg.d, "V": cfg.V, "I": cfg.I,
-                   "gamma": cfg.gamma, "M": cfg.M, "K2": cfg.K2, "B": cfg.B, "R": cfg.R,
+                   "gamma": cfg.gamma, "M": cfg.M, "K2": cfg.K2, "B": cfg.B, "R": cfg.R, "approx": cfg.approx,
                    "l2": f"no flush: inputs larger than L2 (W_lm {lm_bytes / 1e9:.3f} GB streamed twice per step)",
                    "parallelism": f"replicas x{world}"},
         "step_roofline": {"algorithmic_bytes": step_bytes, "achieved_gbs": step_bytes / (ms_per_step / 1e3) / 1e9,

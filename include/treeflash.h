@@ -69,6 +69,14 @@ typedef enum {
                                   computes when the approximator is zero (Sec. 3 "Training") */
 } tf_mode;
 
+/* Which AR-approximator stage 2 runs (TF_MODE_AR only). */
+typedef enum {
+    TF_APPROX_SWIGLU = 0,      /* Eq. 1: h' = h + W_down (SiLU(W_gate x) * (W_up x)), x = [h~ ; e] */
+    TF_APPROX_LINEAR = 1       /* the "w/ Linear" ablation (Sec. 4 "Model Design", Table 3): the
+                                  SwiGLU replaced by one linear layer on the same input,
+                                  h' = h + W_lin x, W_lin [d, 2d], no bias */
+} tf_approx;
+
 /* Device status bits (int32 words written with atomic OR). */
 enum {
     TF_DEV_BAD_TOKEN = 1,      /* a token id outside [0, V) was read; the row/node is skipped */
@@ -91,6 +99,8 @@ typedef struct {
     float rms_eps;        /* RMSNorm epsilon of Eq. 1's normalisations */
     int32_t dtype;        /* tf_dtype */
     int32_t mode;         /* tf_mode */
+    int32_t approx;       /* tf_approx (0 = Eq. 1's SwiGLU); read only in TF_MODE_AR. With
+                             TF_APPROX_LINEAR, I is ignored */
 } tf_dims;
 
 /* Model parameters (device, dims->dtype, row-major, read only, never copied). */
@@ -102,6 +112,8 @@ typedef struct {
     const void* w_gate;   /* [I, 2d] SwiGLU gate projection, input [h~ ; e] */
     const void* w_up;     /* [I, 2d] SwiGLU up projection, input [h~ ; e] */
     const void* w_down;   /* [d, I]  SwiGLU down projection */
+    const void* w_lin;    /* [d, 2d] linear approximator, input [h~ ; e] (TF_APPROX_LINEAR only;
+                             w_gate, w_up and w_down are then not read and may be NULL) */
 } tf_weights;
 
 /* Human-readable name of a status code (static storage). */
@@ -144,6 +156,7 @@ tf_status tf_stage1_marginals(const tf_dims* dims, const tf_weights* w, const vo
  *   row 0:                 h' = h_{t+1} + SwiGLU(RMSNorm(h_{t+1}) :: RMSNorm(Embd(x_t)))
  *   row 1 + (i-2) M + m:   h' = h_{t+i} + SwiGLU(RMSNorm(h_{t+i}) :: RMSNorm(Embd(x^(m)_{t+i-1})))
  * for i = 2..gamma, m = 0..M-1, then q' = softmax(W_lm h' / T) and its K2 largest entries.
+ * With dims->approx == TF_APPROX_LINEAR, W_lin (...) takes the place of SwiGLU(...).
  *  hidden     [b, gamma, d] dtype (as in stage 1)
  *  root_tok   [b] int32: the last accepted token x_t of each sequence
  *  top_ids    [b, gamma, K1] int32: stage-1 output (the first M per depth are used)
@@ -252,7 +265,8 @@ tf_status tf_lmhead_merge(const tf_dims* dims, const void* lm_head, const void* 
                           void* ws, size_t ws_bytes, tf_stream_t stream);
 
 /* Eq. 1 on the R rows of every sequence (stage 2 before the LM head): gathers Embd rows,
- * normalises both halves, runs the SwiGLU MLP and adds the residual.
+ * normalises both halves, runs the SwiGLU MLP (or the linear layer of TF_APPROX_LINEAR) and
+ * adds the residual.
  * h_prime [b, R, d] dtype out (may be NULL: then only the workspace copy is written). */
 tf_status tf_ar_approx(const tf_dims* dims, const tf_weights* w, const void* hidden,
                        const int32_t* root_tok, const int32_t* top_ids, void* h_prime,
@@ -270,7 +284,8 @@ tf_status tf_workspace_h_prime(const tf_dims* dims, void* ws, size_t ws_bytes, v
  * Intermediates of Eq. 1 left by the last tf_ar_approx / tf_stage2_ar_approx (TF_MODE_AR only):
  *   TF_VIEW_X        x = [RMSNorm(h)*w_h ; RMSNorm(Embd(prev))*w_e]   [b*R, 2d] dtype
  *   TF_VIEW_A        SiLU(W_gate x) * (W_up x)                         [b*R, I]  dtype
- *   TF_VIEW_H_PRIME  h' = h + W_down A                                 [b*R, d]  dtype
+ *                    (0 bytes with TF_APPROX_LINEAR)
+ *   TF_VIEW_H_PRIME  h' = h + W_down A  (or h + W_lin x)               [b*R, d]  dtype
  * The partials of the last tf_lmhead_partials over n_rows rows, n_tiles = ceil(V / 256), both
  * float4 tables indexed [block][part][row] with the call's n_rows as the row count:
  *   TF_VIEW_HALVES   [n_tiles][2][n_rows] per half block (128 entries): (max logit m,

@@ -44,10 +44,10 @@ exp/log. Readings of points the paper leaves open (each also listed in the desig
       node expandable, Sec. 4 "Baselines"); "marginal_mary" is the same search restricted
       by the M-ary rule of Sec. 3 (what TreeFlash reduces to with a zeroed approximator).
   R12 The "w/ Linear" ablation (Sec. 4 "Model Design", Table 3) replaces the SwiGLU of
-      Eq. 1 by one linear layer on the same input: h' = h + W_lin (h~ :: e), W_lin [d, 2d],
-      no bias term. The token-dependent part of h' is then W_lin's embedding half applied
-      to e, the same for every hidden state: the "bias conditioned on the previous token"
-      the paper describes.
+      Eq. 1 by one linear map on the same input: h' = h + W_lin (h~ :: e), W_lin [d, 2d],
+      no bias vector. The token-dependent part of h' is then W_lin's embedding half applied
+      to e, the same for every hidden state: the token-dependent offset of the hidden state
+      that Sec. 4 attributes to this variant.
 
 Optional bf16 emulation (`emulate_bf16=True`) rounds to bfloat16 (round to nearest even)
 exactly where a bf16 implementation stores intermediates: the RMSNorm outputs, SiLU(G)*U,

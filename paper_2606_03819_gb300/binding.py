@@ -22,6 +22,7 @@ TF_OK, TF_ERR_INVALID_ARG, TF_ERR_UNSUPPORTED, TF_ERR_WORKSPACE, TF_ERR_CUDA, TF
     TF_ERR_TIMEOUT = range(7)
 TF_BF16, TF_F32 = 0, 1
 MODES = {"ar": 0, "marginal": 1, "marginal_mary": 2}
+APPROX = {"swiglu": 0, "linear": 1}
 TF_DEV_BAD_TOKEN, TF_DEV_UNDERFULL, TF_DEV_NONFINITE, TF_DEV_TIMEOUT, TF_DEV_RECOMPUTED = 1, 2, 4, 8, 16
 
 
@@ -35,12 +36,13 @@ class TfDims(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int32), ("d", ctypes.c_int32), ("V", ctypes.c_int32),
                 ("I", ctypes.c_int32), ("gamma", ctypes.c_int32), ("M", ctypes.c_int32),
                 ("K2", ctypes.c_int32), ("B", ctypes.c_int32), ("temperature", ctypes.c_float),
-                ("rms_eps", ctypes.c_float), ("dtype", ctypes.c_int32), ("mode", ctypes.c_int32)]
+                ("rms_eps", ctypes.c_float), ("dtype", ctypes.c_int32), ("mode", ctypes.c_int32),
+                ("approx", ctypes.c_int32)]
 
 
 class TfWeights(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in
-                ("lm_head", "embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down")]
+                ("lm_head", "embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down", "w_lin")]
 
 
 EXPORTS = ("tf_status_string", "tf_version", "tf_kernel_launches", "tf_workspace_size", "tf_status_reset", "tf_status_read",
@@ -112,6 +114,7 @@ class Dims:
     rms_eps: float = 1e-6
     dtype: str = "bf16"
     mode: str = "ar"
+    approx: str = "swiglu"      # "swiglu" (Eq. 1) or "linear" (the "w/ Linear" ablation)
 
     @property
     def R(self) -> int:
@@ -128,15 +131,15 @@ class Dims:
     def c(self) -> TfDims:
         return TfDims(self.batch, self.d, self.V, self.I, self.gamma, self.M, self.K2, self.B,
                       self.temperature, self.rms_eps, TF_BF16 if self.dtype == "bf16" else TF_F32,
-                      MODES[self.mode])
+                      MODES[self.mode], APPROX[self.approx])
 
     @classmethod
     def from_config(cls, cfg) -> "Dims":
         return cls(cfg.batch, cfg.d, cfg.V, cfg.I, cfg.gamma, cfg.M, cfg.K2, cfg.B, cfg.temperature,
-                   cfg.rms_eps, cfg.dtype, cfg.mode)
+                   cfg.rms_eps, cfg.dtype, cfg.mode, getattr(cfg, "approx", "swiglu"))
 
 
-WEIGHT_KEYS = ("lm_head", "embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down")
+WEIGHT_KEYS = ("lm_head", "embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down", "w_lin")
 
 
 def _ptr(t: Optional[torch.Tensor]):

@@ -28,7 +28,7 @@ constexpr size_t kMaxMergeSmem = 220 * 1024;
 size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Dims {
-    int b, d, V, I, gamma, M, K2, B, K1, R, dtype, mode, n_tiles;
+    int b, d, V, I, gamma, M, K2, B, K1, R, dtype, mode, approx, n_tiles;
     size_t esize;
     float inv_temp, eps;
 };
@@ -48,13 +48,16 @@ tf_status check_dims(const tf_dims* dims, Dims* o) {
     if (d.dtype != TF_BF16 && d.dtype != TF_F32) return TF_ERR_INVALID_ARG;
     if (d.mode != TF_MODE_AR && d.mode != TF_MODE_MARGINAL && d.mode != TF_MODE_MARGINAL_MARY)
         return TF_ERR_INVALID_ARG;
+    if (d.mode == TF_MODE_AR && d.approx != TF_APPROX_SWIGLU && d.approx != TF_APPROX_LINEAR)
+        return TF_ERR_INVALID_ARG;
+    const bool swiglu = d.mode == TF_MODE_AR && d.approx == TF_APPROX_SWIGLU;
     if (!(d.temperature > 0.0f) || !isfinite(d.temperature)) return TF_ERR_INVALID_ARG;
     if (!(d.rms_eps >= 0.0f) || !isfinite(d.rms_eps)) return TF_ERR_INVALID_ARG;
     const int K1 = d.M > d.K2 ? d.M : d.K2;
     if (K1 > d.V) return TF_ERR_INVALID_ARG;
-    if (d.mode == TF_MODE_AR && d.I < 1) return TF_ERR_INVALID_ARG;
+    if (swiglu && d.I < 1) return TF_ERR_INVALID_ARG;
     if (d.gamma > kMaxGamma || d.M > kMaxM || d.K2 > kMaxK || d.B > kMaxB) return TF_ERR_UNSUPPORTED;
-    if (d.dtype == TF_BF16 && (d.d % 64 != 0 || (d.mode == TF_MODE_AR && d.I % 64 != 0)))
+    if (d.dtype == TF_BF16 && (d.d % 64 != 0 || (swiglu && d.I % 64 != 0)))
         return TF_ERR_UNSUPPORTED;
     const int n_tiles = (d.V + kBlockV - 1) / kBlockV;
     if (merge_smem_bytes(n_tiles, d.d, K1) > kMaxMergeSmem) return TF_ERR_UNSUPPORTED;
@@ -64,7 +67,7 @@ tf_status check_dims(const tf_dims* dims, Dims* o) {
     o->b = d.batch;
     o->d = d.d;
     o->V = d.V;
-    o->I = d.mode == TF_MODE_AR ? d.I : 0;
+    o->I = swiglu ? d.I : 0;   // no SwiGLU intermediate otherwise
     o->gamma = d.gamma;
     o->M = d.M;
     o->K2 = d.K2;
@@ -73,6 +76,7 @@ tf_status check_dims(const tf_dims* dims, Dims* o) {
     o->R = static_cast<int>(R);
     o->dtype = d.dtype;
     o->mode = d.mode;
+    o->approx = d.mode == TF_MODE_AR ? d.approx : TF_APPROX_SWIGLU;
     o->n_tiles = n_tiles;
     o->esize = d.dtype == TF_BF16 ? 2 : 4;
     o->inv_temp = 1.0f / d.temperature;
@@ -184,6 +188,12 @@ tf_status do_ar_approx(const Ctx& ctx, const Dims& D, const Layout& L, void* ws,
     TF_TRY(cuda_status(launch_gather_norm(ctx, D.dtype, hidden, w->embed, w->norm_h, w->norm_e, root_tok, top_ids,
                                           D.b, D.gamma, D.M, D.K1, D.d, D.V, D.eps, X)));
     const int rows = D.b * D.R;
+    if (D.approx == TF_APPROX_LINEAR) {
+        if (D.dtype == TF_BF16)
+            return cuda_status(launch_linear_tc(ctx, X, w->w_lin, hidden, rows, D.d, D.R, D.M, D.gamma, hp,
+                                                at<float>(ws, L.kpart)));
+        return cuda_status(launch_linear_simt(ctx, X, w->w_lin, hidden, rows, D.d, D.R, D.M, D.gamma, hp));
+    }
     if (D.dtype == TF_BF16)
         return cuda_status(launch_swiglu_tc(ctx, X, w->w_gate, w->w_up, w->w_down, hidden, rows, D.d, D.I, D.R, D.M,
                                             D.gamma, A, hp, at<float>(ws, L.kpart)));
@@ -193,10 +203,10 @@ tf_status do_ar_approx(const Ctx& ctx, const Dims& D, const Layout& L, void* ws,
 
 tf_status check_weights(const Dims& D, const tf_weights* w, bool need_mlp) {
     if (!w || !aligned16(w->lm_head)) return TF_ERR_INVALID_ARG;
-    if (need_mlp && (!aligned16(w->embed) || !aligned16(w->norm_h) || !aligned16(w->norm_e) ||
-                     !aligned16(w->w_gate) || !aligned16(w->w_up) || !aligned16(w->w_down)))
-        return TF_ERR_INVALID_ARG;
-    (void)D;
+    if (!need_mlp) return TF_OK;
+    if (!aligned16(w->embed) || !aligned16(w->norm_h) || !aligned16(w->norm_e)) return TF_ERR_INVALID_ARG;
+    if (D.approx == TF_APPROX_LINEAR) return aligned16(w->w_lin) ? TF_OK : TF_ERR_INVALID_ARG;
+    if (!aligned16(w->w_gate) || !aligned16(w->w_up) || !aligned16(w->w_down)) return TF_ERR_INVALID_ARG;
     return TF_OK;
 }
 
@@ -206,10 +216,15 @@ struct Prepared {
     Ctx ctx;
 };
 
-tf_status prepare(const tf_dims* dims, void* ws, size_t ws_bytes, tf_stream_t stream, Prepared* p) {
+// Host-side checks of dims and workspace (no CUDA call), then the launch context.
+tf_status validate(const tf_dims* dims, void* ws, size_t ws_bytes, Prepared* p) {
     TF_TRY(check_dims(dims, &p->D));
     p->L = layout(p->D);
-    TF_TRY(check_ws(p->L, ws, ws_bytes));
+    return check_ws(p->L, ws, ws_bytes);
+}
+
+tf_status prepare(const tf_dims* dims, void* ws, size_t ws_bytes, tf_stream_t stream, Prepared* p) {
+    TF_TRY(validate(dims, ws, ws_bytes, p));
     return make_ctx(ws, p->L, stream, &p->ctx);
 }
 
@@ -284,9 +299,10 @@ tf_status tf_lmhead_merge(const tf_dims* dims, const void* lm_head, const void* 
 tf_status tf_stage1_marginals(const tf_dims* dims, const tf_weights* w, const void* hidden, int32_t* top_ids,
                               float* top_logp, void* ws, size_t ws_bytes, tf_stream_t stream) {
     Prepared p;
-    TF_TRY(prepare(dims, ws, ws_bytes, stream, &p));
+    TF_TRY(validate(dims, ws, ws_bytes, &p));
     TF_TRY(check_weights(p.D, w, false));
     if (!aligned16(hidden) || !top_ids || !top_logp) return TF_ERR_INVALID_ARG;
+    TF_TRY(make_ctx(ws, p.L, stream, &p.ctx));
     const int rows = p.D.b * p.D.gamma;
     TF_TRY(do_partials(p.ctx, p.D, p.L, ws, w->lm_head, hidden, rows, /*reset_status=*/true));
     return do_merge(p.ctx, p.D, p.L, ws, w->lm_head, hidden, rows, p.D.K1, top_ids, top_logp);
@@ -295,10 +311,11 @@ tf_status tf_stage1_marginals(const tf_dims* dims, const tf_weights* w, const vo
 tf_status tf_ar_approx(const tf_dims* dims, const tf_weights* w, const void* hidden, const int32_t* root_tok,
                        const int32_t* top_ids, void* h_prime, void* ws, size_t ws_bytes, tf_stream_t stream) {
     Prepared p;
-    TF_TRY(prepare(dims, ws, ws_bytes, stream, &p));
+    TF_TRY(validate(dims, ws, ws_bytes, &p));
     if (p.D.mode != TF_MODE_AR) return TF_ERR_INVALID_ARG;
     TF_TRY(check_weights(p.D, w, true));
     if (!aligned16(hidden) || !root_tok || !top_ids) return TF_ERR_INVALID_ARG;
+    TF_TRY(make_ctx(ws, p.L, stream, &p.ctx));
     TF_TRY(do_ar_approx(p.ctx, p.D, p.L, ws, w, hidden, root_tok, top_ids));
     if (h_prime) {
         const size_t bytes = static_cast<size_t>(p.D.b) * p.D.R * p.D.d * p.D.esize;
@@ -312,10 +329,11 @@ tf_status tf_stage2_ar_approx(const tf_dims* dims, const tf_weights* w, const vo
                               const int32_t* top_ids, int32_t* child_ids, float* child_logp, void* ws,
                               size_t ws_bytes, tf_stream_t stream) {
     Prepared p;
-    TF_TRY(prepare(dims, ws, ws_bytes, stream, &p));
+    TF_TRY(validate(dims, ws, ws_bytes, &p));
     if (p.D.mode != TF_MODE_AR) return TF_ERR_INVALID_ARG;
     TF_TRY(check_weights(p.D, w, true));
     if (!aligned16(hidden) || !root_tok || !top_ids || !child_ids || !child_logp) return TF_ERR_INVALID_ARG;
+    TF_TRY(make_ctx(ws, p.L, stream, &p.ctx));
     TF_TRY(do_ar_approx(p.ctx, p.D, p.L, ws, w, hidden, root_tok, top_ids));
     const int rows = p.D.b * p.D.R;
     const void* hp = at<void>(ws, p.L.hp);

@@ -177,6 +177,12 @@ cudaError_t launch_down_reduce(const Ctx&, const float* partial, int k_splits, i
 cudaError_t launch_swiglu_simt(const Ctx&, const void* X, const void* w_gate, const void* w_up,
                                const void* w_down, const void* hidden, int n_rows, int d, int I,
                                int R, int M, int gamma, void* A, void* h_prime);
+// the "w/ Linear" approximator: h' = h + X W_lin^T, X [n_rows, 2d], W_lin [d, 2d]
+cudaError_t launch_linear_tc(const Ctx&, const void* X, const void* w_lin, const void* hidden,
+                             int n_rows, int d, int R, int M, int gamma, void* h_prime,
+                             float* partial);
+cudaError_t launch_linear_simt(const Ctx&, const void* X, const void* w_lin, const void* hidden,
+                               int n_rows, int d, int R, int M, int gamma, void* h_prime);
 // Part 2 and the mask
 cudaError_t launch_build_tree(const Ctx&, int b, int gamma, int M, int K1, int K2, int B, int V,
                               int mode, int R, const int32_t* root_tok, const int32_t* top_ids,

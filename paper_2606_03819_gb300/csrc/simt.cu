@@ -213,4 +213,16 @@ cudaError_t launch_swiglu_simt(const Ctx& ctx, const void* X, const void* w_gate
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+// The "w/ Linear" approximator: the residual GEMM above with x (K = 2d) in place of A.
+cudaError_t launch_linear_simt(const Ctx& ctx, const void* X, const void* w_lin, const void* hidden, int n_rows, int d,
+                               int R, int M, int gamma, void* h_prime) {
+    if (n_rows <= 0) return cudaSuccess;
+    dim3 grid((d + 63) / 64, (n_rows + 63) / 64);
+    const cudaError_t e = launch_pdl(swiglu_simt_kernel<false>, grid, dim3(256), 0, ctx.stream,
+                                     static_cast<const float*>(X), static_cast<const float*>(w_lin),
+                                     static_cast<const float*>(nullptr), n_rows, 2 * d, d,
+                                     static_cast<float*>(h_prime), static_cast<const float*>(hidden), R, M, gamma);
+    return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 }  // namespace tf

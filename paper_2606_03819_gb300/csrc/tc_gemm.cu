@@ -10,7 +10,8 @@
 //           best (z, id), and per 32-wide chunk the three largest z with the ids of the first
 //           two. Logits never leave the SM.
 //   GATEUP  SwiGLU of Eq. 1, first half: A = SiLU(X W_gate^T) * (X W_up^T), bf16 out.
-//   DOWN    SwiGLU of Eq. 1, second half plus the residual: h' = h + A W_down^T, bf16 out.
+//   DOWN    SwiGLU of Eq. 1, second half plus the residual: h' = h + A W_down^T, bf16 out; the
+//           same epilogue serves the linear approximator of the ablations, h' = h + x W_lin^T.
 //
 // Warp roles (576 threads, one CTA per SM, persistent over work units):
 //   warp 0      TMA producer: one elected lane streams X and W tiles into a ring of stages.
@@ -771,6 +772,48 @@ int choose_k_splits(int base_units, int nk, int num_sms) {
     return ks < 1 ? 1 : ks;
 }
 
+// h' = h + In W^T with In [n_rows, K] (tmap_in, boxes of kBK x kBM) and W [d, K] (tmap_w, boxes of
+// kBK x BN, BN = 128 when d % 128 == 0, else 64): the SwiGLU down projection (K = I, In = A) and
+// the linear approximator (K = 2d, In = x). The residual row of stage-2 row r is the hidden state
+// of its depth; the epilogue adds it in fp32 and rounds once to bf16.
+static cudaError_t run_residual_gemm(const Ctx& ctx, const CUtensorMap& ta, const CUtensorMap& td, int K, const void* hidden,
+                              int n_rows, int d, int R, int M, int gamma, void* h_prime, float* partial) {
+    constexpr int BN = 128;
+    const int m_tiles = (n_rows + kBM - 1) / kBM;
+    const int n_mg = m_tiles == 1 ? 1 : (m_tiles + 1) / 2;
+    const int bn_d = d % BN == 0 ? BN : 64;
+    const int ks2 = choose_k_splits((d / bn_d) * n_mg, K / kBK, ctx.num_sms);
+    EpiParams ed{};
+    ed.out = static_cast<__nv_bfloat16*>(h_prime);
+    ed.ld_out = d;
+    ed.hidden = static_cast<const __nv_bfloat16*>(hidden);
+    ed.R = R;
+    ed.M = M;
+    ed.gamma = gamma;
+    ed.partial = partial;
+    ed.n_cols = d;
+    ed.n_total = d;
+    if (ks2 == 1) {
+        if (bn_d == BN)
+            return m_tiles == 1 ? run_gemm<EPI_DOWN, 1, 1, BN, 6>(ctx, ta, td, td, n_rows, K, d / BN, 1, ed)
+                                : run_gemm<EPI_DOWN, 2, 1, BN, 4>(ctx, ta, td, td, n_rows, K, d / BN, n_mg, ed);
+        return m_tiles == 1 ? run_gemm<EPI_DOWN, 1, 1, 64, 8>(ctx, ta, td, td, n_rows, K, d / 64, 1, ed)
+                            : run_gemm<EPI_DOWN, 2, 1, 64, 5>(ctx, ta, td, td, n_rows, K, d / 64, n_mg, ed);
+    }
+    if (m_tiles == 2 && bn_d == BN && ks2 == 4 && splitk_clusters_fit<EPI_CDOWN, 2, 1, BN, 4, 4>(ctx, d / BN))
+        return run_gemm<EPI_CDOWN, 2, 1, BN, 4, 4>(ctx, ta, td, td, n_rows, K, d / BN, 1, ed, 4);
+    cudaError_t e;
+    if (bn_d == BN)
+        e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 1, BN, 6>(ctx, ta, td, td, n_rows, K, d / BN, 1, ed, ks2)
+                         : run_gemm<EPI_PARTIAL, 2, 1, BN, 4>(ctx, ta, td, td, n_rows, K, d / BN, n_mg, ed, ks2);
+    else
+        e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 1, 64, 8>(ctx, ta, td, td, n_rows, K, d / 64, 1, ed, ks2)
+                         : run_gemm<EPI_PARTIAL, 2, 1, 64, 5>(ctx, ta, td, td, n_rows, K, d / 64, n_mg, ed, ks2);
+    if (e != cudaSuccess) return e;
+    return launch_down_reduce(ctx, partial, ks2, n_rows, d, static_cast<const __nv_bfloat16*>(hidden), R, M, gamma,
+                              static_cast<__nv_bfloat16*>(h_prime));
+}
+
 cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, const void* w_gate, const void* w_up,
                              const void* w_down, const void* hidden, int n_rows, int d, int I, int R, int M,
                              int gamma, void* A, void* h_prime, float* partial) {
@@ -821,35 +864,18 @@ cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, const void* w_gate, 
     }
 
     // ---- down + residual: h' = h + A Wd^T
-    const int ks2 = choose_k_splits((d / bn_d) * n_mg, I / kBK, ctx.num_sms);
-    EpiParams ed{};
-    ed.out = static_cast<__nv_bfloat16*>(h_prime);
-    ed.ld_out = d;
-    ed.hidden = static_cast<const __nv_bfloat16*>(hidden);
-    ed.R = R;
-    ed.M = M;
-    ed.gamma = gamma;
-    ed.partial = partial;
-    ed.n_cols = d;
-    ed.n_total = d;
-    if (ks2 == 1) {
-        if (bn_d == BN)
-            return m_tiles == 1 ? run_gemm<EPI_DOWN, 1, 1, BN, 6>(ctx, ta, td, td, n_rows, I, d / BN, 1, ed)
-                                : run_gemm<EPI_DOWN, 2, 1, BN, 4>(ctx, ta, td, td, n_rows, I, d / BN, n_mg, ed);
-        return m_tiles == 1 ? run_gemm<EPI_DOWN, 1, 1, 64, 8>(ctx, ta, td, td, n_rows, I, d / 64, 1, ed)
-                            : run_gemm<EPI_DOWN, 2, 1, 64, 5>(ctx, ta, td, td, n_rows, I, d / 64, n_mg, ed);
-    }
-    if (m_tiles == 2 && bn_d == BN && ks2 == 4 && splitk_clusters_fit<EPI_CDOWN, 2, 1, BN, 4, 4>(ctx, d / BN))
-        return run_gemm<EPI_CDOWN, 2, 1, BN, 4, 4>(ctx, ta, td, td, n_rows, I, d / BN, 1, ed, 4);
-    if (bn_d == BN)
-        e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 1, BN, 6>(ctx, ta, td, td, n_rows, I, d / BN, 1, ed, ks2)
-                         : run_gemm<EPI_PARTIAL, 2, 1, BN, 4>(ctx, ta, td, td, n_rows, I, d / BN, n_mg, ed, ks2);
-    else
-        e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 1, 64, 8>(ctx, ta, td, td, n_rows, I, d / 64, 1, ed, ks2)
-                         : run_gemm<EPI_PARTIAL, 2, 1, 64, 5>(ctx, ta, td, td, n_rows, I, d / 64, n_mg, ed, ks2);
+    return run_residual_gemm(ctx, ta, td, I, hidden, n_rows, d, R, M, gamma, h_prime, partial);
+}
+
+cudaError_t launch_linear_tc(const Ctx& ctx, const void* X, const void* w_lin, const void* hidden, int n_rows, int d,
+                             int R, int M, int gamma, void* h_prime, float* partial) {
+    if (n_rows <= 0) return cudaSuccess;
+    const int bn = d % 128 == 0 ? 128 : 64;
+    CUtensorMap tx, tw;
+    cudaError_t e = make_tmap(&tx, X, 2 * d, n_rows, kBK, kBM);
+    if (e == cudaSuccess) e = make_tmap(&tw, w_lin, 2 * d, d, kBK, bn);
     if (e != cudaSuccess) return e;
-    return launch_down_reduce(ctx, partial, ks2, n_rows, d, static_cast<const __nv_bfloat16*>(hidden), R, M, gamma,
-                              static_cast<__nv_bfloat16*>(h_prime));
+    return run_residual_gemm(ctx, tx, tw, 2 * d, hidden, n_rows, d, R, M, gamma, h_prime, partial);
 }
 
 }  // namespace tf

@@ -118,3 +118,51 @@ def test_binding_signatures_match_header_arity(lib):
     assert set(arity) == set(declared_functions())
     for name, n in arity.items():
         assert len(getattr(lib, name).argtypes) == n, name
+
+
+def _header_struct_fields(name):
+    src = open(os.path.join(ROOT, "include", "treeflash.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    body = re.search(r"typedef struct \{([^}]*)\}\s*" + name + r"\s*;", src).group(1)
+    return re.findall(r"(\w+)\s*;", body)
+
+
+def test_binding_structs_match_header_layout():
+    # the ctypes structs must list the header's fields in the header's order (the struct is
+    # passed by pointer, so a missing or reordered field would shift every later one)
+    from paper_2606_03819_gb300 import binding as Bn
+    assert [f for f, _ in Bn.TfDims._fields_] == _header_struct_fields("tf_dims")
+    assert [f for f, _ in Bn.TfWeights._fields_] == _header_struct_fields("tf_weights")
+    assert ctypes.sizeof(Bn.TfDims) == 4 * len(Bn.TfDims._fields_)
+
+
+def test_approximator_kind_validation(lib):
+    from paper_2606_03819_gb300 import binding as Bn
+    # the linear approximator has no intermediate width: I is ignored, also its bf16 alignment
+    assert Bn.tf_workspace_size(_dims(approx="linear", I=0)) > 0
+    assert Bn.tf_workspace_size(_dims(approx="linear", I=100, dtype="bf16")) > 0
+    # it needs no A buffer, so its workspace is smaller than the SwiGLU one of the same shape
+    assert Bn.tf_workspace_size(_dims(approx="linear")) < Bn.tf_workspace_size(_dims())
+    # an unknown kind is rejected in TreeFlash mode and ignored by the marginal modes
+    c = _dims().c()
+    c.approx = 7
+    n = ctypes.c_size_t()
+    assert lib.tf_workspace_size(ctypes.byref(c), ctypes.byref(n)) == Bn.TF_ERR_INVALID_ARG
+    c.mode = Bn.MODES["marginal"]
+    assert lib.tf_workspace_size(ctypes.byref(c), ctypes.byref(n)) == Bn.TF_OK
+
+
+def test_linear_approximator_needs_w_lin_not_the_swiglu_weights(lib):
+    # host-side weight checks run before any GPU work: a null w_lin is rejected for the linear
+    # approximator, null SwiGLU weights for the SwiGLU one (argument order: dims, weights,
+    # hidden, root_tok, top_ids, h_prime, ws, ws_bytes, stream)
+    from paper_2606_03819_gb300 import binding as Bn
+    buf = ctypes.create_string_buffer(1 << 16)
+    fake = ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 256   # aligned, never dereferenced
+    for approx, missing in (("linear", "w_lin"), ("swiglu", "w_down")):
+        d = _dims(approx=approx)
+        c = d.c()
+        w = Bn.TfWeights(*[None if k == missing else fake for k in Bn.WEIGHT_KEYS])
+        ws_bytes = Bn.tf_workspace_size(d)
+        st = lib.tf_ar_approx(ctypes.byref(c), ctypes.byref(w), fake, fake, fake, None, fake, ws_bytes, None)
+        assert st == Bn.TF_ERR_INVALID_ARG, approx

@@ -210,6 +210,43 @@ def test_underfull_universe_is_flagged():
     np.testing.assert_array_equal(gpu["node_tok"][0], orc[0].tree.tok)
 
 
+# ------------------------------------------------------------------ "w/ Linear" approximator
+# (Sec. 4 "Model Design", Table 3): h' = h + W_lin [h~ ; e]. The same gather and normalisation,
+# then one residual GEMM with K = 2d (fp32: the CUDA-core kernel; bf16: the tcgen05 kernel, with
+# split-K over 4-CTA clusters for 129..256 rows).
+
+
+def test_fp32_linear_approximator():
+    _, reps = check(synth.get_config("tiny_peaked", approx="linear"))
+    print(reps)
+
+
+@pytest.mark.parametrize("b,V,gamma,M,K2,B", [BF16_SMALL[0], BF16_SMALL[1], BF16_SMALL[2]])
+def test_bf16_linear_approximator_small(b, V, gamma, M, K2, B):
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=b, V=V, gamma=gamma, M=M, K2=K2, B=B,
+                           approx="linear")
+    _, reps = check(cfg)
+    print(reps)
+
+
+def test_bf16_linear_approximator_cluster_split_k():
+    # 241 rows (two M-tiles), d = 512: K = 2d = 1024 split over the 4 CTAs of each cluster
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=1, d=512, V=3000, gamma=16, M=16, K2=16,
+                           B=32, approx="linear")
+    check(cfg)
+
+
+def test_bf16_zero_linear_approximator_equals_mary_marginal_tree():
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=4, V=2000, approx="linear")
+    inp = synth.make_inputs(cfg)
+    inp["w_lin"].zero_()
+    d = parity.device_inputs(inp)
+    a = parity.run_gpu(cfg, d)
+    b = parity.run_gpu(cfg.replace(mode="marginal_mary"), d)
+    for k in ("node_tok", "node_parent", "node_depth", "node_score", "mask", "pos_ids"):
+        np.testing.assert_array_equal(a[k], b[k], err_msg=k)
+
+
 # ------------------------------------------------------------------ full sizes (the measured shapes)
 
 _cache = {}
@@ -222,7 +259,7 @@ def _inputs(name):
     return _cache[name]
 
 
-@pytest.mark.parametrize("name", ["q8_b64", "q8_b32"])
+@pytest.mark.parametrize("name", ["q8_b64", "q8_b32", "q8_b64_linear"])
 def test_full_size_qwen3_8b_shape(name):
     cfg = synth.get_config(name)
     gpu, reps = check(cfg, inp=_inputs(name))

@@ -207,10 +207,9 @@ def test_linear_approximator_identity_blocks():
 
 
 def test_linear_approximator_is_a_token_conditioned_bias():
-    # The paper describes the linear variant as a bias on the hidden state conditioned on the
-    # previous token: for a fixed previous token the shift h' - h - W_lin^h h~ is the same for
-    # every hidden state, and the difference between two previous tokens' h' is the same for
-    # every hidden state.
+    # Sec. 4 characterises the linear variant as a token-dependent offset added to the hidden
+    # state: h' - h - W_lin^h h~ depends on the previous token alone (W_lin^e e), whatever the
+    # hidden state, so rows of one depth differ by their tokens' offsets.
     H, root, W = small_problem(seed=8, gamma=3)
     d = H.shape[1]
     W["w_lin"] = np.random.default_rng(10).normal(0, 0.3, (d, 2 * d))
