@@ -48,6 +48,16 @@ exp/log. Readings of points the paper leaves open (each also listed in the desig
       no bias vector. The token-dependent part of h' is then W_lin's embedding half applied
       to e, the same for every hidden state: the token-dependent offset of the hidden state
       that Sec. 4 attributes to this variant.
+  R13 The "w/ 2-prev" ablation (Sec. 4 "Model Design", Table 3) conditions on the two
+      previous tokens: x = [h~ ; e(x_{t+i-1}) ; e(x_{t+i-2})] in R^{3d} (both embeddings
+      normalised with the one input-embedding norm weight), W_gate, W_up [I, 3d]. Depth 1
+      conditions on (x_t, x_{t-1}), so the step also takes the token before the root. The
+      M-ary tree then needs one row per pair of candidates: row 0 for depth 1, rows 1..M
+      for depth 2 (candidate m of depth 1, x_t), and row 1 + M + (i-3) M^2 + m1 M + m2 for
+      depth i >= 3 (candidate m1 of depth i-1, candidate m2 of depth i-2): 1 + M + M^2
+      (gamma - 2) rows. A popped node of depth i whose token is candidate m of depth i and
+      whose parent's token is candidate m' of depth i-1 gets the children of row
+      (i+1, m, m'); its parent is in the M-ary tree because it was expanded.
 
 Optional bf16 emulation (`emulate_bf16=True`) rounds to bfloat16 (round to nearest even)
 exactly where a bf16 implementation stores intermediates: the RMSNorm outputs, SiLU(G)*U,
@@ -135,11 +145,15 @@ def stage2_conditioning(gamma: int, M: int, root_tok: int, top_ids: np.ndarray):
 
 def ar_approximator(h: np.ndarray, e_raw: np.ndarray, norm_h: np.ndarray, norm_e: np.ndarray,
                     w_gate: np.ndarray, w_up: np.ndarray, w_down: np.ndarray, eps: float,
-                    emulate_bf16: bool = False) -> np.ndarray:
+                    emulate_bf16: bool = False, e2_raw: Optional[np.ndarray] = None) -> np.ndarray:
     """Eq. 1 on a batch of rows: h' = h + SwiGLU(h~ :: e) with h~ = RMSNorm(h) * norm_h and
-    e = RMSNorm(E[prev]) * norm_e (readings R1, R3). h, e_raw: [rows, d]."""
+    e = RMSNorm(E[prev]) * norm_e (readings R1, R3). h, e_raw: [rows, d]. With e2_raw (the
+    embeddings of the token before prev, reading R13) the input is h~ :: e :: e2."""
     rnd = bf16_round if emulate_bf16 else (lambda a: a)
-    x = np.concatenate([rnd(rmsnorm(h, norm_h, eps)), rnd(rmsnorm(e_raw, norm_e, eps))], axis=1)
+    parts = [rnd(rmsnorm(h, norm_h, eps)), rnd(rmsnorm(e_raw, norm_e, eps))]
+    if e2_raw is not None:
+        parts.append(rnd(rmsnorm(e2_raw, norm_e, eps)))
+    x = np.concatenate(parts, axis=1)
     a = rnd(silu(x @ w_gate.T) * (x @ w_up.T))
     return rnd(h + a @ w_down.T)
 
@@ -153,11 +167,45 @@ def linear_approximator(h: np.ndarray, e_raw: np.ndarray, norm_h: np.ndarray, no
     return rnd(h + x @ w_lin.T)
 
 
+def stage2_rows(gamma: int, M: int, approx: str = "swiglu") -> int:
+    """Stage-2 rows of one sequence (readings R4, R13)."""
+    if approx == "swiglu_2prev":
+        return 1 if gamma == 1 else 1 + M + M * M * (gamma - 2)
+    return 1 + M * (gamma - 1)
+
+
+def stage2_conditioning_2prev(gamma: int, M: int, root_tok: int, root_prev: int, top_ids: np.ndarray):
+    """Reading R13: for each stage-2 row, (index of the hidden state it refines, previous
+    token, the token before that)."""
+    hid, p1, p2 = [0], [int(root_tok)], [int(root_prev)]
+    if gamma >= 2:
+        for m in range(M):
+            hid.append(1)
+            p1.append(int(top_ids[0, m]))
+            p2.append(int(root_tok))
+    for i in range(3, gamma + 1):
+        for m1 in range(M):
+            for m2 in range(M):
+                hid.append(i - 1)
+                p1.append(int(top_ids[i - 2, m1]))
+                p2.append(int(top_ids[i - 3, m2]))
+    return (np.array(hid, dtype=np.int64), np.array(p1, dtype=np.int64), np.array(p2, dtype=np.int64))
+
+
 def stage2(H: np.ndarray, root_tok: int, top_ids: np.ndarray, W: dict, M: int,
-           temperature: float, eps: float, emulate_bf16: bool = False, approx: str = "swiglu"):
+           temperature: float, eps: float, emulate_bf16: bool = False, approx: str = "swiglu",
+           root_prev: Optional[int] = None):
     """Stage 2 for one sequence: returns (h_prime [R, d], logp [R, V]). approx: "swiglu"
-    (Eq. 1) or "linear" (reading R12)."""
+    (Eq. 1), "linear" (reading R12) or "swiglu_2prev" (reading R13, which also needs the
+    token before the root, root_prev)."""
     gamma = H.shape[0]
+    if approx == "swiglu_2prev":
+        if root_prev is None:
+            raise ValueError("the two-previous-token approximator needs root_prev")
+        hid, p1, p2 = stage2_conditioning_2prev(gamma, M, root_tok, root_prev, top_ids)
+        hp = ar_approximator(H[hid], W["embed"][p1], W["norm_h"], W["norm_e"], W["w_gate"], W["w_up"],
+                             W["w_down"], eps, emulate_bf16, e2_raw=W["embed"][p2])
+        return hp, log_softmax(lm_head(hp, W["lm_head"], temperature))
     hid, prev = stage2_conditioning(gamma, M, root_tok, top_ids)
     if approx == "swiglu":
         hp = ar_approximator(H[hid], W["embed"][prev], W["norm_h"], W["norm_e"],
@@ -191,11 +239,13 @@ class ChildSource:
     'if v = x^(m)_{t+i}' step, and reading R10 for the marginal baselines).
 
     rows: list of 1-D log-probability arrays (distributions); root_row: index of the
-    distribution of the root's children; child_row(depth, tok) -> index or None."""
+    distribution of the root's children; child_row(depth, tok, parent_tok) -> index or None
+    (parent_tok, the token of the node's parent, matters only for reading R13)."""
 
     def __init__(self, mode: str, gamma: int, M: int, stage1_top_ids: np.ndarray,
-                 stage1_logp: np.ndarray, stage2_logp: Optional[np.ndarray]):
+                 stage1_logp: np.ndarray, stage2_logp: Optional[np.ndarray], approx: str = "swiglu"):
         self.mode, self.gamma, self.M = mode, gamma, M
+        self.two_prev = mode == "ar" and approx == "swiglu_2prev"
         self.top_m = [list(map(int, stage1_top_ids[i, :M])) for i in range(gamma)]
         if mode == "ar":
             self.rows = list(stage2_logp)
@@ -206,7 +256,7 @@ class ChildSource:
         else:
             raise ValueError(mode)
 
-    def child_row(self, depth: int, tok: int) -> Optional[int]:
+    def child_row(self, depth: int, tok: int, parent_tok: Optional[int] = None) -> Optional[int]:
         if depth >= self.gamma:          # reading R7
             return None
         if self.mode == "marginal":      # DDTree: every node shares q_{t+depth+1}
@@ -217,7 +267,12 @@ class ChildSource:
             return None                  # leaf: outside the M-ary tree
         if self.mode == "marginal_mary":
             return depth
-        return 1 + (depth - 1) * self.M + m        # row of q'^(m)_{t+depth+1}
+        if not self.two_prev:
+            return 1 + (depth - 1) * self.M + m    # row of q'^(m)_{t+depth+1}
+        if depth == 1:                             # reading R13: (x^(m)_{t+1}, x_t)
+            return 1 + m
+        mp = self.top_m[depth - 2].index(parent_tok)   # the parent was expanded: in the M-ary tree
+        return 1 + self.M + (depth - 2) * self.M * self.M + m * self.M + mp
 
 
 def build_tree_literal(src: ChildSource, root_tok: int, B: int, keep: Optional[int] = None) -> Tree:
@@ -240,7 +295,7 @@ def build_tree_literal(src: ChildSource, root_tok: int, B: int, keep: Optional[i
         node = len(toks)
         toks.append(v); parents.append(par); depths.append(dep); scores.append(-negs); rows.append(r)
         pops.append((-negs, dep, par, v))
-        cr = src.child_row(dep, v)
+        cr = src.child_row(dep, v, toks[par])
         if cr is not None:
             push_row(cr, node, -negs, dep + 1)
     return _finish(toks, parents, depths, scores, rows, B, pops)
@@ -278,7 +333,7 @@ def build_tree_lazy(src: ChildSource, root_tok: int, B: int, keep: Optional[int]
         toks.append(v); parents.append(par); depths.append(dep); scores.append(-negs); rows.append(r)
         pops.append((-negs, dep, par, v))
         push(r, par, pscore, dep, rank + 1)          # next sibling in the same row
-        cr = src.child_row(dep, v)
+        cr = src.child_row(dep, v, toks[par])
         if cr is not None:
             push(cr, node, -negs, dep + 1, 0)        # best child of the new node
     return _finish(toks, parents, depths, scores, rows, B, pops)
@@ -369,29 +424,32 @@ class SeqResult:
     tree: Tree
     mask: np.ndarray
     pos: np.ndarray
+    approx: str = "swiglu"
 
 
 def draft_sequence(H: np.ndarray, root_tok: int, root_pos: int, W: dict, *, M: int, K2: int,
                    B: int, temperature: float = 1.0, eps: float = 1e-6, mode: str = "ar",
                    emulate_bf16: bool = False, keep: Optional[int] = None,
-                   literal: bool = False, approx: str = "swiglu") -> SeqResult:
+                   literal: bool = False, approx: str = "swiglu",
+                   root_prev: Optional[int] = None) -> SeqResult:
     """One sequence through Algorithm 1 (both parts) and the mask. W holds float64 arrays
     lm_head [V,d], embed [V,d], norm_h [d], norm_e [d], w_gate [I,2d], w_up [I,2d],
-    w_down [d,I] (approx "swiglu") or w_lin [d,2d] (approx "linear", reading R12). `keep`
-    truncates every child list (reading R5); None = whole distributions."""
+    w_down [d,I] (approx "swiglu"; [I,3d] gate/up for "swiglu_2prev", reading R13, which also
+    needs root_prev, the token before the root) or w_lin [d,2d] (approx "linear", reading
+    R12). `keep` truncates every child list (reading R5); None = whole distributions."""
     gamma = H.shape[0]
     K1 = max(M, K2)
     s1_logp, top_ids, top_logp = stage1(H, W["lm_head"], temperature, K1)
     hp = s2 = cids = clp = None
     if mode == "ar":
-        hp, s2 = stage2(H, root_tok, top_ids, W, M, temperature, eps, emulate_bf16, approx)
+        hp, s2 = stage2(H, root_tok, top_ids, W, M, temperature, eps, emulate_bf16, approx, root_prev)
         cids = np.stack([ranked(r, K2) for r in s2])
         clp = np.take_along_axis(s2, cids, axis=1)
-    src = ChildSource(mode, gamma, M, top_ids, s1_logp, s2)
+    src = ChildSource(mode, gamma, M, top_ids, s1_logp, s2, approx)
     builder = build_tree_literal if literal else build_tree_lazy
     tree = builder(src, int(root_tok), B, keep)
     mask, pos = tree_mask(tree.parent, tree.depth, int(root_pos))
-    return SeqResult(s1_logp, top_ids, top_logp, hp, s2, cids, clp, tree, mask, pos)
+    return SeqResult(s1_logp, top_ids, top_logp, hp, s2, cids, clp, tree, mask, pos, approx)
 
 
 def weights_f64(inputs: dict, to_f64) -> dict:
@@ -441,7 +499,7 @@ def selection_margins(res: SeqResult, M: int, K2: int, B: int, mode: str = "ar")
 
 def _next_score_after(res: SeqResult, M, K2, B, mode):
     """Score of the (B+1)-th pop (the best candidate left out), or None."""
-    src = ChildSource(mode, res.top_ids.shape[0], M, res.top_ids, res.s1_logp, res.s2_logp)
+    src = ChildSource(mode, res.top_ids.shape[0], M, res.top_ids, res.s1_logp, res.s2_logp, res.approx)
     t = build_tree_lazy(src, int(res.tree.tok[0]), B + 1, keep=K2 if K2 < B else None)
     if len(t.pops) <= B:
         return None
@@ -467,7 +525,7 @@ def eligible_universe(src: ChildSource, max_nodes: int = 200000):
             out.append((s, depth, p))
             if len(out) > max_nodes:
                 raise RuntimeError("universe too large")
-            cr = src.child_row(depth, v)
+            cr = src.child_row(depth, v, path[-1] if path else None)
             if cr is not None:
                 frontier.append((p, s, cr, depth + 1))
     return out

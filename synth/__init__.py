@@ -45,7 +45,8 @@ class Config:
     B: int
     dtype: str = "bf16"            # "bf16" or "f32": storage and input type of every tensor
     mode: str = "ar"               # "ar" (TreeFlash), "marginal" (DDTree), "marginal_mary"
-    approx: str = "swiglu"         # stage-2 approximator: "swiglu" (Eq. 1) or "linear" (ablation)
+    approx: str = "swiglu"         # stage-2 approximator: "swiglu" (Eq. 1), or the ablations'
+                                   # "linear" and "swiglu_2prev" (two previous tokens)
     temperature: float = 1.0
     rms_eps: float = 1e-6
     seed: int = 0
@@ -56,7 +57,10 @@ class Config:
 
     @property
     def R(self) -> int:
-        """Stage-2 rows per sequence: one for depth 1, M for each depth 2..gamma."""
+        """Stage-2 rows per sequence: one for depth 1, M for each depth 2..gamma (with two
+        previous tokens: M for depth 2 and M^2 for each depth 3..gamma)."""
+        if self.approx == "swiglu_2prev":
+            return 1 if self.gamma == 1 else 1 + self.M + self.M * self.M * (self.gamma - 2)
         return 1 + self.M * (self.gamma - 1)
 
     @property
@@ -95,6 +99,10 @@ CONFIGS = {
     "q8_m64": Config("q8_m64", batch=1, M=64, K2=64, B=64, **_Q8),
     # the q8_b64 step with the "w/ Linear" ablation's approximator (Sec. 4, Table 3)
     "q8_b64_linear": Config("q8_b64_linear", batch=1, M=16, K2=64, B=64, approx="linear", **_Q8),
+    # the q8_b32 and q8_b64 steps with the two-previous-token approximator (the "w/ 2-prev"
+    # ablation): 1 + M + M^2 (gamma - 2) = 905 / 3601 stage-2 rows
+    "q8_b32_2prev": Config("q8_b32_2prev", batch=1, M=8, K2=32, B=32, approx="swiglu_2prev", **_Q8),
+    "q8_b64_2prev": Config("q8_b64_2prev", batch=1, M=16, K2=64, B=64, approx="swiglu_2prev", **_Q8),
     # the q8_b64 step with the vocabulary cut to 32768 (W_lm 268 MB, still twice the L2):
     # small enough for multi-pass profiler captures
     "prof_v32k": Config("prof_v32k", batch=1, M=16, K2=64, B=64, **dict(_Q8, V=32768)),
@@ -163,7 +171,10 @@ def make_inputs(cfg: Config, seed: Optional[int] = None) -> dict:
     w_gate [I, 2d], w_up [I, 2d], w_down [d, I], root_tok [b] int32, root_pos [b] int32,
     h_scale [gamma] float64 (the per-depth hidden-state std that was used), and for the linear
     approximator w_lin [d, 2d] ~ N(0, wd_std^2), drawn last so that every other tensor is the
-    same as for the SwiGLU configuration of the same shape and seed.
+    same as for the SwiGLU configuration of the same shape and seed. For the two-previous-token
+    approximator w_gate and w_up are [I, 3d]: the SwiGLU configuration's [I, 2d] matrices with
+    d more columns (for the second previous token) drawn last, and root_prev [b] int32 is the
+    token before each root.
     """
     seed = cfg.seed if seed is None else seed
     dt = torch.float32 if cfg.dtype == "f32" else torch.bfloat16
@@ -186,6 +197,10 @@ def make_inputs(cfg: Config, seed: Optional[int] = None) -> dict:
                root_tok=root_tok, root_pos=root_pos, h_scale=scales)
     if cfg.approx == "linear":
         out["w_lin"] = _randn(g, (d, 2 * d), cfg.wd_std, dt)
+    elif cfg.approx == "swiglu_2prev":
+        out["w_gate"] = torch.cat([w_gate, _randn(g, (I, d), cfg.w_std, dt)], dim=1).contiguous()
+        out["w_up"] = torch.cat([w_up, _randn(g, (I, d), cfg.w_std, dt)], dim=1).contiguous()
+        out["root_prev"] = torch.randint(0, V, (cfg.batch,), generator=g, dtype=torch.int64).to(torch.int32)
     return out
 
 

@@ -548,3 +548,134 @@ def test_accept_walk_is_the_longest_consistent_root_path(seed):
     path, bonus = O.accept_walk(tok, par, ver)
     assert path == best and bonus == ver[best[-1]]
     assert 1 <= len(path) <= res.tree.depth.max() + 1
+
+
+# ------------------------------------------------------------------ "w/ 2-prev" approximator
+# (Sec. 4 "Model Design", Table 3; reading R13): x = [h~ ; e(prev) ; e(token before prev)],
+# one stage-2 row per pair of M-ary candidates of the two previous depths.
+
+
+def small_problem_2prev(V=32, d=16, I=24, gamma=4, seed=0, extra_std=0.3, **kw):
+    """small_problem with gate/up widened to [I, 3d] (extra columns for the second previous
+    token) and a token before the root."""
+    H, root, W = small_problem(V=V, d=d, I=I, gamma=gamma, seed=seed, **kw)
+    rng = np.random.default_rng(1000 + seed)
+    W = dict(W, w_gate=np.hstack([W["w_gate"], rng.normal(0, extra_std, (I, d))]),
+             w_up=np.hstack([W["w_up"], rng.normal(0, extra_std, (I, d))]))
+    return H, root, int(rng.integers(0, V)), W
+
+
+def test_2prev_row_layout():
+    # gamma = 3, M = 2: depth 1 on (root, token before it); depth 2 on (candidate m of depth 1,
+    # root); depth 3 on (candidate m1 of depth 2, candidate m2 of depth 1), m1-major
+    top = np.array([[10, 11, 99], [20, 21, 98], [30, 31, 97]])
+    hid, p1, p2 = O.stage2_conditioning_2prev(3, 2, root_tok=7, root_prev=5, top_ids=top)
+    assert hid.tolist() == [0, 1, 1, 2, 2, 2, 2]
+    assert p1.tolist() == [7, 10, 11, 20, 20, 21, 21]
+    assert p2.tolist() == [5, 7, 7, 10, 11, 10, 11]
+    assert O.stage2_rows(3, 2, "swiglu_2prev") == 7 == len(hid)
+    assert O.stage2_rows(16, 16, "swiglu_2prev") == 1 + 16 + 256 * 14
+    assert O.stage2_rows(1, 16, "swiglu_2prev") == 1
+    # the child row of a node is the row conditioned on (its token, its parent's token)
+    src = O.ChildSource("ar", 3, 2, top, np.zeros((3, 4)), np.zeros((7, 4)), approx="swiglu_2prev")
+    assert src.child_row(1, 11, 7) == 2
+    assert [src.child_row(2, t, pt) for t in (20, 21) for pt in (10, 11)] == [3, 4, 5, 6]
+    for r in range(3, 7):
+        assert (p1[r], p2[r]) == ({3: 20, 4: 20, 5: 21, 6: 21}[r], {3: 10, 4: 11, 5: 10, 6: 11}[r])
+    assert src.child_row(2, 99, 10) is None and src.child_row(3, 30, 20) is None
+
+
+def test_2prev_approximator_hand_computed():
+    # d = 2, I = 1, norm weights 1, eps = 0; h = (3, 4), e = (1, -1), e2 = (2, 0): RMS sqrt(2)
+    h, e, e2 = np.array([[3.0, 4.0]]), np.array([[1.0, -1.0]]), np.array([[2.0, 0.0]])
+    wg = np.array([[1.0, 0.0, 0.0, 0.0, 1.0, 0.0]])    # G = x0 + x4
+    wu = np.array([[0.0, 1.0, 0.0, 0.0, 0.0, -1.0]])   # U = x1 - x5
+    wd = np.array([[2.0], [-1.0]])
+    x0, x1, x4, x5 = 3 / math.sqrt(12.5), 4 / math.sqrt(12.5), 2 / math.sqrt(2), 0.0
+    G, U = x0 + x4, x1 - x5
+    a = G / (1 + math.exp(-G)) * U
+    got = O.ar_approximator(h, e, np.ones(2), np.ones(2), wg, wu, wd, 0.0, e2_raw=e2)
+    np.testing.assert_allclose(got, np.array([[3 + 2 * a, 4 - a]]), rtol=1e-14)
+
+
+def _run_2prev(zero_extra=False, approx="swiglu_2prev", V=32, gamma=4, M=3, B=12, seed=0, literal=False,
+               **kw):
+    H, root, prev, W = small_problem_2prev(V=V, gamma=gamma, seed=seed, **kw)
+    d = H.shape[1]
+    if zero_extra:
+        W["w_gate"][:, 2 * d:] = 0.0
+        W["w_up"][:, 2 * d:] = 0.0
+    if approx == "swiglu":
+        W = dict(W, w_gate=W["w_gate"][:, :2 * d], w_up=W["w_up"][:, :2 * d])
+    return O.draft_sequence(H, root, 1000, W, M=M, K2=B, B=B, approx=approx, root_prev=prev,
+                            literal=literal)
+
+
+def test_2prev_without_second_token_columns_equals_treeflash():
+    # zero columns for the second previous token: every row (i, m1, m2) is TreeFlash's row
+    # (i, m1), so the trees coincide (pins the row layout and the child-row rule together)
+    for seed in range(4):
+        a = _run_2prev(zero_extra=True, seed=seed)
+        b = _run_2prev(approx="swiglu", seed=seed)
+        M, g = 3, 4
+        for r in range(O.stage2_rows(g, M, "swiglu_2prev")):
+            if r == 0:
+                rb = 0
+            elif r <= M:
+                rb = r
+            else:
+                q = r - 1 - M
+                rb = 1 + (2 + q // (M * M) - 1) * M + (q % (M * M)) // M
+            np.testing.assert_allclose(a.s2_logp[r], b.s2_logp[rb], atol=1e-12)
+        np.testing.assert_array_equal(a.tree.tok, b.tree.tok)
+        np.testing.assert_array_equal(a.tree.parent, b.tree.parent)
+        np.testing.assert_allclose(a.tree.score, b.tree.score, atol=1e-12)
+
+
+def test_2prev_second_token_matters():
+    # with non-zero columns the rows of one (depth, previous token) differ by the token before
+    a = _run_2prev(seed=2, extra_std=1.0)
+    M = 3
+    r = 1 + M                       # depth 3, candidates (m1 = 0, m2 = 0) and (0, 1)
+    assert np.abs(a.s2_logp[r] - a.s2_logp[r + 1]).max() > 1e-3
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_2prev_tree_invariants_and_literal(seed):
+    res = _run_2prev(seed=seed, B=14, h_scale=2.0, extra_std=1.0)
+    _check_structure(res, 14, 4, 3, "ar")
+    t = res.tree
+    # every node's list is the row of (its parent's token, its grandparent's token)
+    for i in range(1, 15):
+        p = int(t.parent[i])
+        if t.depth[i] == 1:
+            assert t.row[i] == 0
+        elif t.depth[i] == 2:
+            assert t.row[i] == 1 + res.top_ids[0, :3].tolist().index(t.tok[p])
+        else:
+            gp = int(t.parent[p])
+            dp = int(t.depth[p])
+            m = res.top_ids[dp - 1, :3].tolist().index(t.tok[p])
+            mp = res.top_ids[dp - 2, :3].tolist().index(t.tok[gp])
+            assert t.row[i] == 1 + 3 + (dp - 2) * 9 + m * 3 + mp
+    lit = _run_2prev(seed=seed, B=14, h_scale=2.0, extra_std=1.0, literal=True)
+    np.testing.assert_array_equal(lit.tree.tok, t.tok)
+    np.testing.assert_array_equal(lit.tree.parent, t.parent)
+
+
+def test_2prev_brute_force_top_b_and_exhaustive_optimum():
+    # V = 16: the tree is the B best path scores of every node the rule allows; V = 4: it
+    # attains the largest summed path probability over all prefix-closed sets
+    H, root, prev, W = small_problem_2prev(V=16, d=16, gamma=4, seed=11, h_scale=2.0, extra_std=1.0)
+    res = O.draft_sequence(H, root, 0, W, M=4, K2=12, B=12, approx="swiglu_2prev", root_prev=prev)
+    src = O.ChildSource("ar", 4, 4, res.top_ids, res.s1_logp, res.s2_logp, approx="swiglu_2prev")
+    uni = O.eligible_universe(src)
+    uni.sort(key=lambda x: (-x[0], x[1]))
+    assert {p for _, _, p in uni[:12]} == set(O.tree_paths(res.tree))
+    assert uni[11][0] - uni[12][0] > 1e-9
+    H, root, prev, W = small_problem_2prev(V=4, d=8, I=8, gamma=3, seed=13, h_scale=1.5, extra_std=1.0)
+    for B in (3, 5):
+        res = O.draft_sequence(H, root, 0, W, M=2, K2=B, B=B, approx="swiglu_2prev", root_prev=prev)
+        src = O.ChildSource("ar", 3, 2, res.top_ids, res.s1_logp, res.s2_logp, approx="swiglu_2prev")
+        got = sum(math.exp(s) for s in res.tree.score[1:])
+        assert abs(O.best_prefix_closed_value(O.eligible_universe(src), B) - got) < 1e-12
