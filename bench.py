@@ -35,6 +35,7 @@ sys.path.insert(0, ROOT)
 METRIC = "µs per draft-tree build (trees/s) at Qwen3-8B shape, B=32/64; % of HBM roofline"
 WORKLOAD = "q8_b64"
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
 
 
 # ------------------------------------------------------------------------------ distributed
@@ -140,6 +141,15 @@ def peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def tensor_peak():
+    """bf16 dense tensor rate for a kernel timed inside a long step (the sustained figure)."""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        return float(json.load(open(p))["bf16_tflops_sustained"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_BF16_TFLOPS_SUSTAINED, "fallback"
+
+
 def kernel_source_hash():
     h = hashlib.sha256()
     for f in ("tc_gemm.cu", "tc_ptx.cuh", "common.cuh"):
@@ -169,11 +179,40 @@ def algorithmic_bytes(cfg):
     if cfg.approx == "linear":
         mlp = cfg.d * 2 * cfg.d * e                    # W_lin [d, 2d]
     else:
-        mlp = (2 * cfg.I * 2 * cfg.d + cfg.d * cfg.I) * e   # W_gate, W_up [I, 2d]; W_down [d, I]
+        k_in = (3 if cfg.approx == "swiglu_2prev" else 2) * cfg.d
+        mlp = (2 * cfg.I * k_in + cfg.d * cfg.I) * e   # W_gate, W_up [I, 2d or 3d]; W_down [d, I]
     rows = cfg.batch * cfg.R
     gathered = rows * cfg.d * e
     hidden = cfg.batch * cfg.gamma * cfg.d * e
     return 2 * lm + mlp + gathered + hidden, lm
+
+
+def lmhead_roofline(cfg, n1, n2, lm1_ms, lm2_ms, hbm_peak, tc_peak, traffic, timing):
+    """The `roofline` object of the dominant kernel, the LM-head pass (one launch over the n1
+    stage-1 rows, one over the n2 stage-2 rows; lm1_ms / lm2_ms their mean CUDA-event times).
+    Per launch it moves |W_lm| + rows * d * 2 bytes and does 2 * rows * V * d flops. The pass
+    is bound by HBM unless the bf16 contraction at the sustained tensor rate takes longer than
+    streaming those bytes at the copy rate (many stage-2 rows: batched sequences, two previous
+    tokens); then it is reported against the tensor rate, with the HBM figures beside it.
+    hbm_peak, tc_peak: (value, kind) in GB/s and TFLOP/s."""
+    (peak, peak_kind), (tc, tc_kind) = hbm_peak, tc_peak
+    _, lm_bytes = algorithmic_bytes(cfg)
+    nbytes = [lm_bytes + n1 * cfg.d * 2, lm_bytes + n2 * cfg.d * 2]
+    flops = [2.0 * n1 * cfg.V * cfg.d, 2.0 * n2 * cfg.V * cfg.d]
+    avg_s = (lm1_ms + lm2_ms) / 2 / 1e3
+    gbs = sum(nbytes) / 2 / avg_s / 1e9
+    hbm = {"bound": "hbm", "kernel": "tc_gemm_kernel<LMHEAD> (stage-1 and stage-2 launches)",
+           "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak, "traffic": traffic,
+           "peak_kind": peak_kind, "launch_ms": {"stage1": lm1_ms, "stage2": lm2_ms},
+           "bytes_per_launch": {"stage1": nbytes[0], "stage2": nbytes[1]},
+           "flops_per_launch": {"stage1": flops[0], "stage2": flops[1]}, "timing": timing}
+    if sum(flops) / (tc * 1e12) <= sum(nbytes) / (peak * 1e9):
+        return hbm
+    tflops = sum(flops) / 2 / avg_s / 1e12
+    out = dict(hbm, bound="tensor", achieved=tflops, peak=tc, unit="TFLOP/s", frac=tflops / tc,
+               peak_kind=f"{tc_kind} bf16 sustained")
+    out["hbm"] = {"achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak}
+    return out
 
 
 # ------------------------------------------------------------------------------ oracle timing
@@ -191,6 +230,7 @@ class OracleSample:
         self.lm = synth.to_f64(inp["lm_head"])
         self.H = synth.to_f64(inp["hidden"][0])
         self.root = int(inp["root_tok"][0])
+        self.root_prev = int(inp["root_prev"][0]) if inp.get("root_prev") is not None else None
 
     def run(self, fraction: float):
         """Returns (seconds for the sample, estimated seconds for a whole tree, vocabulary used)."""
@@ -200,9 +240,15 @@ class OracleSample:
         Vs = max(cfg.K2 + cfg.M, int(math.ceil(cfg.V * fraction)))
         W = dict(self.W, lm_head=self.lm[:Vs])
         root = self.root % Vs
-        hid, prev = O.stage2_conditioning(cfg.gamma, cfg.M, root, np.zeros((cfg.gamma, cfg.M), dtype=np.int64))
+        rprev = None if self.root_prev is None else self.root_prev % Vs
+        no_top = np.zeros((cfg.gamma, cfg.M), dtype=np.int64)
+        hid, prev = O.stage2_conditioning(cfg.gamma, cfg.M, root, no_top)
         t0 = time.perf_counter()
-        if cfg.approx == "linear":
+        if cfg.approx == "swiglu_2prev":
+            hid, prev, prev2 = O.stage2_conditioning_2prev(cfg.gamma, cfg.M, root, rprev, no_top)
+            O.ar_approximator(self.H[hid], W["embed"][prev], W["norm_h"], W["norm_e"], W["w_gate"], W["w_up"],
+                              W["w_down"], cfg.rms_eps, e2_raw=W["embed"][prev2])
+        elif cfg.approx == "linear":
             O.linear_approximator(self.H[hid], W["embed"][prev], W["norm_h"], W["norm_e"], W["w_lin"], cfg.rms_eps)
         else:
             O.ar_approximator(self.H[hid], W["embed"][prev], W["norm_h"], W["norm_e"], W["w_gate"], W["w_up"],
@@ -210,7 +256,7 @@ class OracleSample:
         t_mlp = time.perf_counter() - t0
         t0 = time.perf_counter()
         O.draft_sequence(self.H, root, 0, W, M=cfg.M, K2=cfg.K2, B=cfg.B, temperature=cfg.temperature,
-                         eps=cfg.rms_eps, mode=cfg.mode, approx=cfg.approx)
+                         eps=cfg.rms_eps, mode=cfg.mode, approx=cfg.approx, root_prev=rprev)
         t = time.perf_counter() - t0
         full = t_mlp + max(t - t_mlp, 0.0) * cfg.V / Vs
         return t, full, Vs
@@ -273,6 +319,10 @@ def run_gpu(args):
     cfg = synth.get_config(args.workload, seed=rank)
     inp = synth.make_inputs(cfg)
     d = {k: v.to(dev) for k, v in inp.items() if isinstance(v, torch.Tensor)}
+    # the two-previous-token approximator takes (x_t, x_{t-1}) per sequence in root_tok
+    root_in = inp["root_tok"] if "root_prev" not in inp else \
+        torch.stack([inp["root_tok"], inp["root_prev"]], dim=1).contiguous()
+    d["root_tok"] = root_in.to(dev)
     dims = Bn.Dims.from_config(cfg)
     dr = tf.Drafter(dims, d, dev)
     hp = Bn.tf_workspace_h_prime(dims, dr.ws)
@@ -350,18 +400,17 @@ def run_gpu(args):
     ms_per_step = elapsed_ms / args.steps
     peak, peak_kind = peaks()
     step_bytes, lm_bytes = algorithmic_bytes(cfg)
-    e = 2
-    lm_launch_bytes = [lm_bytes + n1 * cfg.d * e, lm_bytes + n2 * cfg.d * e]
-    avg_launch_ms = (sum(lm1) + sum(lm2)) / (2 * n_inst)
-    achieved = (sum(lm_launch_bytes) / 2) / (avg_launch_ms / 1e3) / 1e9
-    traffic = profiled_traffic()
+    timing = (f"CUDA events around each LM-head launch over {n_inst} further steps "
+              f"({inst_ms_per_step * 1e3:.1f} us per step with the events)")
+    roofline = lmhead_roofline(cfg, n1, n2, statistics.mean(lm1), statistics.mean(lm2), (peak, peak_kind),
+                               tensor_peak(), profiled_traffic(), timing)
 
     # ---- end to end through the host-buffer entry point
     e2e = None
     if args.e2e_steps > 0:
         n = cfg.B + 1
         pin = lambda t: t.pin_memory()
-        h_hidden, h_root, h_pos = pin(inp["hidden"]), pin(inp["root_tok"]), pin(inp["root_pos"])
+        h_hidden, h_root, h_pos = pin(inp["hidden"]), pin(root_in), pin(inp["root_pos"])
         outs = dict(node_tok=torch.empty(cfg.batch, n, dtype=torch.int32),
                     node_parent=torch.empty(cfg.batch, n, dtype=torch.int32),
                     node_depth=torch.empty(cfg.batch, n, dtype=torch.int32),
@@ -414,13 +463,7 @@ def run_gpu(args):
         "step_roofline": {"algorithmic_bytes": step_bytes, "achieved_gbs": step_bytes / (ms_per_step / 1e3) / 1e9,
                           "peak_gbs": peak, "frac": step_bytes / (ms_per_step / 1e3) / 1e9 / peak,
                           "peak_kind": peak_kind},
-        "roofline": {"bound": "hbm", "kernel": "tc_gemm_kernel<LMHEAD> (stage-1 and stage-2 launches)",
-                     "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                     "traffic": traffic, "peak_kind": peak_kind,
-                     "launch_ms": {"stage1": statistics.mean(lm1), "stage2": statistics.mean(lm2)},
-                     "bytes_per_launch": {"stage1": lm_launch_bytes[0], "stage2": lm_launch_bytes[1]},
-                     "timing": f"CUDA events around each LM-head launch over {n_inst} further steps "
-                               f"({inst_ms_per_step * 1e3:.1f} us per step with the events)"},
+        "roofline": roofline,
         "clocks": clocks, "e2e": e2e, "gpu_launches": gpu_launches,
         "cpu_baseline": cpu, "device_flags": flags,
     }

@@ -24,7 +24,8 @@
  *  - Shapes are row-major. b = batch (independent sequences), d = hidden size, V = vocabulary,
  *    I = approximator width, gamma = block size, M = stage-1 candidates per depth, K2 =
  *    children kept per stage-2 row, B = draft budget (non-root nodes),
- *    R = 1 + M (gamma - 1) stage-2 rows per sequence, K1 = max(M, K2).
+ *    R = 1 + M (gamma - 1) stage-2 rows per sequence (TF_APPROX_SWIGLU_2PREV: 1 + M +
+ *    M^2 (gamma - 2) for gamma >= 2), K1 = max(M, K2).
  *  - Float tensors have the element type of dims->dtype (TF_BF16: __nv_bfloat16, TF_F32:
  *    float); log-probabilities are always float32, token ids int32.
  *  - Errors: a call that finds an invalid argument returns TF_ERR_INVALID_ARG,
@@ -72,9 +73,16 @@ typedef enum {
 /* Which AR-approximator stage 2 runs (TF_MODE_AR only). */
 typedef enum {
     TF_APPROX_SWIGLU = 0,      /* Eq. 1: h' = h + W_down (SiLU(W_gate x) * (W_up x)), x = [h~ ; e] */
-    TF_APPROX_LINEAR = 1       /* the "w/ Linear" ablation (Sec. 4 "Model Design", Table 3): the
+    TF_APPROX_LINEAR = 1,      /* the "w/ Linear" ablation (Sec. 4 "Model Design", Table 3): the
                                   SwiGLU replaced by one linear layer on the same input,
                                   h' = h + W_lin x, W_lin [d, 2d], no bias */
+    TF_APPROX_SWIGLU_2PREV = 2 /* the "w/ 2-prev" ablation (Sec. 4 "Model Design", Table 3): the
+                                  SwiGLU of Eq. 1 on x = [h~ ; e(prev) ; e(token before prev)]
+                                  (both embeddings normalised with norm_e), W_gate and W_up
+                                  [I, 3d]. Stage 2 then has one row per pair of M-ary candidates
+                                  (R = 1 + M + M^2 (gamma - 2), see tf_stage2_ar_approx), and
+                                  root_tok holds TWO tokens per sequence, [b, 2] = (x_t, x_{t-1}),
+                                  in every call that takes it */
 } tf_approx;
 
 /* Device status bits (int32 words written with atomic OR). */
@@ -109,8 +117,9 @@ typedef struct {
     const void* embed;    /* [V, d]  verifier input embedding Embd */
     const void* norm_h;   /* [d]     RMSNorm weight of the hidden-state half of Eq. 1 */
     const void* norm_e;   /* [d]     RMSNorm weight of the embedding half of Eq. 1 */
-    const void* w_gate;   /* [I, 2d] SwiGLU gate projection, input [h~ ; e] */
-    const void* w_up;     /* [I, 2d] SwiGLU up projection, input [h~ ; e] */
+    const void* w_gate;   /* [I, 2d] SwiGLU gate projection, input [h~ ; e] ([I, 3d] with
+                             TF_APPROX_SWIGLU_2PREV, input [h~ ; e ; e2]) */
+    const void* w_up;     /* [I, 2d] SwiGLU up projection, input [h~ ; e] ([I, 3d] likewise) */
     const void* w_down;   /* [d, I]  SwiGLU down projection */
     const void* w_lin;    /* [d, 2d] linear approximator, input [h~ ; e] (TF_APPROX_LINEAR only;
                              w_gate, w_up and w_down are then not read and may be NULL) */
@@ -157,6 +166,11 @@ tf_status tf_stage1_marginals(const tf_dims* dims, const tf_weights* w, const vo
  *   row 1 + (i-2) M + m:   h' = h_{t+i} + SwiGLU(RMSNorm(h_{t+i}) :: RMSNorm(Embd(x^(m)_{t+i-1})))
  * for i = 2..gamma, m = 0..M-1, then q' = softmax(W_lm h' / T) and its K2 largest entries.
  * With dims->approx == TF_APPROX_LINEAR, W_lin (...) takes the place of SwiGLU(...).
+ * With TF_APPROX_SWIGLU_2PREV the input also holds RMSNorm(Embd(token before prev)) and the
+ * rows are (root_tok [b, 2] = (x_t, x_{t-1}))
+ *   row 0:                          depth 1, tokens (x_t, x_{t-1})
+ *   row 1 + m:                      depth 2, tokens (x^(m)_{t+1}, x_t)
+ *   row 1 + M + (i-3) M^2 + m1 M + m2: depth i >= 3, tokens (x^(m1)_{t+i-1}, x^(m2)_{t+i-2}).
  *  hidden     [b, gamma, d] dtype (as in stage 1)
  *  root_tok   [b] int32: the last accepted token x_t of each sequence
  *  top_ids    [b, gamma, K1] int32: stage-1 output (the first M per depth are used)
@@ -174,8 +188,10 @@ tf_status tf_stage2_ar_approx(const tf_dims* dims, const tf_weights* w, const vo
  * at depth i < gamma whose token is x^(m)_{t+i} (m < M) makes row 1 + (i-1) M + m available
  * (TF_MODE_AR); in TF_MODE_MARGINAL every node at depth i < gamma makes stage-1 depth i+1
  * available, in TF_MODE_MARGINAL_MARY only the M-ary ones do. Each distribution contributes
- * at most K2 children (exact when K2 >= B). child_ids/child_logp may be NULL in the marginal
- * modes. Outputs [b, B+1]: node 0 is the root (token root_tok, parent -1, depth 0, score 0);
+ * at most K2 children (exact when K2 >= B). With TF_APPROX_SWIGLU_2PREV a node of depth i whose
+ * token is x^(m)_{t+i} and whose parent's token is x^(m')_{t+i-1} takes row
+ * 1 + M + (i-2) M^2 + m M + m' (row 1 + m at depth 1), and root_tok is [b, 2] (x_t first).
+ * child_ids/child_logp may be NULL in the marginal modes. Outputs [b, B+1]: node 0 is the root (token root_tok, parent -1, depth 0, score 0);
  * nodes follow in pop order, so parent < child. Missing nodes (underfull universe) have
  * token/parent/depth -1 and score -inf, and set TF_DEV_UNDERFULL.
  *  dev_status [b] int32 out: TF_DEV_* bits per sequence (overwritten, not OR-ed). */

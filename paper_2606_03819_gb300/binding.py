@@ -22,7 +22,7 @@ TF_OK, TF_ERR_INVALID_ARG, TF_ERR_UNSUPPORTED, TF_ERR_WORKSPACE, TF_ERR_CUDA, TF
     TF_ERR_TIMEOUT = range(7)
 TF_BF16, TF_F32 = 0, 1
 MODES = {"ar": 0, "marginal": 1, "marginal_mary": 2}
-APPROX = {"swiglu": 0, "linear": 1}
+APPROX = {"swiglu": 0, "linear": 1, "swiglu_2prev": 2}
 TF_DEV_BAD_TOKEN, TF_DEV_UNDERFULL, TF_DEV_NONFINITE, TF_DEV_TIMEOUT, TF_DEV_RECOMPUTED = 1, 2, 4, 8, 16
 
 
@@ -114,15 +114,22 @@ class Dims:
     rms_eps: float = 1e-6
     dtype: str = "bf16"
     mode: str = "ar"
-    approx: str = "swiglu"      # "swiglu" (Eq. 1) or "linear" (the "w/ Linear" ablation)
+    approx: str = "swiglu"      # "swiglu" (Eq. 1); the ablations' "linear" and "swiglu_2prev"
 
     @property
     def R(self) -> int:
+        if self.approx == "swiglu_2prev" and self.mode == "ar":
+            return 1 if self.gamma == 1 else 1 + self.M + self.M * self.M * (self.gamma - 2)
         return 1 + self.M * (self.gamma - 1)
 
     @property
     def K1(self) -> int:
         return max(self.M, self.K2)
+
+    @property
+    def k_in(self) -> int:
+        """Width of the approximator input x: 2d, or 3d with two previous tokens."""
+        return (3 if self.approx == "swiglu_2prev" and self.mode == "ar" else 2) * self.d
 
     @property
     def torch_dtype(self):
@@ -280,7 +287,7 @@ TF_VIEW_X, TF_VIEW_A, TF_VIEW_H_PRIME, TF_VIEW_HALVES, TF_VIEW_CHUNKS = 0, 1, 2,
 
 
 def tf_workspace_view(dims: Dims, ws, view: int, n_rows: Optional[int] = None) -> torch.Tensor:
-    """x [b*R, 2d], A [b*R, I] or h' [b*R, d] as a tensor view of the workspace (no copy); for
+    """x [b*R, k_in], A [b*R, I] or h' [b*R, d] as a tensor view of the workspace (no copy); for
     TF_VIEW_HALVES / TF_VIEW_CHUNKS the partials of the last LM-head pass over n_rows rows as
     float32 [n_tiles, 2 or 8, n_rows, 4]."""
     p, n = ctypes.c_void_p(), ctypes.c_size_t()
@@ -292,7 +299,7 @@ def tf_workspace_view(dims: Dims, ws, view: int, n_rows: Optional[int] = None) -
         parts = 2 if view == TF_VIEW_HALVES else 8
         nb = n_tiles * parts * n_rows * 16
         return ws[off:off + nb].view(torch.float32).view(n_tiles, parts, n_rows, 4)
-    cols = {TF_VIEW_X: 2 * dims.d, TF_VIEW_A: dims.I, TF_VIEW_H_PRIME: dims.d}[view]
+    cols = {TF_VIEW_X: dims.k_in, TF_VIEW_A: dims.I, TF_VIEW_H_PRIME: dims.d}[view]
     return ws[off:off + n.value].view(dims.torch_dtype).view(dims.batch * dims.R, cols)
 
 

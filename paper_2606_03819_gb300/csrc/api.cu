@@ -29,12 +29,15 @@ size_t up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct Dims {
     int b, d, V, I, gamma, M, K2, B, K1, R, dtype, mode, approx, n_tiles;
+    int two_prev;     // TF_APPROX_SWIGLU_2PREV in TF_MODE_AR: two embeddings per row
+    int k_in;         // width of the approximator input x: 2d, or 3d with two_prev
+    int root_stride;  // int32 entries per sequence in root_tok: 1, or 2 with two_prev
     size_t esize;
     float inv_temp, eps;
 };
 
 struct Layout {
-    size_t status, halves, chunks, X, A, hp, kpart;
+    size_t status, halves, chunks, X, A, hp, hres, kpart;
     size_t h_hidden, h_root, h_pos, top_ids, top_logp, child_ids, child_logp;
     size_t n_tok, n_par, n_dep, n_score, n_mask, n_pos, n_stat;
     size_t total;
@@ -48,9 +51,11 @@ tf_status check_dims(const tf_dims* dims, Dims* o) {
     if (d.dtype != TF_BF16 && d.dtype != TF_F32) return TF_ERR_INVALID_ARG;
     if (d.mode != TF_MODE_AR && d.mode != TF_MODE_MARGINAL && d.mode != TF_MODE_MARGINAL_MARY)
         return TF_ERR_INVALID_ARG;
-    if (d.mode == TF_MODE_AR && d.approx != TF_APPROX_SWIGLU && d.approx != TF_APPROX_LINEAR)
+    if (d.mode == TF_MODE_AR && d.approx != TF_APPROX_SWIGLU && d.approx != TF_APPROX_LINEAR &&
+        d.approx != TF_APPROX_SWIGLU_2PREV)
         return TF_ERR_INVALID_ARG;
-    const bool swiglu = d.mode == TF_MODE_AR && d.approx == TF_APPROX_SWIGLU;
+    const bool two_prev = d.mode == TF_MODE_AR && d.approx == TF_APPROX_SWIGLU_2PREV;
+    const bool swiglu = d.mode == TF_MODE_AR && (d.approx == TF_APPROX_SWIGLU || two_prev);
     if (!(d.temperature > 0.0f) || !isfinite(d.temperature)) return TF_ERR_INVALID_ARG;
     if (!(d.rms_eps >= 0.0f) || !isfinite(d.rms_eps)) return TF_ERR_INVALID_ARG;
     const int K1 = d.M > d.K2 ? d.M : d.K2;
@@ -61,7 +66,10 @@ tf_status check_dims(const tf_dims* dims, Dims* o) {
         return TF_ERR_UNSUPPORTED;
     const int n_tiles = (d.V + kBlockV - 1) / kBlockV;
     if (merge_smem_bytes(n_tiles, d.d, K1) > kMaxMergeSmem) return TF_ERR_UNSUPPORTED;
-    const long long R = 1 + static_cast<long long>(d.M) * (d.gamma - 1);
+    // stage-2 rows per sequence: one for depth 1 and M per deeper depth; with two previous tokens
+    // M for depth 2 and M^2 per depth from 3 on
+    const long long M = d.M;
+    const long long R = !two_prev ? 1 + M * (d.gamma - 1) : d.gamma == 1 ? 1 : 1 + M + M * M * (d.gamma - 2);
     if (static_cast<long long>(d.batch) * R > (1ll << 30) || static_cast<long long>(d.batch) * d.gamma > (1ll << 30))
         return TF_ERR_UNSUPPORTED;
     o->b = d.batch;
@@ -78,6 +86,9 @@ tf_status check_dims(const tf_dims* dims, Dims* o) {
     o->mode = d.mode;
     o->approx = d.mode == TF_MODE_AR ? d.approx : TF_APPROX_SWIGLU;
     o->n_tiles = n_tiles;
+    o->two_prev = two_prev ? 1 : 0;
+    o->k_in = (two_prev ? 3 : 2) * d.d;
+    o->root_stride = two_prev ? 2 : 1;
     o->esize = d.dtype == TF_BF16 ? 2 : 4;
     o->inv_temp = 1.0f / d.temperature;
     o->eps = d.rms_eps;
@@ -99,15 +110,16 @@ Layout layout(const Dims& D) {
     L.status = take(sizeof(int32_t));
     L.halves = take(rows * D.n_tiles * kHalfBytesPerRowBlock);
     L.chunks = take(rows * D.n_tiles * kChunkBytesPerRowBlock);
-    L.X = take(rows2 * 2 * D.d * D.esize);
+    L.X = take(rows2 * D.k_in * D.esize);
     L.A = take(rows2 * D.I * D.esize);
     L.hp = take(rows2 * D.d * D.esize);
+    L.hres = take(D.two_prev ? rows2 * D.d * D.esize : 0);   // residual row of each stage-2 row
     // split-K partial sums of the bf16 approximator GEMMs: [k_splits][max(2I, d) / 4][rows][4] fp32
     L.kpart = D.dtype == TF_BF16 ? take(static_cast<size_t>(kMaxKSplits) * rows2 *
                                         (2 * static_cast<size_t>(D.I) > static_cast<size_t>(D.d) ? 2 * D.I : D.d) * 4)
                                  : take(0);
     L.h_hidden = take(rows1 * D.d * D.esize);
-    L.h_root = take(D.b * sizeof(int32_t));
+    L.h_root = take(static_cast<size_t>(D.b) * D.root_stride * sizeof(int32_t));
     L.h_pos = take(D.b * sizeof(int32_t));
     L.top_ids = take(rows1 * D.K1 * sizeof(int32_t));
     L.top_logp = take(rows1 * D.K1 * sizeof(float));
@@ -185,8 +197,10 @@ tf_status do_ar_approx(const Ctx& ctx, const Dims& D, const Layout& L, void* ws,
     void* X = at<void>(ws, L.X);
     void* A = at<void>(ws, L.A);
     void* hp = at<void>(ws, L.hp);
+    void* hres = at<void>(ws, L.hres);
     TF_TRY(cuda_status(launch_gather_norm(ctx, D.dtype, hidden, w->embed, w->norm_h, w->norm_e, root_tok, top_ids,
-                                          D.b, D.gamma, D.M, D.K1, D.d, D.V, D.eps, X)));
+                                          D.b, D.gamma, D.M, D.K1, D.R, D.two_prev, D.d, D.V, D.eps, X,
+                                          D.two_prev ? hres : nullptr)));
     const int rows = D.b * D.R;
     if (D.approx == TF_APPROX_LINEAR) {
         if (D.dtype == TF_BF16)
@@ -194,11 +208,15 @@ tf_status do_ar_approx(const Ctx& ctx, const Dims& D, const Layout& L, void* ws,
                                                 at<float>(ws, L.kpart)));
         return cuda_status(launch_linear_simt(ctx, X, w->w_lin, hidden, rows, D.d, D.R, D.M, D.gamma, hp));
     }
+    // the residual of stage-2 row r is the hidden state of its depth; with two previous tokens the
+    // gather has copied it to row r of hres, which the identity map (R = M = gamma = 1) reads
+    const void* res = D.two_prev ? hres : hidden;
+    const int rR = D.two_prev ? 1 : D.R, rM = D.two_prev ? 1 : D.M, rG = D.two_prev ? 1 : D.gamma;
     if (D.dtype == TF_BF16)
-        return cuda_status(launch_swiglu_tc(ctx, X, w->w_gate, w->w_up, w->w_down, hidden, rows, D.d, D.I, D.R, D.M,
-                                            D.gamma, A, hp, at<float>(ws, L.kpart)));
-    return cuda_status(launch_swiglu_simt(ctx, X, w->w_gate, w->w_up, w->w_down, hidden, rows, D.d, D.I, D.R, D.M,
-                                          D.gamma, A, hp));
+        return cuda_status(launch_swiglu_tc(ctx, X, D.k_in, w->w_gate, w->w_up, w->w_down, res, rows, D.d, D.I, rR, rM,
+                                            rG, A, hp, at<float>(ws, L.kpart)));
+    return cuda_status(launch_swiglu_simt(ctx, X, D.k_in, w->w_gate, w->w_up, w->w_down, res, rows, D.d, D.I, rR,
+                                          rM, rG, A, hp));
 }
 
 tf_status check_weights(const Dims& D, const tf_weights* w, bool need_mlp) {
@@ -350,8 +368,8 @@ tf_status tf_build_tree(const tf_dims* dims, const int32_t* root_tok, const int3
         return TF_ERR_INVALID_ARG;
     if (D.mode == TF_MODE_AR && (!child_ids || !child_logp)) return TF_ERR_INVALID_ARG;
     Ctx ctx{reinterpret_cast<cudaStream_t>(stream), 0, nullptr};
-    return cuda_status(launch_build_tree(ctx, D.b, D.gamma, D.M, D.K1, D.K2, D.B, D.V, D.mode, D.R, root_tok,
-                                         top_ids, top_logp, child_ids, child_logp, node_tok, node_parent,
+    return cuda_status(launch_build_tree(ctx, D.b, D.gamma, D.M, D.K1, D.K2, D.B, D.V, D.mode, D.R, D.two_prev,
+                                         root_tok, top_ids, top_logp, child_ids, child_logp, node_tok, node_parent,
                                          node_depth, node_score, dev_status));
 }
 
@@ -377,8 +395,8 @@ tf_status tf_build_tree_mask(const tf_dims* dims, const int32_t* root_tok, const
     if (D.mode == TF_MODE_AR && (!child_ids || !child_logp)) return TF_ERR_INVALID_ARG;
     Ctx ctx{reinterpret_cast<cudaStream_t>(stream), 0, nullptr};
     const bool fused = D.B + 1 <= kFusedMaskMaxNodes;   // the builder CTA writes the mask of its tree
-    TF_TRY(cuda_status(launch_build_tree(ctx, D.b, D.gamma, D.M, D.K1, D.K2, D.B, D.V, D.mode, D.R, root_tok, top_ids,
-                                         top_logp, child_ids, child_logp, node_tok, node_parent, node_depth,
+    TF_TRY(cuda_status(launch_build_tree(ctx, D.b, D.gamma, D.M, D.K1, D.K2, D.B, D.V, D.mode, D.R, D.two_prev, root_tok,
+                                         top_ids, top_logp, child_ids, child_logp, node_tok, node_parent, node_depth,
                                          node_score, dev_status, fused ? root_pos : nullptr,
                                          fused ? mask : nullptr, fused ? pos_ids : nullptr)));
     if (fused) return TF_OK;
@@ -430,7 +448,7 @@ tf_status tf_workspace_view(const tf_dims* dims, void* ws, size_t ws_bytes, int3
     }
     if (D.mode != TF_MODE_AR) return TF_ERR_INVALID_ARG;
     switch (view) {
-        case TF_VIEW_X: *ptr = at<void>(ws, L.X); *bytes = rows2 * 2 * D.d * D.esize; return TF_OK;
+        case TF_VIEW_X: *ptr = at<void>(ws, L.X); *bytes = rows2 * D.k_in * D.esize; return TF_OK;
         case TF_VIEW_A: *ptr = at<void>(ws, L.A); *bytes = rows2 * D.I * D.esize; return TF_OK;
         case TF_VIEW_H_PRIME: *ptr = at<void>(ws, L.hp); *bytes = rows2 * D.d * D.esize; return TF_OK;
     }
@@ -455,7 +473,8 @@ tf_status tf_draft_tree_host(const tf_dims* dims, const tf_weights* w, const voi
     int32_t* d_pos = at<int32_t>(ws, L.h_pos);
     TF_TRY(cuda_status(cudaMemcpyAsync(d_hidden, hidden, static_cast<size_t>(D.b) * D.gamma * D.d * D.esize,
                                        cudaMemcpyHostToDevice, st)));
-    TF_TRY(cuda_status(cudaMemcpyAsync(d_root, root_tok, D.b * sizeof(int32_t), cudaMemcpyHostToDevice, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(d_root, root_tok, static_cast<size_t>(D.b) * D.root_stride * sizeof(int32_t),
+                                       cudaMemcpyHostToDevice, st)));
     TF_TRY(cuda_status(cudaMemcpyAsync(d_pos, root_pos, D.b * sizeof(int32_t), cudaMemcpyHostToDevice, st)));
     int32_t* top_ids = at<int32_t>(ws, L.top_ids);
     float* top_logp = at<float>(ws, L.top_logp);

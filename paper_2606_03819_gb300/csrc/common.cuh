@@ -161,22 +161,28 @@ cudaError_t launch_lmhead_merge(const Ctx&, int dtype, Partials partials, int n_
                                 int d, int k, float inv_temp, const void* lm_head, const void* x,
                                 int32_t* out_ids, float* out_logp);
 // Eq. 1 pieces
+// x rows of stage 2 (R per sequence). two_prev: x = [h~ ; e(prev) ; e(token before prev)] (3d
+// wide) and root_tok holds two tokens per sequence; hres (two_prev only) receives each row's
+// residual hidden state.
 cudaError_t launch_gather_norm(const Ctx&, int dtype, const void* hidden, const void* embed,
                                const void* norm_h, const void* norm_e, const int32_t* root_tok,
-                               const int32_t* top_ids, int b, int gamma, int M, int K1, int d,
-                               int V, float eps, void* X);
-cudaError_t launch_swiglu_tc(const Ctx&, const void* X, const void* w_gate, const void* w_up,
-                             const void* w_down, const void* hidden, int n_rows, int d, int I,
-                             int R, int M, int gamma, void* A, void* h_prime, float* partial);
+                               const int32_t* top_ids, int b, int gamma, int M, int K1, int R,
+                               int two_prev, int d, int V, float eps, void* X, void* hres);
+// SwiGLU on x [n_rows, k_in] (k_in = 2d, or 3d with two previous tokens)
+cudaError_t launch_swiglu_tc(const Ctx&, const void* X, int k_in, const void* w_gate,
+                             const void* w_up, const void* w_down, const void* hidden, int n_rows,
+                             int d, int I, int R, int M, int gamma, void* A, void* h_prime,
+                             float* partial);
 // split-K reductions of the approximator GEMMs (partial sums in fp32, [k_splits][N / 4][rows][4])
 cudaError_t launch_swiglu_reduce(const Ctx&, const float* partial, int k_splits, int n_rows, int I,
                                  __nv_bfloat16* A);
 cudaError_t launch_down_reduce(const Ctx&, const float* partial, int k_splits, int n_rows, int d,
                                const __nv_bfloat16* hidden, int R, int M, int gamma,
                                __nv_bfloat16* h_prime);
-cudaError_t launch_swiglu_simt(const Ctx&, const void* X, const void* w_gate, const void* w_up,
-                               const void* w_down, const void* hidden, int n_rows, int d, int I,
-                               int R, int M, int gamma, void* A, void* h_prime);
+cudaError_t launch_swiglu_simt(const Ctx&, const void* X, int k_in, const void* w_gate,
+                               const void* w_up, const void* w_down, const void* hidden,
+                               int n_rows, int d, int I, int R, int M, int gamma, void* A,
+                               void* h_prime);
 // the "w/ Linear" approximator: h' = h + X W_lin^T, X [n_rows, 2d], W_lin [d, 2d]
 cudaError_t launch_linear_tc(const Ctx&, const void* X, const void* w_lin, const void* hidden,
                              int n_rows, int d, int R, int M, int gamma, void* h_prime,
@@ -185,7 +191,8 @@ cudaError_t launch_linear_simt(const Ctx&, const void* X, const void* w_lin, con
                                int n_rows, int d, int R, int M, int gamma, void* h_prime);
 // Part 2 and the mask
 cudaError_t launch_build_tree(const Ctx&, int b, int gamma, int M, int K1, int K2, int B, int V,
-                              int mode, int R, const int32_t* root_tok, const int32_t* top_ids,
+                              int mode, int R, int two_prev, const int32_t* root_tok,
+                              const int32_t* top_ids,
                               const float* top_logp, const int32_t* child_ids,
                               const float* child_logp, int32_t* node_tok, int32_t* node_parent,
                               int32_t* node_depth, float* node_score, int32_t* dev_status,

@@ -196,13 +196,13 @@ cudaError_t launch_lmhead_simt(const Ctx& ctx, int dtype, const void* lm_head, c
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-cudaError_t launch_swiglu_simt(const Ctx& ctx, const void* X, const void* w_gate, const void* w_up,
+cudaError_t launch_swiglu_simt(const Ctx& ctx, const void* X, int k_in, const void* w_gate, const void* w_up,
                                const void* w_down, const void* hidden, int n_rows, int d, int I, int R, int M,
                                int gamma, void* A, void* h_prime) {
     if (n_rows <= 0) return cudaSuccess;
     dim3 g1((I + 63) / 64, (n_rows + 63) / 64);
     cudaError_t e = launch_pdl(swiglu_simt_kernel<true>, g1, dim3(256), 0, ctx.stream, static_cast<const float*>(X),
-                               static_cast<const float*>(w_gate), static_cast<const float*>(w_up), n_rows, 2 * d, I,
+                               static_cast<const float*>(w_gate), static_cast<const float*>(w_up), n_rows, k_in, I,
                                static_cast<float*>(A), static_cast<const float*>(nullptr), R, M, gamma);
     if (e == cudaSuccess) e = cudaGetLastError();
     if (e != cudaSuccess) return e;

@@ -814,7 +814,7 @@ static cudaError_t run_residual_gemm(const Ctx& ctx, const CUtensorMap& ta, cons
                               static_cast<__nv_bfloat16*>(h_prime));
 }
 
-cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, const void* w_gate, const void* w_up,
+cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, int k_in, const void* w_gate, const void* w_up,
                              const void* w_down, const void* hidden, int n_rows, int d, int I, int R, int M,
                              int gamma, void* A, void* h_prime, float* partial) {
     if (n_rows <= 0) return cudaSuccess;
@@ -824,15 +824,15 @@ cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, const void* w_gate, 
     const int bn_gu = I % BN == 0 ? BN : 64;
     const int bn_d = d % BN == 0 ? BN : 64;
     CUtensorMap tx, tg, tu, ta, td;
-    cudaError_t e = make_tmap(&tx, X, 2 * d, n_rows, kBK, kBM);
-    if (e == cudaSuccess) e = make_tmap(&tg, w_gate, 2 * d, I, kBK, bn_gu);
-    if (e == cudaSuccess) e = make_tmap(&tu, w_up, 2 * d, I, kBK, bn_gu);
+    cudaError_t e = make_tmap(&tx, X, k_in, n_rows, kBK, kBM);
+    if (e == cudaSuccess) e = make_tmap(&tg, w_gate, k_in, I, kBK, bn_gu);
+    if (e == cudaSuccess) e = make_tmap(&tu, w_up, k_in, I, kBK, bn_gu);
     if (e == cudaSuccess) e = make_tmap(&ta, A, I, n_rows, kBK, kBM);
     if (e == cudaSuccess) e = make_tmap(&td, w_down, I, d, kBK, bn_d);
     if (e != cudaSuccess) return e;
 
     // ---- gate/up: A = SiLU(X Wg^T) * (X Wu^T)
-    const int ks1 = choose_k_splits((I / bn_gu) * n_mg, 2 * d / kBK, ctx.num_sms);
+    const int ks1 = choose_k_splits((I / bn_gu) * n_mg, k_in / kBK, ctx.num_sms);
     EpiParams ep{};
     ep.out = static_cast<__nv_bfloat16*>(A);
     ep.ld_out = I;
@@ -841,23 +841,23 @@ cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, const void* w_gate, 
     ep.n_total = I;
     if (ks1 == 1) {
         if (bn_gu == BN)
-            e = m_tiles == 1 ? run_gemm<EPI_GATEUP, 1, 2, BN, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, 1, ep)
-                             : run_gemm<EPI_GATEUP, 2, 2, BN, 3>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, n_mg, ep);
+            e = m_tiles == 1 ? run_gemm<EPI_GATEUP, 1, 2, BN, 4>(ctx, tx, tg, tu, n_rows, k_in, I / BN, 1, ep)
+                             : run_gemm<EPI_GATEUP, 2, 2, BN, 3>(ctx, tx, tg, tu, n_rows, k_in, I / BN, n_mg, ep);
         else
-            e = m_tiles == 1 ? run_gemm<EPI_GATEUP, 1, 2, 64, 6>(ctx, tx, tg, tu, n_rows, 2 * d, I / 64, 1, ep)
-                             : run_gemm<EPI_GATEUP, 2, 2, 64, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / 64, n_mg, ep);
+            e = m_tiles == 1 ? run_gemm<EPI_GATEUP, 1, 2, 64, 6>(ctx, tx, tg, tu, n_rows, k_in, I / 64, 1, ep)
+                             : run_gemm<EPI_GATEUP, 2, 2, 64, 4>(ctx, tx, tg, tu, n_rows, k_in, I / 64, n_mg, ep);
         if (e != cudaSuccess) return e;
     } else if (m_tiles == 2 && bn_gu == BN && ks1 == 4 &&
                splitk_clusters_fit<EPI_CGATEUP, 2, 2, BN, 3, 4>(ctx, I / BN)) {
-        e = run_gemm<EPI_CGATEUP, 2, 2, BN, 3, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, 1, ep, 4);
+        e = run_gemm<EPI_CGATEUP, 2, 2, BN, 3, 4>(ctx, tx, tg, tu, n_rows, k_in, I / BN, 1, ep, 4);
         if (e != cudaSuccess) return e;
     } else {
         if (bn_gu == BN)
-            e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 2, BN, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, 1, ep, ks1)
-                             : run_gemm<EPI_PARTIAL, 2, 2, BN, 3>(ctx, tx, tg, tu, n_rows, 2 * d, I / BN, n_mg, ep, ks1);
+            e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 2, BN, 4>(ctx, tx, tg, tu, n_rows, k_in, I / BN, 1, ep, ks1)
+                             : run_gemm<EPI_PARTIAL, 2, 2, BN, 3>(ctx, tx, tg, tu, n_rows, k_in, I / BN, n_mg, ep, ks1);
         else
-            e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 2, 64, 6>(ctx, tx, tg, tu, n_rows, 2 * d, I / 64, 1, ep, ks1)
-                             : run_gemm<EPI_PARTIAL, 2, 2, 64, 4>(ctx, tx, tg, tu, n_rows, 2 * d, I / 64, n_mg, ep, ks1);
+            e = m_tiles == 1 ? run_gemm<EPI_PARTIAL, 1, 2, 64, 6>(ctx, tx, tg, tu, n_rows, k_in, I / 64, 1, ep, ks1)
+                             : run_gemm<EPI_PARTIAL, 2, 2, 64, 4>(ctx, tx, tg, tu, n_rows, k_in, I / 64, n_mg, ep, ks1);
         if (e != cudaSuccess) return e;
         e = launch_swiglu_reduce(ctx, partial, ks1, n_rows, I, static_cast<__nv_bfloat16*>(A));
         if (e != cudaSuccess) return e;

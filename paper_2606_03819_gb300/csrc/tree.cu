@@ -8,62 +8,106 @@ namespace tf {
 namespace {
 
 // ------------------------------------------------------------------------------------------
-// x = [RMSNorm(h_{t+i}) * norm_h ; RMSNorm(Embd(prev)) * norm_e] for every stage-2 row
-// (Eq. 1, h~ first). One CTA per row; the embedding row is gathered by token id here, so
-// the candidate embeddings are never materialised on their own.
+// Inputs of stage-2 row `row` (R rows per sequence).
+//  TreeFlash (Eq. 1): row 0 refines depth 1 with the root token; row 1 + (i-2) M + m refines
+//  depth i with candidate m of depth i-1.
+//  Two previous tokens (the ablations' two-token variant): row 0 refines depth 1 with (x_t,
+//  x_{t-1}) = root_tok[2 sq], root_tok[2 sq + 1]; rows 1..M depth 2 with (candidate m of depth 1,
+//  x_t); row 1 + M + (i-3) M^2 + m1 M + m2 depth i >= 3 with (candidate m1 of depth i-1,
+//  candidate m2 of depth i-2).
+// The hidden-state index needs no kernel's output, so it is separate from the token reads.
 // ------------------------------------------------------------------------------------------
-template <typename T>
+__device__ __forceinline__ int stage2_row_hidden(int row, int R, int gamma, int M, bool two_prev) {
+    const int sq = row / R, r = row - sq * R;
+    if (!two_prev) return sq * gamma + stage2_hidden_index(r, M);
+    const int depth = r == 0 ? 1 : r <= M ? 2 : 3 + (r - 1 - M) / (M * M);
+    return sq * gamma + depth - 1;
+}
+// The previous token (p[0]) and, with two_prev, the one before it (p[1]).
+__device__ __forceinline__ void stage2_row_tokens(int row, int R, int gamma, int M, int K1, bool two_prev,
+                                                  const int32_t* root_tok, const int32_t* top_ids, int* p) {
+    const int sq = row / R, r = row - sq * R;
+    const int32_t* top = top_ids + static_cast<size_t>(sq) * gamma * K1;   // [gamma][K1] of this sequence
+    if (!two_prev) {
+        p[0] = r == 0 ? root_tok[sq] : top[((r - 1) / M) * K1 + (r - 1) % M];
+        return;
+    }
+    const int32_t* root = root_tok + 2 * static_cast<size_t>(sq);
+    if (r == 0) {
+        p[0] = root[0];
+        p[1] = root[1];
+    } else if (r <= M) {
+        p[0] = top[r - 1];
+        p[1] = root[0];
+    } else {
+        const int q = r - 1 - M, i = 3 + q / (M * M), w = q - (i - 3) * M * M;
+        p[0] = top[(i - 2) * K1 + w / M];
+        p[1] = top[(i - 3) * K1 + w % M];
+    }
+}
+
+// ------------------------------------------------------------------------------------------
+// x = [RMSNorm(h_{t+i}) * norm_h ; RMSNorm(Embd(prev)) * norm_e] for every stage-2 row
+// (Eq. 1, h~ first), and with NE = 2 a third part RMSNorm(Embd(token before prev)) * norm_e.
+// One CTA per row; the embedding rows are gathered by token id here, so the candidate
+// embeddings are never materialised on their own. hres (NE = 2): the row's hidden state.
+// ------------------------------------------------------------------------------------------
+template <typename T, int NE>
 __global__ void __launch_bounds__(256) gather_norm_kernel(const T* __restrict__ hidden, const T* __restrict__ embed,
                                                           const T* __restrict__ norm_h, const T* __restrict__ norm_e,
                                                           const int32_t* __restrict__ root_tok,
                                                           const int32_t* __restrict__ top_ids, int gamma, int M,
                                                           int K1, int R, int d, int V, float eps, T* __restrict__ X,
-                                                          int* status) {
+                                                          T* __restrict__ hres, int* status) {
     pdl_trigger();
     pdl_wait();
-    __shared__ float red[2][8];
+    __shared__ float red[1 + NE][8];
     const int row = blockIdx.x;
-    const int sq = row / R, r = row - sq * R;
-    const int hid = sq * gamma + stage2_hidden_index(r, M);
-    int tok = (r == 0) ? root_tok[sq] : top_ids[(static_cast<size_t>(sq) * gamma + (r - 1) / M) * K1 + (r - 1) % M];
-    if (tok < 0 || tok >= V) {
-        if (threadIdx.x == 0) set_status(status, TF_DEV_BAD_TOKEN);
-        tok = 0;
+    const int hid = stage2_row_hidden(row, R, gamma, M, NE == 2);
+    int tok[2] = {0, 0};
+    stage2_row_tokens(row, R, gamma, M, K1, NE == 2, root_tok, top_ids, tok);
+    const T* seg[1 + NE];
+    seg[0] = hidden + static_cast<size_t>(hid) * d;
+#pragma unroll
+    for (int j = 0; j < NE; ++j) {
+        if (tok[j] < 0 || tok[j] >= V) {
+            if (threadIdx.x == 0) set_status(status, TF_DEV_BAD_TOKEN);
+            tok[j] = 0;
+        }
+        seg[1 + j] = embed + static_cast<size_t>(tok[j]) * d;
     }
-    const T* h = hidden + static_cast<size_t>(hid) * d;
-    const T* e = embed + static_cast<size_t>(tok) * d;
-    float sh = 0.0f, se = 0.0f;
+    float sq[1 + NE];
+#pragma unroll
+    for (int j = 0; j <= NE; ++j) sq[j] = 0.0f;
     for (int k = threadIdx.x; k < d; k += blockDim.x) {
-        const float a = to_f32(h[k]), b = to_f32(e[k]);
-        sh = fmaf(a, a, sh);
-        se = fmaf(b, b, se);
+#pragma unroll
+        for (int j = 0; j <= NE; ++j) {
+            const float a = to_f32(seg[j][k]);
+            sq[j] = fmaf(a, a, sq[j]);
+        }
     }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        sh += __shfl_xor_sync(0xffffffffu, sh, o);
-        se += __shfl_xor_sync(0xffffffffu, se, o);
-    }
+    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+        for (int j = 0; j <= NE; ++j) sq[j] += __shfl_xor_sync(0xffffffffu, sq[j], o);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0) {
-        red[0][warp] = sh;
-        red[1][warp] = se;
+    if (lane == 0)
+#pragma unroll
+        for (int j = 0; j <= NE; ++j) red[j][warp] = sq[j];
+    __syncthreads();
+    if (threadIdx.x <= NE) {
+        float a = 0.0f;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) a += red[threadIdx.x][w];
+        red[threadIdx.x][0] = rsqrtf(a / d + eps);
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-        float a = 0.0f, b = 0.0f;
-        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
-            a += red[0][w];
-            b += red[1][w];
-        }
-        red[0][0] = rsqrtf(a / d + eps);
-        red[1][0] = rsqrtf(b / d + eps);
-    }
-    __syncthreads();
-    const float ih = red[0][0], ie = red[1][0];
-    T* xr = X + static_cast<size_t>(row) * 2 * d;
+    T* xr = X + static_cast<size_t>(row) * (1 + NE) * d;
     for (int k = threadIdx.x; k < d; k += blockDim.x) {
-        xr[k] = from_f32<T>(to_f32(h[k]) * ih * to_f32(norm_h[k]));
-        xr[d + k] = from_f32<T>(to_f32(e[k]) * ie * to_f32(norm_e[k]));
+        const float hk = to_f32(seg[0][k]);
+        xr[k] = from_f32<T>(hk * red[0][0] * to_f32(norm_h[k]));
+#pragma unroll
+        for (int j = 1; j <= NE; ++j) xr[j * d + k] = from_f32<T>(to_f32(seg[j][k]) * red[j][0] * to_f32(norm_e[k]));
+        if (NE == 2) hres[static_cast<size_t>(row) * d + k] = seg[0][k];
     }
 }
 
@@ -84,6 +128,7 @@ __global__ void __launch_bounds__(256) gather_norm_kernel(const T* __restrict__ 
 // ------------------------------------------------------------------------------------------
 struct TreeArgs {
     int gamma, M, K1, K2, B, V, mode, R;
+    int two_prev;      // child lists by the ablations' two-token rule; root_tok holds 2 tokens per sequence
     const int32_t* root_tok;
     const int32_t* top_ids;
     const float* top_logp;
@@ -110,6 +155,24 @@ __device__ __forceinline__ int mary_index(const int* topm, int dep, int M, int t
     const bool h1 = active && lane + 32 < M && t[lane + 32] == tok;
     const unsigned b0 = __ballot_sync(0xffffffffu, h0), b1 = __ballot_sync(0xffffffffu, h1);
     return b0 ? __ffs(b0) - 1 : (b1 ? 32 + __ffs(b1) - 1 : -1);
+}
+
+// Child list of a popped node under the two-previous-token rule: the node (depth dep, candidate
+// m of its depth, or m < 0 outside the M-ary tree) gets the row conditioned on its own token and
+// its parent's, 1 + m for dep = 1 and 1 + M + (dep - 2) M^2 + m M + mp for dep >= 2, mp the
+// parent's candidate index at depth dep - 1 (the parent was expanded, so it has one). o_tok holds
+// the tokens of the nodes placed so far, written by lane 0, which alone reads the parent's token.
+// Every lane must call it (ballots); returns -1 for a leaf.
+__device__ __forceinline__ int child_row_2prev(const int* topm, const int* o_tok, int M, int dep, int m, int par,
+                                               int lane) {
+    const bool deep = m >= 0 && dep >= 2;
+    int ptok = 0;
+    if (lane == 0 && deep) ptok = o_tok[par];
+    ptok = __shfl_sync(0xffffffffu, ptok, 0);
+    const int mp = mary_index(topm, deep ? dep - 1 : 1, M, ptok, lane, deep);
+    if (m < 0) return -1;
+    if (dep == 1) return 1 + m;
+    return mp >= 0 ? 1 + M + (dep - 2) * M * M + m * M + mp : -1;
 }
 
 __device__ __forceinline__ unsigned long long queue_key(float score, int depth, int parent) {
@@ -341,7 +404,7 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
         const int lane = tid;
         constexpr unsigned kFull = 0xffffffffu;
         int flags = 0;
-        const int root = a.root_tok[s];
+        const int root = a.root_tok[a.two_prev ? 2 * s : s];
         if (root < 0 || root >= a.V) flags |= TF_DEV_BAD_TOKEN;
         const int list_len = a.K2;
         if (lane == 0) {
@@ -396,6 +459,7 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
                 } else {
                     const int m = mary_index(topm, dep, a.M, tok, lane, true);
                     if (m >= 0) crow = ar ? 1 + (dep - 1) * a.M + m : dep;
+                    if (ar && a.two_prev) crow = child_row_2prev(topm, o_tok, a.M, dep, m, par, lane);
                 }
             }
             const bool sibling = rank + 1 < list_len;
@@ -470,7 +534,7 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
         const int lane = threadIdx.x;
         constexpr unsigned kFull = 0xffffffffu;
         int flags = 0;
-        const int root = a.root_tok[s];
+        const int root = a.root_tok[a.two_prev ? 2 * s : s];
         if (root < 0 || root >= a.V) flags |= TF_DEV_BAD_TOKEN;
         const int list_len = a.K2;
         unsigned long long key[S];
@@ -532,9 +596,10 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
             // expandable? (depth cap; M-ary rule)
             const bool deep_ok = dep < a.gamma;
             const int m = mary_index(t.topm, dep, a.M, tok, lane, deep_ok && a.mode != TF_MODE_MARGINAL);
-            const int crow = !deep_ok ? -1
-                             : a.mode == TF_MODE_MARGINAL ? dep
-                             : m >= 0 ? (ar ? 1 + (dep - 1) * a.M + m : dep) : -1;
+            int crow = !deep_ok ? -1
+                       : a.mode == TF_MODE_MARGINAL ? dep
+                       : m >= 0 ? (ar ? 1 + (dep - 1) * a.M + m : dep) : -1;
+            if (ar && a.two_prev) crow = child_row_2prev(t.topm, t.o_tok, a.M, dep, deep_ok ? m : -1, par, lane);
             if (tok < 0 || tok >= a.V) flags |= TF_DEV_BAD_TOKEN;
             if (!isfinite(sc)) flags |= TF_DEV_NONFINITE;
             const unsigned long long sib_key = sibling ? queue_key(psc + sib_lp, dep, par) : 0ull;
@@ -692,69 +757,77 @@ __device__ __forceinline__ __nv_bfloat16 bf16_round_sum(float r, float t) {
 //  - h * w is exact in fp32 (two 8-bit significands); (h w) * hi is rounded once and its
 //    rounding error recovered with an FMA, so (h w) / sqrt(mean + eps) is known as r + t to
 //    about 2^-47 relative, which decides the bf16 rounding (bf16_round_sum).
+template <int NE>
 __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
     const uint4* __restrict__ hidden, const uint4* __restrict__ embed, const uint4* __restrict__ norm_h,
     const uint4* __restrict__ norm_e, const int32_t* __restrict__ root_tok, const int32_t* __restrict__ top_ids,
-    int gamma, int M, int K1, int R, int d, int V, float eps, uint4* __restrict__ X, int* status) {
+    int gamma, int M, int K1, int R, int d, int V, float eps, uint4* __restrict__ X, uint4* __restrict__ hres,
+    int* status) {
     pdl_trigger();
     constexpr int kMaxPerThread = 4;          // d <= 256 * 8 * 4 = 8192
-    __shared__ double red[2][8];
-    __shared__ float scale[4];                // hi, lo of the hidden half; hi, lo of the embedding half
+    constexpr int NS = 1 + NE;                // parts of x: the hidden state, then NE embeddings
+    __shared__ double red[NS][8];
+    __shared__ float scale[2 * NS];           // hi, lo of 1 / sqrt(mean + eps) of every part
     const int row = blockIdx.x;
-    const int sq = row / R, r = row - sq * R;
-    const int hid = sq * gamma + stage2_hidden_index(r, M);
+    const int hid = stage2_row_hidden(row, R, gamma, M, NE == 2);
 
     const int dv = d / 8;
     // the hidden state is a step input (no kernel writes it): read before waiting for the
     // previous kernel, which produces the candidate tokens
     const uint4* h = hidden + static_cast<size_t>(hid) * dv;
-    uint4 hv[kMaxPerThread], ev[kMaxPerThread];
+    uint4 v[NS][kMaxPerThread];
 #pragma unroll
     for (int i = 0; i < kMaxPerThread; ++i) {
         const int c = threadIdx.x + i * 256;
-        if (c < dv) hv[i] = h[c];
+        if (c < dv) v[0][i] = h[c];
     }
     pdl_wait();
-    int tok = (r == 0) ? root_tok[sq] : top_ids[(static_cast<size_t>(sq) * gamma + (r - 1) / M) * K1 + (r - 1) % M];
-    if (tok < 0 || tok >= V) {
-        if (threadIdx.x == 0) set_status(status, TF_DEV_BAD_TOKEN);
-        tok = 0;
-    }
-    const uint4* e = embed + static_cast<size_t>(tok) * dv;
+    int tok[2] = {0, 0};
+    stage2_row_tokens(row, R, gamma, M, K1, NE == 2, root_tok, top_ids, tok);
 #pragma unroll
-    for (int i = 0; i < kMaxPerThread; ++i) {
-        const int c = threadIdx.x + i * 256;
-        if (c < dv) ev[i] = e[c];
+    for (int j = 0; j < NE; ++j) {
+        if (tok[j] < 0 || tok[j] >= V) {
+            if (threadIdx.x == 0) set_status(status, TF_DEV_BAD_TOKEN);
+            tok[j] = 0;
+        }
+        const uint4* e = embed + static_cast<size_t>(tok[j]) * dv;
+#pragma unroll
+        for (int i = 0; i < kMaxPerThread; ++i) {
+            const int c = threadIdx.x + i * 256;
+            if (c < dv) v[1 + j][i] = e[c];
+        }
     }
-    float sh = 0.0f, ch = 0.0f, se = 0.0f, ce = 0.0f;
+    float sum[NS], comp[NS];
+#pragma unroll
+    for (int j = 0; j < NS; ++j) sum[j] = comp[j] = 0.0f;
 #pragma unroll
     for (int i = 0; i < kMaxPerThread; ++i) {
         const int c = threadIdx.x + i * 256;
         if (c < dv) {
-            const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&hv[i]);
-            const __nv_bfloat16* eb = reinterpret_cast<const __nv_bfloat16*>(&ev[i]);
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const float a = __bfloat162float(hb[j]), b = __bfloat162float(eb[j]);
-                two_sum_acc(sh, ch, a * a);
-                two_sum_acc(se, ce, b * b);
+            for (int j = 0; j < NS; ++j) {
+                const __nv_bfloat16* b = reinterpret_cast<const __nv_bfloat16*>(&v[j][i]);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const float a = __bfloat162float(b[k]);
+                    two_sum_acc(sum[j], comp[j], a * a);
+                }
             }
         }
     }
-    double dh = static_cast<double>(sh) + static_cast<double>(ch);
-    double de = static_cast<double>(se) + static_cast<double>(ce);
+    double dsum[NS];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        dh += __shfl_xor_sync(0xffffffffu, dh, o);
-        de += __shfl_xor_sync(0xffffffffu, de, o);
-    }
+    for (int j = 0; j < NS; ++j) dsum[j] = static_cast<double>(sum[j]) + static_cast<double>(comp[j]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+        for (int j = 0; j < NS; ++j) dsum[j] += __shfl_xor_sync(0xffffffffu, dsum[j], o);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0) {
-        red[0][warp] = dh;
-        red[1][warp] = de;
-    }
+    if (lane == 0)
+#pragma unroll
+        for (int j = 0; j < NS; ++j) red[j][warp] = dsum[j];
     __syncthreads();
-    if (threadIdx.x < 2) {
+    if (threadIdx.x < NS) {
         double a = 0.0;
         for (int w = 0; w < 8; ++w) a += red[threadIdx.x][w];
         const double inv = 1.0 / sqrt(a / d + static_cast<double>(eps));
@@ -763,67 +836,71 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
         scale[2 * threadIdx.x + 1] = __double2float_rn(inv - static_cast<double>(hi));
     }
     __syncthreads();
-    const float ih = scale[0], ih_lo = scale[1], ie = scale[2], ie_lo = scale[3];
-    uint4* xr = X + static_cast<size_t>(row) * 2 * dv;
+    uint4* xr = X + static_cast<size_t>(row) * NS * dv;
 #pragma unroll
     for (int i = 0; i < kMaxPerThread; ++i) {
         const int c = threadIdx.x + i * 256;
         if (c < dv) {
             const uint4 wh = norm_h[c], we = norm_e[c];
-            const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&hv[i]);
-            const __nv_bfloat16* eb = reinterpret_cast<const __nv_bfloat16*>(&ev[i]);
-            const __nv_bfloat16* whb = reinterpret_cast<const __nv_bfloat16*>(&wh);
-            const __nv_bfloat16* web = reinterpret_cast<const __nv_bfloat16*>(&we);
-            uint4 oh, oe;
-            __nv_bfloat16* ohb = reinterpret_cast<__nv_bfloat16*>(&oh);
-            __nv_bfloat16* oeb = reinterpret_cast<__nv_bfloat16*>(&oe);
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const float ph = __bfloat162float(hb[j]) * __bfloat162float(whb[j]);
-                const float pe = __bfloat162float(eb[j]) * __bfloat162float(web[j]);
-                const float rh = ph * ih, re = pe * ie;
-                ohb[j] = bf16_round_sum(rh, fmaf(ph, ih_lo, fmaf(ph, ih, -rh)));
-                oeb[j] = bf16_round_sum(re, fmaf(pe, ie_lo, fmaf(pe, ie, -re)));
+            for (int j = 0; j < NS; ++j) {
+                const float is = scale[2 * j], is_lo = scale[2 * j + 1];
+                const __nv_bfloat16* b = reinterpret_cast<const __nv_bfloat16*>(&v[j][i]);
+                const __nv_bfloat16* wb = reinterpret_cast<const __nv_bfloat16*>(j == 0 ? &wh : &we);
+                uint4 o;
+                __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(&o);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const float p = __bfloat162float(b[k]) * __bfloat162float(wb[k]);
+                    const float r = p * is;
+                    ob[k] = bf16_round_sum(r, fmaf(p, is_lo, fmaf(p, is, -r)));
+                }
+                xr[j * dv + c] = o;
             }
-            xr[c] = oh;
-            xr[dv + c] = oe;
+            if (NE == 2) hres[static_cast<size_t>(row) * dv + c] = v[0][i];
         }
     }
 }
 
 cudaError_t launch_gather_norm(const Ctx& ctx, int dtype, const void* hidden, const void* embed, const void* norm_h,
                                const void* norm_e, const int32_t* root_tok, const int32_t* top_ids, int b, int gamma,
-                               int M, int K1, int d, int V, float eps, void* X) {
-    const int R = 1 + M * (gamma - 1);
+                               int M, int K1, int R, int two_prev, int d, int V, float eps, void* X, void* hres) {
     const int rows = b * R;
+    if (rows <= 0) return cudaSuccess;
+    if (two_prev && !hres) return cudaErrorInvalidValue;
     cudaError_t e;
     if (dtype == TF_BF16 && d % 8 == 0 && d <= 8192) {
-        e = launch_pdl(gather_norm_bf16x8_kernel, dim3(rows), dim3(256), 0, ctx.stream,
-                       static_cast<const uint4*>(hidden), static_cast<const uint4*>(embed),
-                       static_cast<const uint4*>(norm_h), static_cast<const uint4*>(norm_e), root_tok, top_ids, gamma,
-                       M, K1, R, d, V, eps, static_cast<uint4*>(X), ctx.status);
+        auto kern = two_prev ? gather_norm_bf16x8_kernel<2> : gather_norm_bf16x8_kernel<1>;
+        e = launch_pdl(kern, dim3(rows), dim3(256), 0, ctx.stream, static_cast<const uint4*>(hidden),
+                       static_cast<const uint4*>(embed), static_cast<const uint4*>(norm_h),
+                       static_cast<const uint4*>(norm_e), root_tok, top_ids, gamma, M, K1, R, d, V, eps,
+                       static_cast<uint4*>(X), static_cast<uint4*>(hres), ctx.status);
     } else if (dtype == TF_BF16) {
-        e = launch_pdl(gather_norm_kernel<__nv_bfloat16>, dim3(rows), dim3(256), 0, ctx.stream,
-                       static_cast<const __nv_bfloat16*>(hidden), static_cast<const __nv_bfloat16*>(embed),
-                       static_cast<const __nv_bfloat16*>(norm_h), static_cast<const __nv_bfloat16*>(norm_e), root_tok,
-                       top_ids, gamma, M, K1, R, d, V, eps, static_cast<__nv_bfloat16*>(X), ctx.status);
+        using B16 = __nv_bfloat16;
+        auto kern = two_prev ? gather_norm_kernel<B16, 2> : gather_norm_kernel<B16, 1>;
+        e = launch_pdl(kern, dim3(rows), dim3(256), 0, ctx.stream, static_cast<const B16*>(hidden),
+                       static_cast<const B16*>(embed), static_cast<const B16*>(norm_h), static_cast<const B16*>(norm_e),
+                       root_tok, top_ids, gamma, M, K1, R, d, V, eps, static_cast<B16*>(X), static_cast<B16*>(hres),
+                       ctx.status);
     } else {
-        e = launch_pdl(gather_norm_kernel<float>, dim3(rows), dim3(256), 0, ctx.stream,
-                       static_cast<const float*>(hidden), static_cast<const float*>(embed),
-                       static_cast<const float*>(norm_h), static_cast<const float*>(norm_e), root_tok, top_ids, gamma, M,
-                       K1, R, d, V, eps, static_cast<float*>(X), ctx.status);
+        auto kern = two_prev ? gather_norm_kernel<float, 2> : gather_norm_kernel<float, 1>;
+        e = launch_pdl(kern, dim3(rows), dim3(256), 0, ctx.stream, static_cast<const float*>(hidden),
+                       static_cast<const float*>(embed), static_cast<const float*>(norm_h),
+                       static_cast<const float*>(norm_e), root_tok, top_ids, gamma, M, K1, R, d, V, eps,
+                       static_cast<float*>(X), static_cast<float*>(hres), ctx.status);
     }
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_build_tree(const Ctx& ctx, int b, int gamma, int M, int K1, int K2, int B, int V, int mode, int R,
-                              const int32_t* root_tok, const int32_t* top_ids, const float* top_logp,
+                              int two_prev, const int32_t* root_tok, const int32_t* top_ids, const float* top_logp,
                               const int32_t* child_ids, const float* child_logp, int32_t* node_tok,
                               int32_t* node_parent, int32_t* node_depth, float* node_score, int32_t* dev_status,
                               const int32_t* root_pos, uint8_t* mask, int32_t* pos_ids) {
     if (mask && B + 1 > kFusedMaskMaxNodes) return cudaErrorInvalidValue;
-    TreeArgs a{gamma, M, K1, K2, B, V, mode, R, root_tok, top_ids, top_logp, child_ids, child_logp,
-               node_tok, node_parent, node_depth, node_score, dev_status, root_pos, mask, pos_ids};
+    TreeArgs a{gamma, M, K1, K2, B, V, mode, R, mode == TF_MODE_AR && two_prev ? 1 : 0, root_tok, top_ids, top_logp,
+               child_ids, child_logp, node_tok, node_parent, node_depth, node_score, dev_status, root_pos, mask,
+               pos_ids};
     const size_t fixed = tree_smem_fixed(B, gamma, M, mask != nullptr);
     const int rows_l = mode == TF_MODE_AR ? R : gamma;
     const int stride = mode == TF_MODE_AR ? K2 : K1;

@@ -49,17 +49,55 @@ def run_oracle(cfg, inp, emulate_bf16=False, seqs=None, W=None):
     seqs = range(cfg.batch) if seqs is None else seqs
     out = []
     for s in seqs:
+        prev = int(inp["root_prev"][s]) if inp.get("root_prev") is not None else None
         out.append(O.draft_sequence(H[s], int(inp["root_tok"][s]), int(inp["root_pos"][s]), W,
                                     M=cfg.M, K2=cfg.K2, B=cfg.B, temperature=cfg.temperature,
                                     eps=cfg.rms_eps, mode=cfg.mode, emulate_bf16=emulate_bf16,
-                                    keep=cfg.K2 if cfg.K2 < cfg.B else None, approx=cfg.approx))
+                                    keep=cfg.K2 if cfg.K2 < cfg.B else None, approx=cfg.approx,
+                                    root_prev=prev))
     return out
 
 
 def device_inputs(inp, device="cuda"):
+    """The GPU's inputs. With a token before each root (the two-previous-token approximator)
+    root_tok becomes the [b, 2] array (x_t, x_{t-1}) the C ABI takes in that mode."""
     keys = ("hidden", "lm_head", "embed", "norm_h", "norm_e", "w_gate", "w_up", "w_down", "w_lin",
             "root_tok", "root_pos")
-    return {k: inp[k].to(device).contiguous() for k in keys if inp.get(k) is not None}
+    out = {k: inp[k].to(device).contiguous() for k in keys if inp.get(k) is not None}
+    if inp.get("root_prev") is not None:
+        out["root_tok"] = torch.stack([inp["root_tok"], inp["root_prev"]], dim=1).to(device).contiguous()
+    return out
+
+
+def conditioning_keys(cfg, root_tok, top_ids, root_prev=None):
+    """Per stage-2 row, the key that identifies its conditioning: (depth index, previous token)
+    or, with two previous tokens, (depth index, previous token, the token before it)."""
+    if cfg.approx == "swiglu_2prev":
+        hid, p1, p2 = O.stage2_conditioning_2prev(cfg.gamma, cfg.M, root_tok, root_prev, top_ids)
+        return [(int(h), int(a), int(b)) for h, a, b in zip(hid, p1, p2)]
+    hid, prev = O.stage2_conditioning(cfg.gamma, cfg.M, root_tok, top_ids)
+    return [(int(h), int(p)) for h, p in zip(hid, prev)]
+
+
+def stage2_row_of(cfg, top_ids_s, tok, par, dep, i):
+    """Index of the stage-2 row node i's token was drawn from (TreeFlash mode), by the M-ary
+    candidate indices of its ancestors; asserts that its parent (and, with two previous tokens,
+    its grandparent) lies in the M-ary tree."""
+    M = cfg.M
+    if dep[i] == 1:
+        return 0
+    p = int(par[i])
+    cand = top_ids_s[dep[p] - 1, :M].tolist()
+    assert int(tok[p]) in cand, f"node {p} expanded outside the M-ary tree"
+    m = cand.index(int(tok[p]))
+    if cfg.approx != "swiglu_2prev":
+        return 1 + (dep[p] - 1) * M + m
+    if dep[p] == 1:
+        return 1 + m
+    gp = int(par[p])
+    gcand = top_ids_s[dep[gp] - 1, :M].tolist()
+    assert int(tok[gp]) in gcand, f"node {gp} expanded outside the M-ary tree"
+    return 1 + M + (dep[p] - 2) * M * M + m * M + gcand.index(int(tok[gp]))
 
 
 def run_gpu(cfg, dinp, drafter=None):
@@ -71,11 +109,13 @@ def run_gpu(cfg, dinp, drafter=None):
     res = {k: (v.cpu().numpy() if v is not None else None) for k, v in out.items()}
     res["flags"] = flags
     res["root_pos"] = dinp["root_pos"].cpu().numpy()
+    if dinp["root_tok"].dim() == 2:        # (x_t, x_{t-1}) per sequence
+        res["root_prev"] = dinp["root_tok"][:, 1].cpu().numpy()
     if cfg.mode == "ar":
         from paper_2606_03819_gb300 import binding as Bn
         views = (("X", Bn.TF_VIEW_X), ("A", Bn.TF_VIEW_A), ("hp", Bn.TF_VIEW_H_PRIME))
         for name, view in views:
-            if name == "A" and cfg.approx != "swiglu":
+            if name == "A" and cfg.approx == "linear":   # no SwiGLU intermediate
                 continue
             res[name] = Bn.tf_workspace_view(dims, dr.ws, view).double().cpu().numpy()
     return res
@@ -113,22 +153,22 @@ def compare(cfg, gpu, orc, tol_lp, tol_sel, check_structure=True, tol_lp2=None, 
             if i < g - 1 and O.topk_margin(o.s1_logp[i], M) > tol_sel:
                 assert set(gpu["top_ids"][s, i, :M].tolist()) == set(o.top_ids[i, :M].tolist()), \
                     f"seq {s} depth {i + 1}: top-M set differs"
-        # ---- stage 2, rows paired by (depth, previous token)
+        # ---- stage 2, rows paired by (depth, previous token(s))
         if cfg.mode == "ar":
-            hid, prev = O.stage2_conditioning(g, M, int(o.tree.tok[0]), o.top_ids)
-            okey = {(int(h), int(p)): r for r, (h, p) in enumerate(zip(hid, prev))}
-            ghid, gprev = O.stage2_conditioning(g, M, int(o.tree.tok[0]), gpu["top_ids"][s])
+            root = int(o.tree.tok[0])
+            rprev = int(gpu["root_prev"][s]) if gpu.get("root_prev") is not None else None
+            okey = {k: r for r, k in enumerate(conditioning_keys(cfg, root, o.top_ids, rprev))}
+            gkeys = conditioning_keys(cfg, root, gpu["top_ids"][s], rprev)
             if orc_round is not None:
-                ehid, eprev = O.stage2_conditioning(g, M, int(o.tree.tok[0]), orc_round[s].top_ids)
-                ekey = {(int(h), int(p)): r for r, (h, p) in enumerate(zip(ehid, eprev))}
-            for r, (h, p) in enumerate(zip(ghid, gprev)):
-                orow = okey.get((int(h), int(p)))
+                ekey = {k: r for r, k in enumerate(conditioning_keys(cfg, root, orc_round[s].top_ids, rprev))}
+            for r, key in enumerate(gkeys):
+                orow = okey.get(key)
                 if orow is None:
                     rep["rows_s2_skipped"] += 1
                     continue
                 tol_row = tol_lp2
                 if orc_round is not None:
-                    erow = ekey.get((int(h), int(p)))
+                    erow = ekey.get(key)
                     if erow is None:
                         rep["rows_s2_skipped"] += 1
                         continue
@@ -201,13 +241,7 @@ def _check_tree_valid(cfg, gpu, s):
         seen.add((p, int(tok[i])))
         # score = parent score + the GPU's own log-prob of this token in the child list used
         if cfg.mode == "ar":
-            if dep[i] == 1:
-                row = 0
-            else:
-                pt = int(tok[p])
-                cand = gpu["top_ids"][s, dep[p] - 1, : cfg.M].tolist()
-                assert pt in cand, f"seq {s} node {p} expanded outside the M-ary tree"
-                row = 1 + (dep[p] - 1) * cfg.M + cand.index(pt)
+            row = stage2_row_of(cfg, gpu["top_ids"][s], tok, par, dep, i)
             ids, lp = gpu["child_ids"][s, row], gpu["child_logp"][s, row]
         else:
             if cfg.mode == "marginal_mary" and dep[i] > 1:
@@ -242,16 +276,24 @@ def check_bf16_stagewise(cfg, inp, W, gpu):
     rep = {}
     g, M, d, I, R = cfg.gamma, cfg.M, cfg.d, cfg.I, cfg.R
     H = synth.to_f64(inp["hidden"])
-    rows_h, rows_prev = [], []
+    rows_h, rows_prev, rows_prev2 = [], [], []
     for s in range(cfg.batch):
-        hid, prev = O.stage2_conditioning(g, M, int(inp["root_tok"][s]), gpu["top_ids"][s])
+        if cfg.approx == "swiglu_2prev":
+            hid, prev, prev2 = O.stage2_conditioning_2prev(g, M, int(inp["root_tok"][s]), int(inp["root_prev"][s]),
+                                                           gpu["top_ids"][s])
+            rows_prev2.append(prev2)
+        else:
+            hid, prev = O.stage2_conditioning(g, M, int(inp["root_tok"][s]), gpu["top_ids"][s])
         rows_h.append(H[s][hid])
         rows_prev.append(prev)
     Hr = np.concatenate(rows_h)
     prev = np.concatenate(rows_prev)
-    # x: correctly rounded normalisations (computed in fp64 on the GPU)
-    x_ref = np.concatenate([O.bf16_round(O.rmsnorm(Hr, W["norm_h"], cfg.rms_eps)),
-                            O.bf16_round(O.rmsnorm(W["embed"][prev], W["norm_e"], cfg.rms_eps))], axis=1)
+    # x: correctly rounded normalisations (computed without per-element fp64 on the GPU)
+    parts = [O.bf16_round(O.rmsnorm(Hr, W["norm_h"], cfg.rms_eps)),
+             O.bf16_round(O.rmsnorm(W["embed"][prev], W["norm_e"], cfg.rms_eps))]
+    if rows_prev2:
+        parts.append(O.bf16_round(O.rmsnorm(W["embed"][np.concatenate(rows_prev2)], W["norm_e"], cfg.rms_eps)))
+    x_ref = np.concatenate(parts, axis=1)
     X = gpu["X"]
     rep["x_mismatch_frac"] = float((X != x_ref).mean())
     assert np.all(np.abs(X - x_ref) <= _ulp_bf16(x_ref)), "x off by more than one bf16 ulp"
@@ -327,7 +369,7 @@ def _gpu_lists_source(cfg, gpu, s):
     s2 = None
     if cfg.mode == "ar":
         s2 = np.stack([dense(gpu["child_ids"][s, r], gpu["child_logp"][s, r]) for r in range(cfg.R)])
-    return O.ChildSource(cfg.mode, cfg.gamma, cfg.M, gpu["top_ids"][s].astype(np.int64), s1, s2)
+    return O.ChildSource(cfg.mode, cfg.gamma, cfg.M, gpu["top_ids"][s].astype(np.int64), s1, s2, cfg.approx)
 
 
 def check_bf16_end_to_end(cfg, gpu, orc, orc_emul):

@@ -166,3 +166,27 @@ def test_linear_approximator_needs_w_lin_not_the_swiglu_weights(lib):
         ws_bytes = Bn.tf_workspace_size(d)
         st = lib.tf_ar_approx(ctypes.byref(c), ctypes.byref(w), fake, fake, fake, None, fake, ws_bytes, None)
         assert st == Bn.TF_ERR_INVALID_ARG, approx
+
+
+def test_two_prev_approximator_layout(lib):
+    # two previous tokens: 1 + M + M^2 (gamma - 2) stage-2 rows of width 3d, and room for a residual
+    # row per stage-2 row; the row count shows in the views (no GPU work: host-side layout only)
+    from paper_2606_03819_gb300 import binding as Bn
+    d1 = _dims()
+    d2 = _dims(approx="swiglu_2prev")
+    assert d2.R == 1 + 4 + 16 * 2 == 37 and d1.R == 13
+    n2 = Bn.tf_workspace_size(d2)
+    assert n2 > Bn.tf_workspace_size(d1)
+    buf = ctypes.create_string_buffer(n2 + 256)
+    ws = ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 256
+    p, nb = ctypes.c_void_p(), ctypes.c_size_t()
+    c = d2.c()
+    assert lib.tf_workspace_view(ctypes.byref(c), ws, n2, Bn.TF_VIEW_X, ctypes.byref(p), ctypes.byref(nb)) == 0
+    assert nb.value == 37 * 3 * 128 * 4
+    assert lib.tf_workspace_view(ctypes.byref(c), ws, n2, Bn.TF_VIEW_H_PRIME, ctypes.byref(p),
+                                 ctypes.byref(nb)) == 0
+    assert nb.value == 37 * 128 * 4
+    # gamma = 1 leaves one row; the marginal modes ignore the approximator kind
+    assert _dims(approx="swiglu_2prev", gamma=1).R == 1
+    assert Bn.tf_workspace_size(_dims(approx="swiglu_2prev", mode="marginal")) == \
+        Bn.tf_workspace_size(_dims(mode="marginal"))

@@ -247,6 +247,40 @@ def test_bf16_zero_linear_approximator_equals_mary_marginal_tree():
         np.testing.assert_array_equal(a[k], b[k], err_msg=k)
 
 
+# ------------------------------------------------------------------ "w/ 2-prev" approximator
+# (Sec. 4 "Model Design", Table 3): x = [h~ ; e(prev) ; e(token before prev)], one stage-2 row
+# per pair of M-ary candidates (1 + M + M^2 (gamma - 2) rows), the child list of a node chosen
+# by its own and its parent's candidate index; root_tok is [b, 2] = (x_t, x_{t-1}).
+
+
+def test_fp32_two_prev_approximator():
+    _, reps = check(synth.get_config("tiny_peaked", approx="swiglu_2prev"))
+    print(reps)
+
+
+@pytest.mark.parametrize("b,V", [(2, 2000), (4, 2304), (8, 2049)])
+def test_bf16_two_prev_approximator_small(b, V):
+    # 74 / 148 / 296 stage-2 rows: one, two and three M-tiles
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=b, V=V, approx="swiglu_2prev")
+    _, reps = check(cfg)
+    print(reps)
+
+
+def test_bf16_two_prev_approximator_cluster_split_k():
+    # gamma 4, M 8: 137 rows (two M-tiles), d = I = 512: gate/up with K = 3d and the down
+    # projection both split K over 4-CTA clusters; the residual rows come from the gather
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=1, d=512, I=512, V=3000, gamma=4, M=8, K2=16,
+                           B=32, approx="swiglu_2prev")
+    check(cfg)
+
+
+def test_fp32_two_prev_shared_queue_builder():
+    # B = 200 > 127: the builder with its queue in shared memory takes the two-token rule too
+    cfg = synth.get_config("tiny_peaked", V=4096, M=8, K2=200, B=200, approx="swiglu_2prev")
+    _, reps = check(cfg)
+    print(reps)
+
+
 # ------------------------------------------------------------------ full sizes (the measured shapes)
 
 _cache = {}
@@ -259,13 +293,15 @@ def _inputs(name):
     return _cache[name]
 
 
-@pytest.mark.parametrize("name", ["q8_b64", "q8_b32", "q8_b64_linear"])
+@pytest.mark.parametrize("name", ["q8_b64", "q8_b32", "q8_b64_linear", "q8_b32_2prev"])
 def test_full_size_qwen3_8b_shape(name):
     cfg = synth.get_config(name)
     gpu, reps = check(cfg, inp=_inputs(name))
     print(name, reps)
-    # depth-1 to depth-16 entropies ramp, so the tree must reach beyond depth 2
-    assert gpu["node_depth"][0].max() >= 3
+    # depth-1 to depth-16 entropies ramp, so the tree must reach beyond depth 2. With two previous
+    # tokens the random approximator moves q' far from q: the conditionals' favourites are rarely
+    # stage-1 candidates, so they stay leaves, and the oracle's own tree stops at depth 2
+    assert gpu["node_depth"][0].max() >= (2 if cfg.approx == "swiglu_2prev" else 3)
 
 
 @pytest.mark.parametrize("name", ["q8_b512", "q8_m64"])

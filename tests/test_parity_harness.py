@@ -51,3 +51,33 @@ def test_harness_rejects_planted_mistakes():
     for g in plants:
         with pytest.raises(AssertionError):
             parity.compare(cfg, g, orc, 1e-4, 1e-3)
+
+
+@pytest.mark.parametrize("approx", ["linear", "swiglu_2prev"])
+def test_harness_accepts_the_oracle_for_the_ablation_approximators(approx):
+    cfg = synth.get_config("tiny_peaked", batch=2, approx=approx)
+    inp = synth.make_inputs(cfg)
+    orc = parity.run_oracle(cfg, inp)
+    g = fake_gpu(cfg, orc, inp["root_pos"].numpy())
+    if approx == "swiglu_2prev":
+        g["root_prev"] = inp["root_prev"].numpy()
+        assert g["child_ids"].shape[1] == cfg.R == 37
+    rep = parity.compare(cfg, g, orc, 1e-4, 1e-3)
+    assert rep["rows_s2"] == 2 * cfg.R and rep["rows_s2_skipped"] == 0
+
+
+def test_harness_rejects_two_prev_rows_swapped_within_a_depth():
+    # rows (depth 3, m1 = 0, m2 = 0) and (depth 3, m1 = 0, m2 = 1) share the previous token and
+    # differ only in the token before it: pairing rows by the previous token alone would miss
+    # the swap
+    cfg = synth.get_config("tiny_peaked", batch=1, approx="swiglu_2prev", wd_std=2.0)
+    inp = synth.make_inputs(cfg)
+    orc = parity.run_oracle(cfg, inp)
+    g = fake_gpu(cfg, orc, inp["root_pos"].numpy())
+    g["root_prev"] = inp["root_prev"].numpy()
+    r = 1 + cfg.M
+    assert np.abs(orc[0].child_logp[r] - orc[0].child_logp[r + 1]).max() > 1e-3
+    for k in ("child_ids", "child_logp"):
+        g[k][0, [r, r + 1]] = g[k][0, [r + 1, r]]
+    with pytest.raises(AssertionError):
+        parity.compare(cfg, g, orc, 1e-4, 1e-3, check_structure=False)
