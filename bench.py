@@ -157,15 +157,16 @@ def kernel_source_hash():
     return h.hexdigest()[:16]
 
 
-def profiled_traffic():
+def profiled_traffic(workload: str):
     """dram bytes per launch of the LM-head pass from the committed ncu summary, or None when
-    the kernel sources changed since the counters were taken."""
+    the kernel sources changed since the counters were taken or the summary covers another
+    workload (it was scaled to the measured one)."""
     p = os.path.join(ROOT, "profiles", "lmhead_traffic.json")
     try:
         d = json.load(open(p))
     except (OSError, ValueError):
         return None
-    if d.get("source_hash") != kernel_source_hash():
+    if d.get("source_hash") != kernel_source_hash() or not str(d.get("scaled_to", "")).startswith(workload + " "):
         return None
     return d.get("dram_bytes_per_launch")
 
@@ -403,7 +404,7 @@ def run_gpu(args):
     timing = (f"CUDA events around each LM-head launch over {n_inst} further steps "
               f"({inst_ms_per_step * 1e3:.1f} us per step with the events)")
     roofline = lmhead_roofline(cfg, n1, n2, statistics.mean(lm1), statistics.mean(lm2), (peak, peak_kind),
-                               tensor_peak(), profiled_traffic(), timing)
+                               tensor_peak(), profiled_traffic(cfg.name), timing)
 
     # ---- end to end through the host-buffer entry point
     e2e = None

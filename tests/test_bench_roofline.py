@@ -40,3 +40,11 @@ def test_algorithmic_bytes_follow_the_approximator():
     # SwiGLU 2 I 2d + d I weights; linear d 2d; two tokens 2 I 3d + d I and more gathered rows
     assert base - lin == (2 * I * 2 * d + d * I - d * 2 * d) * 2
     assert two - base == (2 * I * d) * 2 + (3601 - 241) * d * 2
+
+
+def test_traffic_record_applies_to_its_own_workload_only():
+    # the committed ncu record was scaled to the measured workload; other workloads get null
+    rec = bench.profiled_traffic("q8_b64")
+    assert rec is None or rec > 1.2e9
+    assert bench.profiled_traffic("q8_b64_2prev") is None
+    assert bench.profiled_traffic("q8_b6") is None
