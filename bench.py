@@ -13,6 +13,8 @@ CUDA-event duration, from a second pass of the same steps with events around the
 launches. `gpu_launches` is the library's own count of kernels launched in the timed region. `e2e` is the same metric
 through tf_draft_tree_host with the step's inputs and outputs in pinned host memory, copies
 inside the timed region. `cpu_baseline` is the fp64 oracle on the host cores on a bounded sample.
+`torch_eager` times the same step written with PyTorch library calls (logits materialised,
+Part 2 as a host loop, as in the paper's implementation): a reference point, not a competitor.
 
 Multi-GPU (torchrun, one rank per GPU): every rank builds its own trees (independent replicas,
 no collective on the data path); value = all trees built / max over ranks of the timed span.
@@ -214,6 +216,79 @@ def lmhead_roofline(cfg, n1, n2, lm1_ms, lm2_ms, hbm_peak, tc_peak, traffic, tim
                peak_kind=f"{tc_kind} bf16 sustained")
     out["hbm"] = {"achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak}
     return out
+
+
+# ------------------------------------------------------------------------------ library-call reference
+
+def torch_eager_tree(cfg, w, hidden, root_tok):
+    """The drafting step written with PyTorch library calls, as a timing reference point (the
+    way the paper's own implementation runs Part 1, with Part 2 as a host loop; App. B):
+    matmuls in the tensors' dtype, log_softmax and topk on full fp32 logits (which reach
+    memory), Eq. 1 as torch ops, then the best-first selection with heapq on the host.
+    TreeFlash mode with the SwiGLU approximator only. Returns per sequence (tok, parent, depth,
+    score) lists of the B + 1 nodes in pop order. Not used by the library; runs on any device."""
+    import heapq
+
+    import torch
+    import torch.nn.functional as F
+    b, g, M, K2, B, d = cfg.batch, cfg.gamma, cfg.M, cfg.K2, cfg.B, cfg.d
+    K1 = max(M, K2)
+    W = w["lm_head"]
+    logp1 = torch.log_softmax((hidden.reshape(b * g, d) @ W.T).float() / cfg.temperature, dim=-1)
+    _, i1 = torch.topk(logp1, K1, dim=-1)
+    i1 = i1.view(b, g, K1)
+    # stage-2 rows: depth 1 on the root token, depth i on each candidate of depth i - 1
+    depth_of_row = torch.tensor([0] + [i for i in range(1, g) for _ in range(M)], device=hidden.device)
+    prev = torch.cat([root_tok.view(b, 1).long(), i1[:, : g - 1, :M].reshape(b, (g - 1) * M)], dim=1)
+    h_rows = hidden[:, depth_of_row, :]
+
+    def rms(x, wt):
+        xf = x.float()
+        return (xf * torch.rsqrt(xf.pow(2).mean(-1, keepdim=True) + cfg.rms_eps) * wt.float()).to(x.dtype)
+    x = torch.cat([rms(h_rows, w["norm_h"]), rms(w["embed"][prev], w["norm_e"])], dim=-1)
+    a = (F.silu((x @ w["w_gate"].T).float()) * (x @ w["w_up"].T).float()).to(x.dtype)
+    hp = (h_rows.float() + (a @ w["w_down"].T).float()).to(x.dtype)
+    logp2 = torch.log_softmax((hp.reshape(b * cfg.R, d) @ W.T).float() / cfg.temperature, dim=-1)
+    v2, i2 = torch.topk(logp2, K2, dim=-1)
+    top_m = i1[:, :, :M].cpu().tolist()
+    v2 = v2.view(b, cfg.R, K2).cpu().tolist()
+    i2 = i2.view(b, cfg.R, K2).cpu().tolist()
+    trees = []
+    for s in range(b):
+        toks, pars, deps, scores = [int(root_tok[s])], [-1], [0], [0.0]
+        heap = [(-v2[s][0][0], 1, 0, 0, 0, 0.0)]   # (-score, depth, parent, row, rank, parent score)
+        while heap and len(toks) < B + 1:
+            negs, dep, par, row, rank, psc = heapq.heappop(heap)
+            node = len(toks)
+            tok = i2[s][row][rank]
+            toks.append(tok)
+            pars.append(par)
+            deps.append(dep)
+            scores.append(-negs)
+            if rank + 1 < K2:
+                heapq.heappush(heap, (-(psc + v2[s][row][rank + 1]), dep, par, row, rank + 1, psc))
+            if dep < g and tok in top_m[s][dep - 1]:
+                crow = 1 + (dep - 1) * M + top_m[s][dep - 1].index(tok)
+                heapq.heappush(heap, (-(-negs + v2[s][crow][0]), dep + 1, node, crow, 0, -negs))
+        trees.append((toks, pars, deps, scores))
+    return trees
+
+
+def time_torch_eager(cfg, w, hidden, root_tok, steps: int):
+    """Wall-clock trees/s of torch_eager_tree on the GPU (each step ends with the host loop,
+    so it synchronises)."""
+    import torch
+    for _ in range(2):
+        torch_eager_tree(cfg, w, hidden, root_tok)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        torch_eager_tree(cfg, w, hidden, root_tok)
+    torch.cuda.synchronize()
+    t = (time.perf_counter() - t0) / steps
+    return {"value": cfg.batch / t, "unit": "trees/s", "ms_per_step": t * 1e3, "steps": steps,
+            "what": "torch library calls on the GPU (bf16 matmuls, fp32 logits in HBM, log_softmax, topk) "
+                    "plus a heapq best-first loop on the host; a reference point, not the product path"}
 
 
 # ------------------------------------------------------------------------------ oracle timing
@@ -438,6 +513,14 @@ def run_gpu(args):
         e2e = {"value": cfg.batch * args.e2e_steps * world / t_e2e, "unit": "trees/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
+    # ---- the same step with torch library calls (rank 0, N = 1; SwiGLU TreeFlash mode only)
+    eager = None
+    if rank == 0 and world == 1 and args.torch_eager_steps > 0 and cfg.mode == "ar" and cfg.approx == "swiglu":
+        try:
+            eager = time_torch_eager(cfg, d, H, d["root_tok"], args.torch_eager_steps)
+        except Exception as exc:   # a reference point must not cost the measured line
+            eager = {"error": f"{type(exc).__name__}: {exc}"[:200]}
+
     # ---- CPU baseline: the oracle on the host cores (rank 0, N = 1 only)
     cpu = None
     if rank == 0 and world == 1 and args.cpu_baseline_s > 0:
@@ -466,7 +549,7 @@ def run_gpu(args):
                           "peak_kind": peak_kind},
         "roofline": roofline,
         "clocks": clocks, "e2e": e2e, "gpu_launches": gpu_launches,
-        "cpu_baseline": cpu, "device_flags": flags,
+        "cpu_baseline": cpu, "torch_eager": eager, "device_flags": flags,
     }
     print(json.dumps(line), flush=True)
 
@@ -480,6 +563,8 @@ def main():
     ap.add_argument("--workload", default=WORKLOAD,
                     help="synthetic workload (synth.CONFIGS); default the measured Qwen3-8B-shape B=64 step")
     ap.add_argument("--e2e-steps", type=int, default=300)
+    ap.add_argument("--torch-eager-steps", type=int, default=20,
+                    help="steps of the torch library-call reference point (0 = skip)")
     ap.add_argument("--cpu-baseline-s", type=float, default=20.0,
                     help="approximate seconds of oracle work for the cpu_baseline sample (0 = skip)")
     args = ap.parse_args()

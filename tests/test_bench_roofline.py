@@ -48,3 +48,23 @@ def test_traffic_record_applies_to_its_own_workload_only():
     assert rec is None or rec > 1.2e9
     assert bench.profiled_traffic("q8_b64_2prev") is None
     assert bench.profiled_traffic("q8_b6") is None
+
+
+def test_torch_eager_reference_builds_the_oracles_tree():
+    # the library-call reference point of bench.py computes the same tree as the oracle (fp32 on
+    # the CPU here; on the GPU it runs in the workload's dtype)
+    import numpy as np
+    import torch
+
+    import parity
+    for batch, seed in ((1, 0), (3, 4)):
+        cfg = synth.get_config("tiny_peaked", batch=batch, seed=seed)
+        inp = synth.make_inputs(cfg)
+        w = {k: v for k, v in inp.items() if isinstance(v, torch.Tensor)}
+        trees = bench.torch_eager_tree(cfg, w, inp["hidden"], inp["root_tok"])
+        orc = parity.run_oracle(cfg, inp)
+        for s, (tok, par, dep, score) in enumerate(trees):
+            np.testing.assert_array_equal(tok, orc[s].tree.tok)
+            np.testing.assert_array_equal(par, orc[s].tree.parent)
+            np.testing.assert_array_equal(dep, orc[s].tree.depth)
+            np.testing.assert_allclose(score, orc[s].tree.score, atol=1e-4)
