@@ -338,6 +338,27 @@ class OracleSample:
         return t, full, Vs
 
 
+def cpu_model() -> str:
+    """The host CPU's model name (x86 "model name"; on Arm the implementer / part codes)."""
+    try:
+        info = open("/proc/cpuinfo").read().splitlines()
+    except OSError:
+        info = []
+    for key in ("model name", "Model name"):
+        for line in info:
+            if line.startswith(key):
+                return line.split(":", 1)[1].strip()
+    fields = {}
+    for line in info:
+        if ":" in line:
+            k, v = (x.strip() for x in line.split(":", 1))
+            fields.setdefault(k, v)
+    if "CPU part" in fields:
+        return f"Arm implementer {fields.get('CPU implementer', '?')} part {fields['CPU part']}"
+    import platform
+    return platform.machine()
+
+
 def cpu_threads():
     for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
         if os.environ.get(k, "").isdigit():
@@ -376,7 +397,8 @@ def run_reference(args):
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": cfg.name, "batch": cfg.batch, "d": cfg.d, "V": cfg.V, "I": cfg.I,
                        "gamma": cfg.gamma, "M": cfg.M, "K2": cfg.K2, "B": cfg.B, "approx": cfg.approx},
-            "cpu_baseline": {"value": value, "unit": "trees/s", "cores": cores, "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": value, "unit": "trees/s", "cores": cores, "cpu_model": cpu_model(),
+                             "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "trees/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -528,7 +550,8 @@ def run_gpu(args):
         _, full_est, _ = orc.run(1 / 64)
         frac = min(1.0, max(1 / 64, args.cpu_baseline_s / max(full_est, 1e-3)))
         t, full, Vs = orc.run(frac)
-        cpu = {"value": 1.0 / full, "unit": "trees/s", "cores": cpu_threads(), "kind": "oracle",
+        cpu = {"value": 1.0 / full, "unit": "trees/s", "cores": cpu_threads(), "cpu_model": cpu_model(),
+               "kind": "oracle",
                "sample": f"fp64 numpy oracle, 1 sequence, vocabulary cut to {Vs} of {cfg.V} "
                          f"({t:.1f} s), LM-head/softmax/sort time scaled to the full V"}
 

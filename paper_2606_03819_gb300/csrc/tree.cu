@@ -76,24 +76,24 @@ __global__ void __launch_bounds__(256) gather_norm_kernel(const T* __restrict__ 
         }
         seg[1 + j] = embed + static_cast<size_t>(tok[j]) * d;
     }
-    float sq[1 + NE];
+    float sumsq[1 + NE];
 #pragma unroll
-    for (int j = 0; j <= NE; ++j) sq[j] = 0.0f;
+    for (int j = 0; j <= NE; ++j) sumsq[j] = 0.0f;
     for (int k = threadIdx.x; k < d; k += blockDim.x) {
 #pragma unroll
         for (int j = 0; j <= NE; ++j) {
             const float a = to_f32(seg[j][k]);
-            sq[j] = fmaf(a, a, sq[j]);
+            sumsq[j] = fmaf(a, a, sumsq[j]);
         }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1)
 #pragma unroll
-        for (int j = 0; j <= NE; ++j) sq[j] += __shfl_xor_sync(0xffffffffu, sq[j], o);
+        for (int j = 0; j <= NE; ++j) sumsq[j] += __shfl_xor_sync(0xffffffffu, sumsq[j], o);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0)
 #pragma unroll
-        for (int j = 0; j <= NE; ++j) red[j][warp] = sq[j];
+        for (int j = 0; j <= NE; ++j) red[j][warp] = sumsq[j];
     __syncthreads();
     if (threadIdx.x <= NE) {
         float a = 0.0f;
