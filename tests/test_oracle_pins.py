@@ -491,6 +491,29 @@ def test_oracle_matches_frozen_golden():
         np.testing.assert_allclose(res.tree.score, g["score"], rtol=1e-12)
 
 
+def test_oracle_variants_match_frozen_golden():
+    # the same guard for the ablations' approximators (tests/golden/tiny_variants_seed0.json)
+    import json
+    import os
+    import synth
+    path = os.path.join(os.path.dirname(__file__), "golden", "tiny_variants_seed0.json")
+    gold = json.load(open(path))
+    assert set(gold) == {"tiny_peaked/linear", "tiny_peaked/swiglu_2prev"}
+    for key, g in gold.items():
+        name, approx = key.split("/")
+        cfg = synth.get_config(name, approx=approx)
+        inp = synth.make_inputs(cfg)
+        W = O.weights_f64(inp, synth.to_f64)
+        prev = int(inp["root_prev"][0]) if "root_prev" in inp else None
+        res = O.draft_sequence(synth.to_f64(inp["hidden"])[0], int(inp["root_tok"][0]),
+                               int(inp["root_pos"][0]), W, M=cfg.M, K2=cfg.K2, B=cfg.B, approx=approx,
+                               root_prev=prev)
+        assert res.tree.tok.tolist() == g["tok"]
+        assert res.tree.parent.tolist() == g["parent"]
+        np.testing.assert_allclose(res.tree.score, g["score"], rtol=1e-12)
+        np.testing.assert_allclose(res.child_logp[0], g["child_logp_row0"], rtol=1e-12)
+
+
 # ------------------------------------------------------------------ verification walk
 
 
