@@ -172,7 +172,8 @@ tf_status tf_stage1_marginals(const tf_dims* dims, const tf_weights* w, const vo
  *   row 1 + m:                      depth 2, tokens (x^(m)_{t+1}, x_t)
  *   row 1 + M + (i-3) M^2 + m1 M + m2: depth i >= 3, tokens (x^(m1)_{t+i-1}, x^(m2)_{t+i-2}).
  *  hidden     [b, gamma, d] dtype (as in stage 1)
- *  root_tok   [b] int32: the last accepted token x_t of each sequence
+ *  root_tok   [b] int32: the last accepted token x_t of each sequence ([b, 2] = (x_t, x_{t-1})
+ *             with TF_APPROX_SWIGLU_2PREV)
  *  top_ids    [b, gamma, K1] int32: stage-1 output (the first M per depth are used)
  *  child_ids  [b, R, K2] int32 out, child_logp [b, R, K2] float out (exact log-softmax).
  * h' is kept in the workspace (bf16 path: rounded to bf16, as the MLP's output type).
@@ -191,8 +192,8 @@ tf_status tf_stage2_ar_approx(const tf_dims* dims, const tf_weights* w, const vo
  * at most K2 children (exact when K2 >= B). With TF_APPROX_SWIGLU_2PREV a node of depth i whose
  * token is x^(m)_{t+i} and whose parent's token is x^(m')_{t+i-1} takes row
  * 1 + M + (i-2) M^2 + m M + m' (row 1 + m at depth 1), and root_tok is [b, 2] (x_t first).
- * child_ids/child_logp may be NULL in the marginal modes. Outputs [b, B+1]: node 0 is the root (token root_tok, parent -1, depth 0, score 0);
- * nodes follow in pop order, so parent < child. Missing nodes (underfull universe) have
+ * child_ids/child_logp may be NULL in the marginal modes. Outputs [b, B+1]: node 0 is the
+ * root (token x_t, parent -1, depth 0, score 0); nodes follow in pop order, so parent < child. Missing nodes (underfull universe) have
  * token/parent/depth -1 and score -inf, and set TF_DEV_UNDERFULL.
  *  dev_status [b] int32 out: TF_DEV_* bits per sequence (overwritten, not OR-ed). */
 tf_status tf_build_tree(const tf_dims* dims, const int32_t* root_tok,
@@ -225,7 +226,8 @@ tf_status tf_build_tree_mask(const tf_dims* dims, const int32_t* root_tok, const
  * makes the copies asynchronous): copies hidden/root_tok/root_pos to the device, runs stage 1,
  * stage 2 (TF_MODE_AR) and tf_build_tree_mask, copies the tree, mask and status back, and
  * synchronises `stream`.
- * Host inputs: hidden [b, gamma, d] dtype, root_tok [b], root_pos [b]. Host outputs:
+ * Host inputs: hidden [b, gamma, d] dtype, root_tok [b] ([b, 2] with TF_APPROX_SWIGLU_2PREV),
+ * root_pos [b]. Host outputs:
  * node_tok, node_parent, node_depth [b, B+1] int32, node_score [b, B+1] float,
  * mask [b, B+1, B+1] uint8, pos_ids [b, B+1] int32, dev_status [b] int32 (per-sequence bits
  * OR-ed with the workspace status word). Weights stay on the device. The workspace size is
