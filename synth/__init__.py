@@ -103,6 +103,9 @@ CONFIGS = {
     # ablation): 1 + M + M^2 (gamma - 2) = 905 / 3601 stage-2 rows
     "q8_b32_2prev": Config("q8_b32_2prev", batch=1, M=8, K2=32, B=32, approx="swiglu_2prev", **_Q8),
     "q8_b64_2prev": Config("q8_b64_2prev", batch=1, M=16, K2=64, B=64, approx="swiglu_2prev", **_Q8),
+    # the q8_b64 step with the approximator width the paper's parameter counts imply for a
+    # Qwen3-8B verifier (its intermediate size, I = 12288)
+    "q8_b64_paper_i": Config("q8_b64_paper_i", batch=1, M=16, K2=64, B=64, **dict(_Q8, I=12288)),
     # the q8_b64 step with the vocabulary cut to 32768 (W_lm 268 MB, still twice the L2):
     # small enough for multi-pass profiler captures
     "prof_v32k": Config("prof_v32k", batch=1, M=16, K2=64, B=64, **dict(_Q8, V=32768)),

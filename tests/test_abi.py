@@ -190,3 +190,33 @@ def test_two_prev_approximator_layout(lib):
     assert _dims(approx="swiglu_2prev", gamma=1).R == 1
     assert Bn.tf_workspace_size(_dims(approx="swiglu_2prev", mode="marginal")) == \
         Bn.tf_workspace_size(_dims(mode="marginal"))
+
+
+def test_view_and_mode_checks_before_any_gpu_work(lib):
+    # host-only checks: the SwiGLU intermediate view is empty for the linear approximator; the
+    # approximator calls need TreeFlash mode; the merge's k is bounded by 512 and V
+    from paper_2606_03819_gb300 import binding as Bn
+    d = _dims(approx="linear")
+    n = Bn.tf_workspace_size(d)
+    buf = ctypes.create_string_buffer(n + 256)
+    ws = ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 256
+    p, nb = ctypes.c_void_p(), ctypes.c_size_t()
+    c = d.c()
+    assert lib.tf_workspace_view(ctypes.byref(c), ws, n, Bn.TF_VIEW_A, ctypes.byref(p), ctypes.byref(nb)) == 0
+    assert nb.value == 0
+    assert lib.tf_workspace_view(ctypes.byref(c), ws, n, 99, ctypes.byref(p), ctypes.byref(nb)) == \
+        Bn.TF_ERR_INVALID_ARG
+    marg = _dims(mode="marginal")
+    cm = marg.c()
+    nm = Bn.tf_workspace_size(marg)
+    w = Bn.TfWeights(*[ws for _ in Bn.WEIGHT_KEYS])
+    assert lib.tf_ar_approx(ctypes.byref(cm), ctypes.byref(w), ws, ws, ws, None, ws, nm, None) == \
+        Bn.TF_ERR_INVALID_ARG
+    assert lib.tf_workspace_h_prime(ctypes.byref(cm), ws, nm, ctypes.byref(p)) == Bn.TF_ERR_INVALID_ARG
+    assert lib.tf_workspace_view(ctypes.byref(cm), ws, nm, Bn.TF_VIEW_X, ctypes.byref(p),
+                                 ctypes.byref(nb)) == Bn.TF_ERR_INVALID_ARG
+    # a workspace one byte short, or misaligned, is refused
+    assert lib.tf_workspace_view(ctypes.byref(c), ws, n - 1, Bn.TF_VIEW_X, ctypes.byref(p),
+                                 ctypes.byref(nb)) == Bn.TF_ERR_WORKSPACE
+    assert lib.tf_workspace_view(ctypes.byref(c), ws + 16, n, Bn.TF_VIEW_X, ctypes.byref(p),
+                                 ctypes.byref(nb)) == Bn.TF_ERR_WORKSPACE
