@@ -59,7 +59,7 @@ class Config:
     def R(self) -> int:
         """Stage-2 rows per sequence: one for depth 1, M for each depth 2..gamma (with two
         previous tokens: M for depth 2 and M^2 for each depth 3..gamma)."""
-        if self.approx == "swiglu_2prev":
+        if self.approx == "swiglu_2prev" and self.mode == "ar":
             return 1 if self.gamma == 1 else 1 + self.M + self.M * self.M * (self.gamma - 2)
         return 1 + self.M * (self.gamma - 1)
 
@@ -200,7 +200,7 @@ def make_inputs(cfg: Config, seed: Optional[int] = None) -> dict:
                root_tok=root_tok, root_pos=root_pos, h_scale=scales)
     if cfg.approx == "linear":
         out["w_lin"] = _randn(g, (d, 2 * d), cfg.wd_std, dt)
-    elif cfg.approx == "swiglu_2prev":
+    elif cfg.approx == "swiglu_2prev" and cfg.mode == "ar":
         out["w_gate"] = torch.cat([w_gate, _randn(g, (I, d), cfg.w_std, dt)], dim=1).contiguous()
         out["w_up"] = torch.cat([w_up, _randn(g, (I, d), cfg.w_std, dt)], dim=1).contiguous()
         out["root_prev"] = torch.randint(0, V, (cfg.batch,), generator=g, dtype=torch.int64).to(torch.int32)
