@@ -21,11 +21,14 @@
 //               the two warps of a group on the same lanes split the columns in halves.
 // A work unit is (N tile, group of MT M-tiles). With MT = 2 both slots hold one unit (M-tile j
 // in slot j); with MT = 1 consecutive units alternate slots so the epilogue of one overlaps the
-// MMAs of the next. With clusters of CL = 2 CTAs (the LM head over more than 128 rows), units
-// are dealt to clusters, CTA r of a cluster takes M-tile r of the unit's pair, and each CTA
-// loads half of the unit's weight tile and multicasts it to both; a stage is free again once
-// both CTAs' MMAs have consumed it. Every wait is bounded: after a time limit the kernel raises TF_DEV_TIMEOUT,
-// drains its in-flight copies and MMAs, frees TMEM and returns.
+// MMAs of the next. With clusters of CL = 2 CTAs (the LM head over more than 128 rows) the two
+// CTAs are a tcgen05 CTA pair: units are dealt to clusters, CTA r of a cluster stages M-tile r of
+// the unit's pair of M-tiles and weight rows [128 r, 128 r + 128) of the unit's 256-row weight
+// tile, and the even CTA issues one cta_group::2 MMA (M = 256, N = 256) per K slice that reads
+// both CTAs' shared memory and writes each CTA's 128 rows into its own TMEM. W is read once, each
+// CTA stages 32 KB per stage instead of 48 KB, and each keeps one TMEM slot per unit, so its
+// epilogue overlaps the next unit's MMAs. Every wait is bounded: after a time limit the kernel
+// raises TF_DEV_TIMEOUT, drains its in-flight copies and MMAs, frees TMEM and returns.
 #include <cuda.h>
 #include <math.h>
 
@@ -73,11 +76,13 @@ __device__ __forceinline__ Unit decode_unit(int u, int n_mgroups, int k_splits) 
     return w;
 }
 
-template <int MT, int NB, int BN, int STAGES>
+// PAIR: a CTA of a cta_group::2 pair, which stages half of the weight tile (BN / 2 rows).
+template <int MT, int NB, int BN, int STAGES, bool PAIR = false>
 struct TileCfg {
     static constexpr int kABytes = kBM * kBK * 2;
-    static constexpr int kBBytes = BN * kBK * 2;
-    static constexpr int kStageBytes = MT * kABytes + NB * kBBytes;
+    static constexpr int kBBytes = BN * kBK * 2;                    // the whole weight tile of a stage
+    static constexpr int kBBytesCta = PAIR ? kBBytes / 2 : kBBytes;  // the part this CTA stages
+    static constexpr int kStageBytes = MT * kABytes + NB * kBBytesCta;
     static constexpr int kBarrierBytes = 256;
     static constexpr int kSmemBytes = STAGES * kStageBytes + kBarrierBytes + 1024;
     static_assert(NB * BN <= 256, "one accumulator slot is 256 TMEM columns");
@@ -148,15 +153,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_w0,
                const __grid_constant__ CUtensorMap tmap_w1, int n_rows, int K, int n_ntiles,
                int n_mgroups, int k_splits, int w_stream_once, EpiParams ep, int* status) {
-    using C = TileCfg<MT, NB, BN, STAGES>;
-    // Two kinds of cluster: kMulticast, two CTAs on two M-tiles sharing each weight tile by TMA
-    // multicast; kSplitK, CL CTAs on the CL K-ranges of one output tile (one tile per cluster),
-    // whose accumulators are summed through distributed shared memory.
+    // Two kinds of cluster: kPair, a CTA pair on two M-tiles sharing each weight tile through
+    // cta_group::2 MMAs; kSplitK, CL CTAs on the CL K-ranges of one output tile (one tile per
+    // cluster), whose accumulators are summed through distributed shared memory.
     constexpr bool kSplitK = EPI == EPI_CGATEUP || EPI == EPI_CDOWN;
-    constexpr bool kMulticast = CL > 1 && !kSplitK;
-    static_assert(CL == 1 || kSplitK || (CL == 2 && NB == 1), "clusters of two share one weight operand");
+    constexpr bool kPair = CL > 1 && !kSplitK;
+    using C = TileCfg<MT, NB, BN, STAGES, kPair>;
+    static_assert(CL == 1 || kSplitK || (CL == 2 && NB == 1 && MT == 1), "a CTA pair shares one weight operand");
     static_assert(!kSplitK || (CL == 4 && MT == 2 && BN == 128), "cluster split-K: 4 K-ranges of a 256 x 128 tile");
-    constexpr uint16_t kClusterMask = static_cast<uint16_t>((1u << CL) - 1u);
     pdl_trigger();
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -171,12 +175,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    // Units are dealt to clusters. Multicast: CTA `crank` of a cluster takes M-tile group member
-    // crank of every unit. Split-K: a unit is an output tile and CTA crank takes K-range crank.
-    // With CL = 1 a cluster is one CTA.
+    // Units are dealt to clusters. Pair: CTA `crank` of a cluster takes M-tile group member crank
+    // of every unit. Split-K: a unit is an output tile and CTA crank takes K-range crank. With
+    // CL = 1 a cluster is one CTA.
     const int n_units = kSplitK ? n_ntiles * n_mgroups : n_ntiles * n_mgroups * k_splits;
     const int crank = CL > 1 ? static_cast<int>(ptx::cluster_ctarank()) : 0;
-    const int m_cl = kMulticast ? CL : 1, m_rank = kMulticast ? crank : 0;   // M-tiles of a cluster, this CTA's
+    const int m_cl = kPair ? CL : 1, m_rank = kPair ? crank : 0;   // M-tiles of a cluster, this CTA's
+    const bool leader = !kPair || crank == 0;                     // the pair's MMA issuer
     const int cid = CL > 1 ? static_cast<int>(ptx::cluster_id_x()) : static_cast<int>(blockIdx.x);
     const int ncl = CL > 1 ? static_cast<int>(ptx::cluster_count_x()) : static_cast<int>(gridDim.x);
     const int nk = K / kBK / k_splits;      // K-steps per unit (K % (64 * k_splits) == 0)
@@ -184,28 +189,48 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         if constexpr (kSplitK) return Unit{u / n_mgroups, u % n_mgroups, crank};
         return decode_unit(u, n_mgroups, k_splits);
     };
+    // shared::cluster address of this CTA's barrier `bar` as seen at the same offset in the pair's
+    // even CTA (pair mode: the barriers the issuer waits on) or in the odd one
+    auto in_leader = [&](uint64_t* bar) {
+        return kPair && crank != 0 ? ptx::mapa_shared(ptx::smem_u32(bar), 0) : ptx::smem_u32(bar);
+    };
+    auto in_peer = [&](uint64_t* bar) { return ptx::mapa_shared(ptx::smem_u32(bar), 1); };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             ptx::mbar_init(&full[s], 1);
-            ptx::mbar_init(&empty[s], m_cl);   // freed once every CTA sharing the stage has consumed it
+            ptx::mbar_init(&empty[s], 1);
         }
         for (int g = 0; g < 2; ++g) {
             ptx::mbar_init(&tfull[g], 1);
-            ptx::mbar_init(&tempty[g], 32 * kEpiWarps / 2);
+            // pair: one arrival per epilogue warp of both CTAs (used in the even CTA only)
+            ptx::mbar_init(&tempty[g], kPair ? 2 * (kEpiWarps / 2) : 32 * kEpiWarps / 2);
         }
         ptx::mbar_init(drain, 1);
         *abort_flag = 0;
         ptx::fence_barrier_init();
     }
-    if (warp == 1) {
-        ptx::tmem_alloc(tmem_slot, 512);
-        ptx::tmem_relinquish();
+    if constexpr (kPair) {
+        // both CTAs of the pair are running and their barriers exist before the collective
+        // allocation and before either CTA signals the other's barriers
+        ptx::cluster_sync();
+        if (warp == 1) {
+            ptx::tmem_alloc_pair(tmem_slot, 512);
+            ptx::tmem_relinquish_pair();
+        }
+        ptx::tc_fence_before();
+        __syncthreads();
+        ptx::tc_fence_after();
+    } else {
+        if (warp == 1) {
+            ptx::tmem_alloc(tmem_slot, 512);
+            ptx::tmem_relinquish();
+        }
+        ptx::tc_fence_before();
+        __syncthreads();
+        if constexpr (CL > 1) ptx::cluster_sync();   // the peers' barriers exist before any remote access
+        ptx::tc_fence_after();
     }
-    ptx::tc_fence_before();
-    __syncthreads();
-    if constexpr (CL > 1) ptx::cluster_sync();   // the peers' barriers exist before any multicast
-    ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
     if (!(warp == 0 && lane == 0)) pdl_wait();   // the producer waits after its weight prefetch
     // a call's status word starts at zero; cleared here, after every earlier kernel has finished,
@@ -220,12 +245,21 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             if (NB == 2) ptx::prefetch_tmap(&tmap_w1);
             const uint64_t pol_x = ptx::policy_evict_last();
             const uint64_t pol_w = w_stream_once ? ptx::policy_evict_first() : ptx::policy_evict_last();
-            // Weight tiles of one stage. In a cluster each CTA fetches its share of the rows and
-            // multicasts it to every CTA of the cluster (tmap_w0's box is BN / CL rows high).
+            // Pair: both CTAs' copies of a stage complete on the even CTA's full barrier, which
+            // the even CTA alone arms with the bytes of both halves.
+            constexpr uint32_t kTxBytes = (kPair ? 2 : 1) * C::kStageBytes;
+            auto load_x = [&](uint8_t* sp, uint64_t* bar, int j, int kb, int mt) {
+                if constexpr (kPair)
+                    ptx::tma_load_2d_pair(sp + j * C::kABytes, &tmap_x, in_leader(bar), kb * kBK, mt * kBM, pol_x);
+                else
+                    ptx::tma_load_2d(sp + j * C::kABytes, &tmap_x, bar, kb * kBK, mt * kBM, pol_x);
+            };
+            // Weight tiles of one stage; in a pair each CTA stages its half of the rows
+            // (tmap_w0's box is BN / 2 rows high).
             auto load_w = [&](uint8_t* sp, uint64_t* bar, int kb, int nt) {
-                if constexpr (kMulticast) {
-                    ptx::tma_load_2d_multicast(sp + MT * C::kABytes + crank * (C::kBBytes / CL), &tmap_w0, bar,
-                                               kb * kBK, nt * BN + crank * (BN / CL), kClusterMask, pol_w);
+                if constexpr (kPair) {
+                    ptx::tma_load_2d_pair(sp + MT * C::kABytes, &tmap_w0, in_leader(bar), kb * kBK,
+                                          nt * BN + crank * (BN / 2), pol_w);
                 } else {
                     ptx::tma_load_2d(sp + MT * C::kABytes, &tmap_w0, bar, kb * kBK, nt * BN, pol_w);
                     if (NB == 2)
@@ -239,7 +273,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 const Unit w = unit_of(cid);
                 pre = nk < STAGES ? nk : STAGES;
                 for (int i = 0; i < pre; ++i) {
-                    ptx::mbar_arrive_expect_tx(&full[i], C::kStageBytes);
+                    if (leader) ptx::mbar_arrive_expect_tx(&full[i], kTxBytes);
                     load_w(smem + i * C::kStageBytes, &full[i], w.kx * nk + i, w.nt);
                 }
             }
@@ -260,11 +294,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                     }
                     uint8_t* sp = smem + stage * C::kStageBytes;
                     const bool w_done = it < pre;     // weight tiles already requested above
-                    if (!w_done) ptx::mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
+                    if (!w_done && leader) ptx::mbar_arrive_expect_tx(&full[stage], kTxBytes);
 #pragma unroll
-                    for (int j = 0; j < MT; ++j)
-                        ptx::tma_load_2d(sp + j * C::kABytes, &tmap_x, &full[stage], kb * kBK, (mt0 + j) * kBM,
-                                         pol_x);
+                    for (int j = 0; j < MT; ++j) load_x(sp, &full[stage], j, kb, mt0 + j);
                     if (!w_done) load_w(sp, &full[stage], kb, nt);
                     issued_mask |= 1u << stage;
                     last_parity[stage] = phase;
@@ -279,16 +311,26 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 set_status(status, TF_DEV_TIMEOUT);
             }
             // No copy may still be writing this CTA's shared memory when it exits: wait for the
-            // last load of every stage (already complete unless another role gave up early).
-            for (int s = 0; s < STAGES; ++s)
-                if (issued_mask & (1u << s)) ptx::mbar_wait(&full[s], last_parity[s], nullptr, kWaitLimitNs);
+            // last load of every stage (already complete unless another role gave up early). The
+            // odd CTA of a pair has no barrier of its own to wait on: its copies complete on the
+            // even CTA's barriers, which the even CTA's producer waits for here before both CTAs
+            // meet at the final cluster barrier; after giving up it waits a fixed 100 us, far
+            // longer than any copy takes once issued.
+            if (leader) {
+                for (int s = 0; s < STAGES; ++s)
+                    if (issued_mask & (1u << s)) ptx::mbar_wait(&full[s], last_parity[s], nullptr, kWaitLimitNs);
+            } else if (!ok) {
+                const uint64_t t0 = ptx::globaltimer_ns();
+                while (ptx::globaltimer_ns() - t0 < 100000ull) {
+                }
+            }
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
+        if (lane == 0 && leader) {
             // the NB weight tiles of a stage are adjacent in shared memory with the same swizzle, so
             // one MMA of N = NB * BN covers them: A is read from shared memory once per k-step
-            constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kBM, NB * BN);
+            constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kPair ? 2 * kBM : kBM, NB * BN);
             int stage = 0;
             uint32_t phase = 0;
             uint32_t use[2] = {0u, 0u};
@@ -297,11 +339,14 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             for (int u = cid; u < n_units && ok; u += ncl, ++kl) {
                 const int g0 = (MT == 2) ? 0 : (kl & 1);
                 for (int j = 0; j < MT && ok; ++j)
-                    ok = ptx::mbar_wait(&tempty[g0 + j], (use[g0 + j] & 1u) ^ 1u, abort_flag, kWaitLimitNs);
+                    ok = kPair ? ptx::mbar_wait_cluster(&tempty[g0 + j], (use[g0 + j] & 1u) ^ 1u, abort_flag, kWaitLimitNs)
+                               : ptx::mbar_wait(&tempty[g0 + j], (use[g0 + j] & 1u) ^ 1u, abort_flag, kWaitLimitNs);
                 if (!ok) break;
                 ptx::tc_fence_after();
                 for (int kb = 0; kb < nk; ++kb) {     // position inside the unit's K range
-                    if (!ptx::mbar_wait(&full[stage], phase, abort_flag, kWaitLimitNs)) {
+                    const bool landed = kPair ? ptx::mbar_wait_cluster(&full[stage], phase, abort_flag, kWaitLimitNs)
+                                              : ptx::mbar_wait(&full[stage], phase, abort_flag, kWaitLimitNs);
+                    if (!landed) {
                         ok = false;
                         break;
                     }
@@ -314,14 +359,20 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
 #pragma unroll
                         for (int j = 0; j < MT; ++j) {
                             const uint64_t ad = ptx::sw128_kmajor_desc(a0 + j * C::kABytes + kk * 32);
-                            ptx::mma_bf16(tmem_base + 256u * (g0 + j), ad, bd, kIdesc, (kb | kk) != 0 ? 1u : 0u);
+                            const uint32_t acc = (kb | kk) != 0 ? 1u : 0u;
+                            if constexpr (kPair)
+                                ptx::mma_bf16_pair(tmem_base + 256u * (g0 + j), ad, bd, kIdesc, acc);
+                            else
+                                ptx::mma_bf16(tmem_base + 256u * (g0 + j), ad, bd, kIdesc, acc);
                         }
                     }
-                    // frees the stage (in every CTA of the cluster) once these MMAs finish
-                    if constexpr (kMulticast)
-                        ptx::mma_commit_multicast(&empty[stage], kClusterMask);
-                    else
+                    // frees the stage (in both CTAs of a pair) once these MMAs finish
+                    if constexpr (kPair) {
+                        ptx::mma_commit_pair(ptx::smem_u32(&empty[stage]));
+                        ptx::mma_commit_pair(in_peer(&empty[stage]));
+                    } else {
                         ptx::mma_commit(&empty[stage]);
+                    }
                     if (++stage == STAGES) {
                         stage = 0;
                         phase ^= 1u;
@@ -329,7 +380,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 }
                 if (!ok) break;
                 for (int j = 0; j < MT; ++j) {
-                    ptx::mma_commit(&tfull[g0 + j]);
+                    if constexpr (kPair) {
+                        ptx::mma_commit_pair(ptx::smem_u32(&tfull[g0 + j]));
+                        ptx::mma_commit_pair(in_peer(&tfull[g0 + j]));
+                    } else {
+                        ptx::mma_commit(&tfull[g0 + j]);
+                    }
                     ++use[g0 + j];
                 }
             }
@@ -338,7 +394,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 set_status(status, TF_DEV_TIMEOUT);
             }
             // every MMA issued so far must finish before TMEM is released
-            ptx::mma_commit(drain);
+            if constexpr (kPair)
+                ptx::mma_commit_pair(ptx::smem_u32(drain));
+            else
+                ptx::mma_commit(drain);
             ptx::mbar_wait(drain, 0, nullptr, kWaitLimitNs);
         }
     } else {
@@ -349,6 +408,17 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         const int half = (e % (kEpiWarps / 2)) / 4; // which half of the columns this warp takes
         uint32_t use = 0;
         int kl = 0;
+        // hands the accumulator slot back to the MMA issuer; in a pair one arrival per warp on
+        // the even CTA's barrier, after the warp's TMEM loads have completed
+        auto release_slot = [&](int slot) {
+            ptx::tc_fence_before();
+            if constexpr (kPair) {
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive_cluster(in_leader(&tempty[slot]));
+            } else {
+                ptx::mbar_arrive(&tempty[slot]);
+            }
+        };
         for (int u = cid; u < n_units; u += ncl, ++kl) {
             if (MT == 1 && (kl & 1) != g) continue;
             if (!ptx::mbar_wait(&tfull[g], use & 1u, abort_flag, kWaitLimitNs)) {
@@ -421,8 +491,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                     if (row < n_rows)
                         P.halves[P.half_at(nt, half, row)] = make_float4(hm, hsum, hbv, __int_as_float(hbid));
                 }
-                ptx::tc_fence_before();
-                ptx::mbar_arrive(&tempty[g]);
+                release_slot(g);
             } else if constexpr (EPI == EPI_PARTIAL) {
                 // float4-major: each store instruction writes the warp's 32 rows of 4 columns, 512
                 // contiguous bytes
@@ -443,8 +512,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                         }
                     }
                 }
-                ptx::tc_fence_before();
-                ptx::mbar_arrive(&tempty[g]);
+                release_slot(g);
             } else if constexpr (EPI == EPI_GATEUP) {
 #pragma unroll 1
                 for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
@@ -465,8 +533,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                             dst[j] = make_uint4(packed[4 * j], packed[4 * j + 1], packed[4 * j + 2], packed[4 * j + 3]);
                     }
                 }
-                ptx::tc_fence_before();
-                ptx::mbar_arrive(&tempty[g]);
+                release_slot(g);
             } else {  // EPI_DOWN
                 int hid_row = 0;
                 if (row < n_rows) {
@@ -497,8 +564,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                         }
                     }
                 }
-                ptx::tc_fence_before();
-                ptx::mbar_arrive(&tempty[g]);
+                release_slot(g);
             }
         }
     }
@@ -618,7 +684,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     if (warp == 1) {
         __syncwarp();
         ptx::tc_fence_after();
-        ptx::tmem_dealloc(tmem_base, 512);
+        if constexpr (kPair)
+            ptx::tmem_dealloc_pair(tmem_base, 512);
+        else
+            ptx::tmem_dealloc(tmem_base, 512);
     }
 }
 
@@ -683,7 +752,7 @@ int resident_clusters(K kern, int smem, int cl, int num_sms) {
 template <int EPI, int MT, int NB, int BN, int STAGES, int CL = 1>
 cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& tw0, const CUtensorMap& tw1,
                      int n_rows, int K, int n_ntiles, int n_mgroups, const EpiParams& ep, int k_splits = 1) {
-    using C = TileCfg<MT, NB, BN, STAGES>;
+    using C = TileCfg<MT, NB, BN, STAGES, (CL == 2 && EPI != EPI_CGATEUP && EPI != EPI_CDOWN)>;
     auto kern = tc_gemm_kernel<EPI, MT, NB, BN, STAGES, CL>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (e != cudaSuccess) return e;
@@ -746,9 +815,10 @@ cudaError_t launch_lmhead_tc(const Ctx& ctx, const void* lm_head, const void* x,
     if (n_rows <= 0) return cudaSuccess;
     const int n_tiles = (V + kBlockV - 1) / kBlockV;
     const int m_tiles = (n_rows + kBM - 1) / kBM;
-    // More than one M-tile: clusters of two CTAs, one M-tile each, share every weight tile (each
-    // fetches half of its rows and multicasts them), so W_lm is read once while each CTA keeps
-    // one TMEM slot per unit and overlaps its epilogue with the next unit's MMAs.
+    // More than one M-tile: CTA pairs (clusters of two), one M-tile each, share every weight tile
+    // through cta_group::2 MMAs (each stages half of its rows), so W_lm is read once while each
+    // CTA keeps one TMEM slot per unit and overlaps its epilogue with the next unit's MMAs; 32 KB
+    // per CTA and stage leaves room for seven stages.
     const int cl = m_tiles == 1 ? 1 : 2;
     CUtensorMap tx, tw;
     cudaError_t e = make_tmap(&tx, x, d, n_rows, kBK, kBM);
@@ -760,7 +830,7 @@ cudaError_t launch_lmhead_tc(const Ctx& ctx, const void* lm_head, const void* x,
     ep.inv_temp = inv_temp;
     ep.reset_status = reset_status ? 1 : 0;
     if (m_tiles == 1) return run_gemm<EPI_LMHEAD, 1, 1, kBlockV, 4>(ctx, tx, tw, tw, n_rows, d, n_tiles, 1, ep);
-    return run_gemm<EPI_LMHEAD, 1, 1, kBlockV, 4, 2>(ctx, tx, tw, tw, n_rows, d, n_tiles, (m_tiles + 1) / 2, ep);
+    return run_gemm<EPI_LMHEAD, 1, 1, kBlockV, 7, 2>(ctx, tx, tw, tw, n_rows, d, n_tiles, (m_tiles + 1) / 2, ep);
 }
 
 // Split-K factor for a GEMM with `base_units` (N tiles x M-tile groups) and nk K-steps: enough
