@@ -466,6 +466,59 @@ def test_mask_invariants(mode):
     np.testing.assert_array_equal(res.pos, 1000 + res.tree.depth)
 
 
+def test_topk_margin_hand_values():
+    # the gap between the k-th and (k+1)-th largest entries, by hand; every value is a binary
+    # fraction, so the differences are exact
+    v = np.array([5.0, 1.0, 3.0, 2.5, -1.0])
+    assert [O.topk_margin(v, k) for k in (1, 2, 3, 4)] == [2.0, 0.5, 1.5, 2.0]
+    assert O.topk_margin(v, 5) == np.inf
+
+
+def _hand_result(mode, s1, s2, M, K2, B):
+    """A SeqResult built from hand-written (unnormalised) log-probability lists; ids ranked
+    by value, the tree by the lazy builder."""
+    s1 = np.array(s1, dtype=np.float64)
+    s2 = None if s2 is None else np.array(s2, dtype=np.float64)
+    top_ids = np.stack([O.ranked(r, s1.shape[1]) for r in s1])
+    src = O.ChildSource(mode, s1.shape[0], M, top_ids, s1, s2)
+    tree = O.build_tree_lazy(src, 9, B, keep=K2 if K2 < B else None)
+    return O.SeqResult(s1, top_ids, None, None, s2, None, None, tree, None, None)
+
+
+def test_selection_margins_hand_values():
+    # The margins that decide where the GPU tree must match exactly, on hand-made lists whose
+    # gaps are known exactly. A wrong rank (k vs k + 1), a wrong (B+1)-th pop or a missing term
+    # changes at least one of the expected values below.
+    #
+    # DDTree (marginal), gamma = 2, B = 2. Universe: t0 -1, (t0,u0) -1.25, t1 -2.25,
+    # (t1,u0) -2.5, ... Pops: -1, -1.25; the best left out is t1 at -2.25, so the set margin
+    # is 1.0 and the order margin (gap between the two pops) 0.25. The stage-1 rank-M gap
+    # (0.0625 at M = 2) does not enter: DDTree expands every node.
+    r = _hand_result("marginal", [[-1, -2.25, -2.3125, -7], [-0.25, -3, -3.5, -9]], None, M=2, K2=4, B=2)
+    assert list(r.tree.tok) == [9, 0, 0]
+    assert O.selection_margins(r, 2, 4, 2, "marginal") == (1.0, 0.25)
+    # TreeFlash, gamma = 2, M = 2: stage-2 row 0 holds the root's children, row 1 the children
+    # of depth-1 candidate 0 (token 0), row 2 those of candidate 1 (token 1).
+    s2 = [[-0.5, -2, -2.5, -6], [-1, -1.125, -4, -4.5], [-0.375, -3, -3.125, -4]]
+    # Rank-M gap of depth 1: 3.0. Universe: t0 -0.5, (t0,0) -1.5, (t0,1) -1.625, t1 -2,
+    # (t1,0) -2.375, t2 -2.5, ... (t2, t3 are leaves). B = 3 pops -0.5, -1.5, -1.625; the best
+    # left out is t1 at -2, so the set margin is min(3.0, 0.375) and the order margin
+    # min(0.375, 1.0, 0.125).
+    wide = [[-1, -1.5, -4.5, -5], [-1, -2, -3, -4]]
+    r = _hand_result("ar", wide, s2, M=2, K2=4, B=3)
+    assert list(r.tree.tok) == [9, 0, 0, 1]
+    assert O.selection_margins(r, 2, 4, 3, "ar") == (0.375, 0.125)
+    # the same with the stage-1 rank-M gap of depth 1 shrunk to 0.125: it decides both
+    narrow = [[-1, -1.5, -1.625, -5], [-1, -2, -3, -4]]
+    r = _hand_result("ar", narrow, s2, M=2, K2=4, B=3)
+    assert O.selection_margins(r, 2, 4, 3, "ar") == (0.125, 0.125)
+    # K2 = 2 < B = 3 truncates every list after two entries; the rank-2 gaps of the stage-2
+    # rows are 0.5, 2.875 and 0.125 (row 2), the smallest term of the set margin
+    r = _hand_result("ar", wide, s2, M=2, K2=2, B=3)
+    assert list(r.tree.tok) == [9, 0, 0, 1]
+    assert O.selection_margins(r, 2, 2, 3, "ar") == (0.125, 0.125)
+
+
 def test_margins_are_positive_and_finite_for_generic_inputs():
     res = _run(seed=5, B=10, M=3)
     sm, om = O.selection_margins(res, 3, 10, 10)
