@@ -37,6 +37,7 @@ sys.path.insert(0, ROOT)
 METRIC = "µs per draft-tree build (trees/s) at Qwen3-8B shape, B=32/64; % of HBM roofline"
 WORKLOAD = "q8_b64"
 FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0          # GB300 HBM3e, nominal (~8 TB/s); the measured copy rate is the peak
 FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
 
 
@@ -206,6 +207,7 @@ def lmhead_roofline(cfg, n1, n2, lm1_ms, lm2_ms, hbm_peak, tc_peak, traffic, tim
     gbs = sum(nbytes) / 2 / avg_s / 1e9
     hbm = {"bound": "hbm", "kernel": "tc_gemm_kernel<LMHEAD> (stage-1 and stage-2 launches)",
            "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak, "traffic": traffic,
+           "frac_nominal": gbs / NOMINAL_HBM_GBS,
            "peak_kind": peak_kind, "launch_ms": {"stage1": lm1_ms, "stage2": lm2_ms},
            "bytes_per_launch": {"stage1": nbytes[0], "stage2": nbytes[1]},
            "flops_per_launch": {"stage1": flops[0], "stage2": flops[1]}, "timing": timing}
@@ -336,6 +338,45 @@ class OracleSample:
         t = time.perf_counter() - t0
         full = t_mlp + max(t - t_mlp, 0.0) * cfg.V / Vs
         return t, full, Vs
+
+
+def oracle_sample_child(path: str) -> None:
+    """Child side of oracle_single_thread: load the sample's tensors, run the oracle once on
+    them and print (seconds, estimated seconds per tree, vocabulary used) as JSON."""
+    import torch
+    import synth
+    d = torch.load(path)
+    cfg = synth.get_config(d["workload"])
+    orc = OracleSample(cfg, d["inp"])
+    t, full, Vs = orc.run(d["inp"]["lm_head"].shape[0] / cfg.V)
+    print(json.dumps({"t": t, "full": full, "Vs": Vs}), flush=True)
+
+
+def oracle_single_thread(cfg, inp, frac):
+    """The oracle's sample on one host core: a child process started with the BLAS and OpenMP
+    thread counts set to 1 before numpy loads (they cannot be changed afterwards). It gets the
+    sample's tensors in their own dtype (the vocabulary-dependent ones cut to the sample's
+    vocabulary; every token the sample can reach lies below it) through a temporary file."""
+    import tempfile
+    import torch
+    Vs = max(cfg.K2 + cfg.M, int(math.ceil(cfg.V * frac)))
+    keys = ("hidden", "root_tok", "root_prev", "norm_h", "norm_e", "w_gate", "w_up", "w_down", "w_lin")
+    sample = {k: inp[k][:1] if k in ("hidden", "root_tok", "root_prev") else inp[k]
+              for k in keys if inp.get(k) is not None}
+    sample["lm_head"] = inp["lm_head"][:Vs].clone()
+    sample["embed"] = inp["embed"][:Vs].clone()
+    with tempfile.TemporaryDirectory() as td:
+        path = os.path.join(td, "sample.pt")
+        torch.save({"workload": cfg.name, "inp": sample}, path)
+        env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-sample", path], env=env,
+                           capture_output=True, text=True, timeout=900)
+    if r.returncode != 0:
+        return {"error": (r.stderr.strip().splitlines() or ["child failed"])[-1][:200]}
+    res = json.loads(r.stdout.strip().splitlines()[-1])
+    return {"value": 1.0 / res["full"], "unit": "trees/s", "cores": 1, "kind": "oracle",
+            "sample": f"fp64 numpy oracle on one core, 1 sequence, vocabulary cut to {res['Vs']} of {cfg.V} "
+                      f"({res['t']:.1f} s), LM-head/softmax/sort time scaled to the full V"}
 
 
 def cpu_model() -> str:
@@ -554,6 +595,8 @@ def run_gpu(args):
                "kind": "oracle",
                "sample": f"fp64 numpy oracle, 1 sequence, vocabulary cut to {Vs} of {cfg.V} "
                          f"({t:.1f} s), LM-head/softmax/sort time scaled to the full V"}
+        # the same oracle on one core, on a smaller cut of the vocabulary (about as long)
+        cpu["single_thread"] = oracle_single_thread(cfg, inp, max(1 / 1024, frac / max(cpu_threads(), 1)))
 
     if rank != 0:
         return
@@ -561,7 +604,7 @@ def run_gpu(args):
     line = {
         "metric": METRIC, "value": value, "unit": "trees/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "us_per_tree": ms_per_step * 1e3 / cfg.batch,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype,
         "data": "synthetic (seeded N(0,0.02) weights, hidden states scaled to 2-4 nat marginals)",
         "config": {"workload": cfg.name, "batch": cfg.batch, "d": cfg.d, "V": cfg.V, "I": cfg.I,
                    "gamma": cfg.gamma, "M": cfg.M, "K2": cfg.K2, "B": cfg.B, "R": cfg.R, "approx": cfg.approx,
@@ -569,7 +612,10 @@ def run_gpu(args):
                    "parallelism": f"replicas x{world}"},
         "step_roofline": {"algorithmic_bytes": step_bytes, "achieved_gbs": step_bytes / (ms_per_step / 1e3) / 1e9,
                           "peak_gbs": peak, "frac": step_bytes / (ms_per_step / 1e3) / 1e9 / peak,
-                          "peak_kind": peak_kind},
+                          "peak_kind": peak_kind, "nominal_gbs": NOMINAL_HBM_GBS,
+                          "frac_nominal": step_bytes / (ms_per_step / 1e3) / 1e9 / NOMINAL_HBM_GBS,
+                          "target": "70 % of the HBM roofline, judged against the measured copy rate "
+                                    "(peak_gbs); frac_nominal is the same figure against 8 TB/s"},
         "roofline": roofline,
         "clocks": clocks, "e2e": e2e, "gpu_launches": gpu_launches,
         "cpu_baseline": cpu, "torch_eager": eager, "device_flags": flags,
@@ -590,8 +636,11 @@ def main():
                     help="steps of the torch library-call reference point (0 = skip)")
     ap.add_argument("--cpu-baseline-s", type=float, default=20.0,
                     help="approximate seconds of oracle work for the cpu_baseline sample (0 = skip)")
+    ap.add_argument("--cpu-sample", default=None, help=argparse.SUPPRESS)   # child of oracle_single_thread
     args = ap.parse_args()
-    if args.impl == "reference":
+    if args.cpu_sample:
+        oracle_sample_child(args.cpu_sample)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_gpu(args)

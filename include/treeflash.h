@@ -136,6 +136,17 @@ int32_t tf_version(void);
  * the kernels of a timed region: read it before and after. */
 uint64_t tf_kernel_launches(void);
 
+/* Failure detection. Every wait inside the tensor-core kernels (a TMA copy landing, an MMA
+ * finishing, an accumulator being drained) gives up after a time limit, 2 s by default: the
+ * kernel then sets TF_DEV_TIMEOUT in the status word, waits (again bounded, always 2 s) for
+ * its own copies and MMAs in flight, frees its tensor memory and returns, so the context stays
+ * usable and tf_status_read reports TF_ERR_TIMEOUT. This sets the limit of those waits for
+ * progress for every later launch in the process (ns = 0 restores the default); the waits that
+ * drain in-flight work keep 2 s. A limit shorter than a copy's latency makes every call time
+ * out, which is how the failure path is tested. Host only; returns TF_ERR_INVALID_ARG above
+ * 60 s. It does not cover calls already enqueued. */
+tf_status tf_set_wait_limit_ns(uint64_t ns);
+
 /* Validate `dims` and return the workspace bytes every call below needs for these dims
  * (the maximum over all calls, so one buffer serves the whole step). Host only; no GPU
  * work. The workspace must be device memory, 256-byte aligned, and must not be used by two
@@ -345,7 +356,10 @@ tf_status tf_workspace_view(const tf_dims* dims, void* ws, size_t ws_bytes, int3
  * return TF_ERR_UNSUPPORTED before any GPU work. Other arguments are checked as in
  * tf_stage1_marginals (TF_ERR_INVALID_ARG, TF_ERR_UNSUPPORTED).
  * The first call on a device looks up the array's device address (cudaGetSymbolAddress, with
- * that device current) and caches it; make that first call before any stream capture.
+ * that device current) and keeps it for that device's current CUDA context; make that first
+ * call before any stream capture. A call in a new context of the device (after cudaDeviceReset,
+ * or after the primary context was released and re-created) looks the address up again, so it
+ * too should precede any capture.
  * Every call on a device shares the one array: calls that can overlap on the GPU (different
  * streams, or threads sharing a device without ordering) race and corrupt each other's results.
  * Issue them on one stream, or order them. */

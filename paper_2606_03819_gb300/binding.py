@@ -48,7 +48,8 @@ class TfWeights(ctypes.Structure):
 EXPORTS = ("tf_status_string", "tf_version", "tf_kernel_launches", "tf_workspace_size", "tf_status_reset", "tf_status_read",
            "tf_stage1_marginals", "tf_stage2_ar_approx", "tf_build_tree", "tf_tree_mask", "tf_build_tree_mask",
            "tf_draft_tree_host", "tf_lmhead_partials", "tf_lmhead_merge", "tf_ar_approx",
-           "tf_workspace_h_prime", "tf_workspace_view", "tf_stage1_marginals_static", "tf_accept_walk")
+           "tf_workspace_h_prime", "tf_workspace_view", "tf_stage1_marginals_static", "tf_accept_walk",
+           "tf_set_wait_limit_ns")
 
 _lib = None
 
@@ -69,6 +70,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
         "tf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
         "tf_version": (I32, []),
         "tf_kernel_launches": (ctypes.c_uint64, []),
+        "tf_set_wait_limit_ns": (ctypes.c_int, [ctypes.c_uint64]),
         "tf_workspace_size": (ctypes.c_int, [D, ctypes.POINTER(SZ)]),
         "tf_status_reset": (ctypes.c_int, [P, SZ, P]),
         "tf_status_read": (ctypes.c_int, [P, SZ, ctypes.POINTER(I32), P]),
@@ -173,6 +175,12 @@ def tf_version() -> int:
 def tf_kernel_launches() -> int:
     """Kernels launched by the library so far in this process."""
     return int(load_library().tf_kernel_launches())
+
+
+def tf_set_wait_limit_ns(ns: int) -> None:
+    """Limit of the tensor-core kernels' waits for progress, for every later launch (0 = the
+    default 2 s); a limit below a copy's latency makes calls time out (TF_DEV_TIMEOUT)."""
+    _check("tf_set_wait_limit_ns", load_library().tf_set_wait_limit_ns(int(ns)))
 
 
 def tf_workspace_size(dims: Dims) -> int:

@@ -14,8 +14,10 @@ size_t merge_smem_bytes(int n_tiles, int d, int k);
 
 namespace {
 std::atomic<unsigned long long> g_kernel_launches{0};
+std::atomic<unsigned long long> g_wait_limit_ns{0};
 }
 void note_launch() { g_kernel_launches.fetch_add(1, std::memory_order_relaxed); }
+unsigned long long wait_limit_ns() { return g_wait_limit_ns.load(std::memory_order_relaxed); }
 }  // namespace tf
 
 namespace {
@@ -266,6 +268,12 @@ const char* tf_status_string(tf_status s) {
 int32_t tf_version(void) { return 100; }
 
 uint64_t tf_kernel_launches(void) { return tf::g_kernel_launches.load(std::memory_order_relaxed); }
+
+tf_status tf_set_wait_limit_ns(uint64_t ns) {
+    if (ns > 60ull * 1000000000ull) return TF_ERR_INVALID_ARG;
+    tf::g_wait_limit_ns.store(ns, std::memory_order_relaxed);
+    return TF_OK;
+}
 
 tf_status tf_workspace_size(const tf_dims* dims, size_t* bytes) {
     if (!bytes) return TF_ERR_INVALID_ARG;

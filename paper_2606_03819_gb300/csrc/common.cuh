@@ -97,6 +97,9 @@ __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.lau
 
 // Host-side count of kernels launched by this library (tf_kernel_launches).
 void note_launch();
+// Limit of the tensor-core kernels' waits for progress, set by tf_set_wait_limit_ns (0: the
+// kernels' own default).
+unsigned long long wait_limit_ns();
 
 template <typename... KArgs, typename... Args>
 cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,

@@ -12,6 +12,8 @@
 //
 // The kernels are the ones tf_stage1_marginals runs (same launchers, same arguments); only the
 // place of the per-block partials and of the status word differs.
+#include <cuda.h>
+
 #include <mutex>
 
 #include "common.cuh"
@@ -34,22 +36,60 @@ static_assert(kScratchBytes % 256 == 0 && kScratchBytes > kStatusBytes, "scratch
 // the device memory: host code must use the address cudaGetSymbolAddress returns instead.
 static __device__ __align__(256) uint8_t g_scratch[kScratchBytes];
 
+// The context a device address belongs to: the driver's unique id of the calling thread's
+// current context (cuCtxGetCurrent + cuCtxGetId, reached through the runtime's driver entry
+// points). A device reset or a re-created primary context gives a new id, and with it a new
+// lookup of the array's address. Returns false if the driver offers no such id.
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+bool current_context_id(unsigned long long* id) {
+    static const CtxGetCurrentFn get_current = [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            p = nullptr;
+        return reinterpret_cast<CtxGetCurrentFn>(p);
+    }();
+    static const CtxGetIdFn get_id = [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            p = nullptr;
+        return reinterpret_cast<CtxGetIdFn>(p);
+    }();
+    CUcontext ctx = nullptr;
+    if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx) return false;
+    return get_id(ctx, id) == CUDA_SUCCESS;
+}
+
 std::mutex g_setup_mutex;
 void* g_scratch_addr[kMaxDevices] = {};
+unsigned long long g_scratch_ctx[kMaxDevices] = {};
 
-// Device address of g_scratch on the current device `dev`, looked up once per device (under a
-// lock, so threads may race to the first call) and cached.
+// Device address of g_scratch on the current device `dev`: looked up once per device and
+// context (under a lock, so threads may race to the first call) and kept. Without a context id
+// from the driver it is looked up on every call, which allocates nothing either.
 tf_status scratch_address(int dev, uint8_t** out) {
     if (dev < 0 || dev >= kMaxDevices) return TF_ERR_UNSUPPORTED;
+    // No current context yet (this thread's first runtime call on the device): the lookup below
+    // binds the runtime's primary context, and the id is read after it.
+    unsigned long long ctx = 0;
+    bool have_ctx = current_context_id(&ctx);
     std::lock_guard<std::mutex> lock(g_setup_mutex);
-    if (!g_scratch_addr[dev]) {
+    if (!have_ctx || !g_scratch_addr[dev] || g_scratch_ctx[dev] != ctx) {
         void* p = nullptr;
         const cudaError_t e = cudaGetSymbolAddress(&p, g_scratch);
         if (e != cudaSuccess || !p) {
             (void)cudaGetLastError();  // do not leave the error for a later launch check to find
             return TF_ERR_CUDA;
         }
-        g_scratch_addr[dev] = p;
+        if (!have_ctx) have_ctx = current_context_id(&ctx);
+        g_scratch_addr[dev] = have_ctx ? p : nullptr;   // no id: look it up again next call
+        g_scratch_ctx[dev] = ctx;
+        *out = static_cast<uint8_t*>(p);
+        return TF_OK;
     }
     *out = static_cast<uint8_t*>(g_scratch_addr[dev]);
     return TF_OK;

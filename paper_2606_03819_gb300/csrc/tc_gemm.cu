@@ -60,6 +60,8 @@ struct EpiParams {
     int n_cols;                  //          accumulator nb of N tile nt at columns nb * n_total + nt * BN
     int n_total;                 // N of the whole GEMM (n_ntiles * BN)
     int reset_status;            // LMHEAD: zero *status first (the first kernel of a stage-1 call)
+    unsigned long long wait_ns;  // limit of every wait for progress (0: kWaitLimitNs); the waits
+                                 // that drain in-flight copies and MMAs always take kWaitLimitNs
 };
 
 // Work unit u -> (N tile, M-tile group, K split); consecutive units share the N tile and K split
@@ -185,6 +187,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     const int cid = CL > 1 ? static_cast<int>(ptx::cluster_id_x()) : static_cast<int>(blockIdx.x);
     const int ncl = CL > 1 ? static_cast<int>(ptx::cluster_count_x()) : static_cast<int>(gridDim.x);
     const int nk = K / kBK / k_splits;      // K-steps per unit (K % (64 * k_splits) == 0)
+    const uint64_t wait_ns = ep.wait_ns ? ep.wait_ns : kWaitLimitNs;
     auto unit_of = [&](int u) {
         if constexpr (kSplitK) return Unit{u / n_mgroups, u % n_mgroups, crank};
         return decode_unit(u, n_mgroups, k_splits);
@@ -288,7 +291,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 const Unit w = unit_of(u);
                 const int nt = w.nt, mt0 = (w.mg * m_cl + m_rank) * MT;
                 for (int kb = w.kx * nk; kb < (w.kx + 1) * nk; ++kb, ++it) {
-                    if (!ptx::mbar_wait(&empty[stage], phase ^ 1u, abort_flag, kWaitLimitNs)) {
+                    if (!ptx::mbar_wait(&empty[stage], phase ^ 1u, abort_flag, wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -339,13 +342,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             for (int u = cid; u < n_units && ok; u += ncl, ++kl) {
                 const int g0 = (MT == 2) ? 0 : (kl & 1);
                 for (int j = 0; j < MT && ok; ++j)
-                    ok = kPair ? ptx::mbar_wait_cluster(&tempty[g0 + j], (use[g0 + j] & 1u) ^ 1u, abort_flag, kWaitLimitNs)
-                               : ptx::mbar_wait(&tempty[g0 + j], (use[g0 + j] & 1u) ^ 1u, abort_flag, kWaitLimitNs);
+                    ok = kPair ? ptx::mbar_wait_cluster(&tempty[g0 + j], (use[g0 + j] & 1u) ^ 1u, abort_flag, wait_ns)
+                               : ptx::mbar_wait(&tempty[g0 + j], (use[g0 + j] & 1u) ^ 1u, abort_flag, wait_ns);
                 if (!ok) break;
                 ptx::tc_fence_after();
                 for (int kb = 0; kb < nk; ++kb) {     // position inside the unit's K range
-                    const bool landed = kPair ? ptx::mbar_wait_cluster(&full[stage], phase, abort_flag, kWaitLimitNs)
-                                              : ptx::mbar_wait(&full[stage], phase, abort_flag, kWaitLimitNs);
+                    const bool landed = kPair ? ptx::mbar_wait_cluster(&full[stage], phase, abort_flag, wait_ns)
+                                              : ptx::mbar_wait(&full[stage], phase, abort_flag, wait_ns);
                     if (!landed) {
                         ok = false;
                         break;
@@ -421,7 +424,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         };
         for (int u = cid; u < n_units; u += ncl, ++kl) {
             if (MT == 1 && (kl & 1) != g) continue;
-            if (!ptx::mbar_wait(&tfull[g], use & 1u, abort_flag, kWaitLimitNs)) {
+            if (!ptx::mbar_wait(&tfull[g], use & 1u, abort_flag, wait_ns)) {
                 *abort_flag = 1;
                 set_status(status, TF_DEV_TIMEOUT);
                 break;
@@ -751,9 +754,11 @@ int resident_clusters(K kern, int smem, int cl, int num_sms) {
 
 template <int EPI, int MT, int NB, int BN, int STAGES, int CL = 1>
 cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& tw0, const CUtensorMap& tw1,
-                     int n_rows, int K, int n_ntiles, int n_mgroups, const EpiParams& ep, int k_splits = 1) {
+                     int n_rows, int K, int n_ntiles, int n_mgroups, const EpiParams& ep_in, int k_splits = 1) {
     using C = TileCfg<MT, NB, BN, STAGES, (CL == 2 && EPI != EPI_CGATEUP && EPI != EPI_CDOWN)>;
     auto kern = tc_gemm_kernel<EPI, MT, NB, BN, STAGES, CL>;
+    EpiParams ep = ep_in;
+    ep.wait_ns = wait_limit_ns();
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (e != cudaSuccess) return e;
     const int n_units = n_ntiles * n_mgroups * k_splits;

@@ -44,19 +44,19 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-// Wait until the phase with the given parity has completed. Gives up (returns false) after
-// `limit_ns` nanoseconds or when *abort becomes non-zero (abort may be null), so no caller
-// can spin forever.
+// Wait until the phase with the given parity has completed. Gives up (returns false) once
+// `limit_ns` nanoseconds have passed since the first failed poll, or when *abort becomes
+// non-zero (abort may be null), so no caller can spin forever.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
                                           uint64_t limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
+    // try_wait itself suspends for a while before it reports an incomplete phase, so the
+    // deadline and the abort flag are checked after every failed poll (only while waiting)
     const uint64_t t0 = globaltimer_ns();
-    for (uint32_t i = 1;; ++i) {
+    for (;;) {
         if (mbar_try_wait(bar, parity)) return true;
-        if ((i & 63u) == 0) {
-            if (abort != nullptr && *abort) return false;
-            if (globaltimer_ns() - t0 > limit_ns) return false;
-        }
+        if (abort != nullptr && *abort) return false;
+        if (globaltimer_ns() - t0 > limit_ns) return false;
     }
 }
 
@@ -213,12 +213,10 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity
                                                   uint64_t limit_ns) {
     if (mbar_try_wait_cluster(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
-    for (uint32_t i = 1;; ++i) {
+    for (;;) {
         if (mbar_try_wait_cluster(bar, parity)) return true;
-        if ((i & 63u) == 0) {
-            if (abort != nullptr && *abort) return false;
-            if (globaltimer_ns() - t0 > limit_ns) return false;
-        }
+        if (abort != nullptr && *abort) return false;
+        if (globaltimer_ns() - t0 > limit_ns) return false;
     }
 }
 
