@@ -4,19 +4,18 @@ Both sides read the same seeded inputs from synth/. The oracle runs in float64 (
 bf16 rounding at the points where the CUDA path stores bf16). Comparison rules:
 
 * log-probabilities (stage-1 top-K1, stage-2 top-K2, node scores): every value the GPU reports
-  for a token id must be within `tol_lp` of the oracle's exact log-probability of that id, and
-  the GPU's sorted values must match the oracle's sorted top values rank by rank within
-  `tol_lp` (so a swap of two near-equal entries is allowed, a wrong value is not). Node scores
-  are sums of up to depth log-probabilities and get depth * tol_lp.
-* ids: the top-M candidate set of every depth (which decides the M-ary tree) must equal the
-  oracle's whenever the oracle's gap at rank M exceeds `tol_sel`; stage-2 rows are paired with
-  oracle rows by (depth, previous token).
-* tree: when the oracle's order margin exceeds `tol_sel` the token, parent and depth arrays
-  must be bit-exact (same pop order); when only the set margin does, the trees must be equal
-  as sets of token paths. Otherwise only validity is checked (prefix-closed, M-ary rule,
-  scores = sums of the GPU's own child log-probs).
-* mask / position ids: always bit-exact against the oracle's mask of the GPU's own tree, and
-  against the oracle's tree when that was required to match.
+  for a token id must be within the bound of the oracle's exact log-probability of that id, and
+  the GPU's sorted values must match the oracle's sorted top values rank by rank (so a swap of
+  two near-equal entries is allowed, a wrong value is not); stage-2 rows are paired with oracle
+  rows by their conditioning (depth, previous token(s)).
+* fp32 path (compare): everything against the plain oracle within 1e-4; the top-M candidate
+  sets, and the tree's tokens, parents, depths, mask and position ids, bit-exact wherever the
+  oracle's selection margins exceed 1e-3 (as sets of token paths where only the set margin does).
+* bf16 path (check_bf16_end_to_end, BF16): stage 1 against the plain oracle, stage 2 and the
+  tree against the oracle that rounds to bf16 where the GPU stores bf16; the structure is
+  compared at every cut of the oracle's pop order that the node-score bound decides. Each stage
+  is also checked on the GPU's own inputs to it (check_bf16_stagewise).
+* mask / position ids: always bit-exact against the oracle's mask of the GPU's own tree.
 """
 from __future__ import annotations
 
@@ -27,15 +26,9 @@ import synth
 from oracle import treeflash_oracle as O
 
 TOLS = {
-    # lp: stage-1 log-probs vs the plain fp64 oracle; lp2: stage-2 log-probs vs the plain oracle,
-    # on top of the oracle's own emulated-minus-plain difference (the bf16 path rounds x,
-    # SiLU(G)*U and h' to bf16 before the next GEMM); lp_emul: everything vs the oracle that
-    # rounds at those points (the
-    # remaining difference is fp32-vs-fp64 accumulation flipping a bf16 rounding, worth up to
-    # |w| * ulp(h') per flipped element); sel: selection margin above which the tree structure
-    # must match exactly (twice the per-log-prob tolerance).
-    "f32": dict(lp=1e-4, lp2=1e-4, lp_emul=1e-4, sel=1e-3),
-    "bf16": dict(lp=2e-2, lp2=2e-2, lp_emul=2e-2, sel=4e-2),
+    # fp32 path against the plain fp64 oracle: lp, every log-probability; sel, the selection
+    # margin above which the tree structure must match exactly. The bf16 path's bounds are BF16.
+    "f32": dict(lp=1e-4, sel=1e-3),
 }
 
 
@@ -134,14 +127,10 @@ def _check_row(gpu_ids, gpu_lp, full_lp, tol, what):
     return max(err_id, err_rank)
 
 
-def compare(cfg, gpu, orc, tol_lp, tol_sel, check_structure=True, tol_lp2=None, orc_round=None,
-            round_factor=1.0):
-    """Assert parity of one batch; returns a small report dict.
-
-    orc_round: the bf16-emulating oracle's results for the same sequences. When given, every
-    stage-2 row may additionally deviate by the oracle's own emulated-minus-plain difference at
-    the reported ids (|gpu - plain| <= |gpu - emulated| + |emulated - plain|)."""
-    tol_lp2 = tol_lp if tol_lp2 is None else tol_lp2
+def compare(cfg, gpu, orc, tol_lp, tol_sel, check_structure=True):
+    """Assert parity of one batch against one oracle result per sequence (the fp32 path's
+    rule: every log-probability within tol_lp, structure exact beyond tol_sel); returns a small
+    report dict."""
     rep = dict(max_err_s1=0.0, max_err_s2=0.0, max_err_score=0.0, rows_s2=0, rows_s2_skipped=0,
                exact_trees=0, set_trees=0, valid_only_trees=0)
     M, g = cfg.M, cfg.gamma
@@ -159,24 +148,12 @@ def compare(cfg, gpu, orc, tol_lp, tol_sel, check_structure=True, tol_lp2=None, 
             rprev = int(gpu["root_prev"][s]) if gpu.get("root_prev") is not None else None
             okey = {k: r for r, k in enumerate(conditioning_keys(cfg, root, o.top_ids, rprev))}
             gkeys = conditioning_keys(cfg, root, gpu["top_ids"][s], rprev)
-            if orc_round is not None:
-                ekey = {k: r for r, k in enumerate(conditioning_keys(cfg, root, orc_round[s].top_ids, rprev))}
             for r, key in enumerate(gkeys):
                 orow = okey.get(key)
                 if orow is None:
                     rep["rows_s2_skipped"] += 1
                     continue
-                tol_row = tol_lp2
-                if orc_round is not None:
-                    erow = ekey.get(key)
-                    if erow is None:
-                        rep["rows_s2_skipped"] += 1
-                        continue
-                    ids = gpu["child_ids"][s, r]
-                    tol_row = tol_lp2 + round_factor * float(
-                        np.abs(orc_round[s].s2_logp[erow][ids] - o.s2_logp[orow][ids]).max())
-                    rep["max_round_allowance"] = max(rep.get("max_round_allowance", 0.0), tol_row - tol_lp2)
-                e = _check_row(gpu["child_ids"][s, r], gpu["child_logp"][s, r], o.s2_logp[orow], tol_row,
+                e = _check_row(gpu["child_ids"][s, r], gpu["child_logp"][s, r], o.s2_logp[orow], tol_lp,
                                f"seq {s} stage-2 row {r}")
                 rep["max_err_s2"] = max(rep["max_err_s2"], e)
                 rep["rows_s2"] += 1
@@ -195,7 +172,7 @@ def compare(cfg, gpu, orc, tol_lp, tol_sel, check_structure=True, tol_lp2=None, 
                 present = o.tree.parent >= 0
                 present[0] = True
                 err = np.abs(sc[present] - o.tree.score[present])
-                lim = np.maximum(dep[present], 1) * max(tol_lp, tol_lp2)
+                lim = np.maximum(dep[present], 1) * tol_lp
                 assert (err <= lim).all(), f"seq {s}: node score off by {err.max():.3g}"
                 rep["max_err_score"] = max(rep["max_err_score"], float(err.max()))
                 rep["exact_trees"] += 1
@@ -261,9 +238,27 @@ def _check_tree_valid(cfg, gpu, s):
 # ------------------------------------------------------------------------------------------
 
 ACC_REL = 2.0 ** -14     # tensor-core fp32 accumulation: relative to the sum of |terms|
-E2E_ROUND_FACTOR = 2.0   # stage-2 allowance vs the plain oracle, in units of the emulating
-                         # oracle's own deviation (two realizations of the same bf16 storage)
-E2E_TREE_MARGIN = 0.25   # plain-oracle set margin above which the trees must coincide
+
+# The bf16 end-to-end contract. The paper runs its method in bf16 (Sec. 4, Setup), and this path
+# stores x, SiLU(G)*U and h' in bf16 between its tensor-core GEMMs (reading R11). The reference
+# is therefore the oracle that rounds at exactly those points; what remains between the two is
+# fp32 tensor-core accumulation against fp64, which flips a small fraction of those roundings.
+#  s1:   stage-1 log-probabilities against the plain oracle (bf16 inputs, nothing rounded before
+#        them, fp32 accumulation): measured at most 1.5e-4 over the full-size workloads.
+#  s2:   stage-2 log-probabilities against the emulating oracle, every reported id and rank by
+#        rank. Measured maxima on the full-size workloads: q8_b32 0.024 and q8_b64 0.031 (8
+#        sequences each, 247k entries; median 0.0012), q8_b512 0.025, q8_m64 0.033, batch32
+#        0.025, q8_b32_2prev 0.048, wide_flat 0.040, wide_peaked 0.054 (its larger hidden states
+#        make each flipped bf16 rounding of h' weigh more). The bound is about twice the largest.
+#        Against the plain oracle the same entries differ by up to 0.14, as much as the
+#        emulating oracle itself differs from the plain one: the bf16 storage, not the kernels.
+#  node: node scores (sums of log-probabilities along a path) against the emulating oracle's
+#        score of the same path: measured at most 0.028 (wide_peaked; batch32 0.027, q8_b64
+#        0.0155 over 8 trees), with no growth in depth (the tree uses each row's best entries,
+#        where the log-sum-exp error cancels). The bound is about twice the largest; it decides
+#        where the structure must match.
+BF16 = dict(s1=1e-3, s2=0.1, node=0.06)
+UNIVERSE_EXTRA = 16      # universe nodes listed beyond the budget for the cut test
 
 
 def _ulp_bf16(x):
@@ -335,7 +330,7 @@ def _check_lmhead_and_builder(cfg, W, gpu, hp, rep):
     err = 0.0
     for r in range(hp.shape[0]):
         s, rr = divmod(r, R)
-        err = max(err, _check_row(gpu["child_ids"][s, rr], gpu["child_logp"][s, rr], lp[r], 2e-2,
+        err = max(err, _check_row(gpu["child_ids"][s, rr], gpu["child_logp"][s, rr], lp[r], BF16["s1"],
                                   f"seq {s} stage-2 row {rr} (LM head of the GPU's h')"))
     rep["lmhead_logp_err"] = err
     # Part 2 on the GPU's own lists: the oracle's builder must pick the same tree
@@ -373,17 +368,119 @@ def _gpu_lists_source(cfg, gpu, s):
 
 
 def check_bf16_end_to_end(cfg, gpu, orc, orc_emul):
-    """bf16 path against the plain fp64 oracle: stage 1 within 2e-2; every stage-2 row within
-    2e-2 plus E2E_ROUND_FACTOR times the emulating oracle's own deviation from the plain one on
-    that row (the effect of storing x, SiLU(G)*U and h' in bf16); trees equal as sets where the
-    plain oracle's set margin exceeds E2E_TREE_MARGIN."""
-    rep = compare(cfg, gpu, orc, 2e-2, np.inf, check_structure=False, tol_lp2=2e-2,
-                  orc_round=orc_emul if cfg.mode == "ar" else None, round_factor=E2E_ROUND_FACTOR)
-    rep["e2e_set_trees"] = 0
-    for s, o in enumerate(orc):
-        set_m, _ = O.selection_margins(o, cfg.M, cfg.K2, cfg.B, cfg.mode)
-        if set_m > E2E_TREE_MARGIN:
-            assert _paths(gpu["node_tok"][s], gpu["node_parent"][s]) == set(O.tree_paths(o.tree)), \
-                f"seq {s}: tree differs from the plain oracle's"
-            rep["e2e_set_trees"] += 1
+    """The bf16 path end to end (BF16 explains the bounds). orc: the plain fp64 oracle;
+    orc_emul: the oracle that rounds x, SiLU(G)*U and h' to bf16 where the GPU stores them (None
+    in the marginal modes, where nothing is stored in bf16 before the log-probabilities)."""
+    T = BF16
+    ar = cfg.mode == "ar"
+    ref = orc_emul if ar else orc
+    M, g = cfg.M, cfg.gamma
+    rep = dict(max_err_s1=0.0, max_err_s2_emul=0.0, max_err_s2_plain=0.0, max_emul_minus_plain=0.0,
+               max_err_node=0.0, rows_s2=0, rows_s2_skipped=0, cuts=0, cuts_determined=0,
+               prefix_nodes=0, exact_trees=0, set_trees=0, excluded_trees=0)
+    for s, (o, e) in enumerate(zip(orc, ref)):
+        # ---- stage 1 against the plain oracle (nothing is rounded before it)
+        for i in range(g):
+            err = _check_row(gpu["top_ids"][s, i], gpu["top_logp"][s, i], o.s1_logp[i], T["s1"],
+                             f"seq {s} depth {i + 1}")
+            rep["max_err_s1"] = max(rep["max_err_s1"], err)
+        # the M-ary candidate sets decide the tree's universe: equal wherever the gap at rank M
+        # exceeds twice the stage-1 bound; a set inside that band excludes the tree below
+        same_sets = True
+        if cfg.mode != "marginal":
+            for i in range(g - 1):
+                if set(gpu["top_ids"][s, i, :M].tolist()) != set(o.top_ids[i, :M].tolist()):
+                    assert O.topk_margin(o.s1_logp[i], M) <= 2 * T["s1"], f"seq {s} depth {i + 1}: top-M set differs"
+                    same_sets = False
+        # ---- stage 2 against the emulating oracle, rows paired by their conditioning
+        if ar:
+            root = int(o.tree.tok[0])
+            rprev = int(gpu["root_prev"][s]) if gpu.get("root_prev") is not None else None
+            ekey = {k: r for r, k in enumerate(conditioning_keys(cfg, root, e.top_ids, rprev))}
+            for r, key in enumerate(conditioning_keys(cfg, root, gpu["top_ids"][s], rprev)):
+                erow = ekey.get(key)
+                if erow is None:
+                    rep["rows_s2_skipped"] += 1
+                    continue
+                ids, lp = gpu["child_ids"][s, r], gpu["child_logp"][s, r]
+                err = _check_row(ids, lp, e.s2_logp[erow], T["s2"], f"seq {s} stage-2 row {r}")
+                rep["max_err_s2_emul"] = max(rep["max_err_s2_emul"], err)
+                # reported, not bounded: the plain oracle stores nothing in bf16
+                rep["max_err_s2_plain"] = max(rep["max_err_s2_plain"], float(np.abs(lp - o.s2_logp[erow][ids]).max()))
+                rep["max_emul_minus_plain"] = max(rep["max_emul_minus_plain"],
+                                                  float(np.abs(e.s2_logp[erow][ids] - o.s2_logp[erow][ids]).max()))
+                rep["rows_s2"] += 1
+        # ---- tree: valid, its mask exact, and its structure against the reference oracle's
+        _check_tree_valid(cfg, gpu, s)
+        par, dep = gpu["node_parent"][s], gpu["node_depth"][s]
+        m, pos = O.tree_mask(par.astype(np.int64), dep.astype(np.int64), int(gpu["root_pos"][s]))
+        np.testing.assert_array_equal(gpu["mask"][s], m, err_msg=f"seq {s} mask of own tree")
+        np.testing.assert_array_equal(gpu["pos_ids"][s], pos, err_msg=f"seq {s} pos of own tree")
+        if not same_sets:
+            rep["excluded_trees"] += 1
+            continue
+        tau = T["node"] if ar else g * T["s1"]
+        _compare_cuts(cfg, gpu, s, e, tau, rep)
     return rep
+
+
+def _compare_cuts(cfg, gpu, s, e, tau, rep):
+    """Structure of the GPU's tree against the oracle result e wherever tau decides it.
+
+    The oracle's universe in pop order (the B best nodes and UNIVERSE_EXTRA more) has scores
+    s_1 >= s_2 >= ...; every GPU node score is within tau of the oracle's score of the same
+    path. The set of the j best nodes is then the same on both sides whenever
+    min over i <= j of (s_i - tau) > max over i > j of (s_i + tau) (nodes beyond the listed
+    ones score at most the last listed score). At every such cut j the GPU's first j nodes must
+    be the oracle's first j nodes as a set of token paths; over the longest run of such cuts from
+    j = 1 the pop order is fixed, so tokens, parents and depths must match bit for bit; with every
+    cut up to B decided the whole tree, its mask and position ids must."""
+    B = cfg.B
+    src = O.ChildSource(cfg.mode, cfg.gamma, cfg.M, e.top_ids, e.s1_logp, e.s2_logp, cfg.approx)
+    root = int(e.tree.tok[0])
+    keep = cfg.K2 if cfg.K2 < B else None
+    big = O.build_tree_lazy(src, root, B + UNIVERSE_EXTRA, keep)
+    pops = np.array([p[0] for p in big.pops], dtype=np.float64)
+    ep = O.tree_paths(big)
+    n = len(pops)
+    gp = []
+    paths = {0: ()}
+    for i in range(1, B + 1):
+        if gpu["node_parent"][s, i] < 0:
+            gp.append(None)
+            continue
+        paths[i] = paths[int(gpu["node_parent"][s, i])] + (int(gpu["node_tok"][s, i]),)
+        gp.append(paths[i])
+    # GPU node scores against the oracle's scores of the same paths
+    es = dict(zip(ep, pops))
+    for i, p in enumerate(gp):
+        if p is not None and p in es:
+            err = abs(float(gpu["node_score"][s, i + 1]) - es[p])
+            assert err <= tau, f"seq {s} node {i + 1}: score off by {err:.3g} > {tau}"
+            rep["max_err_node"] = max(rep["max_err_node"], err)
+    lo = np.minimum.accumulate(pops - tau)
+    hi = np.maximum.accumulate((pops + tau)[::-1])[::-1]
+    tail = pops[-1] + tau if n == B + UNIVERSE_EXTRA else -np.inf   # else the universe is exhausted
+    decided = []
+    for j in range(1, min(B, n) + 1):
+        outside = max(hi[j] if j < n else -np.inf, tail)
+        if lo[j - 1] > outside:
+            decided.append(j)
+            assert set(gp[:j]) == set(ep[:j]), f"seq {s}: the best {j} nodes differ from the oracle's"
+    rep["cuts"] += B
+    rep["cuts_determined"] += len(decided)
+    prefix = 0
+    while prefix < len(decided) and decided[prefix] == prefix + 1:
+        prefix += 1
+    ref_tok, ref_par, ref_dep = big.tok[: B + 1], big.parent[: B + 1], big.depth[: B + 1]
+    np.testing.assert_array_equal(gpu["node_tok"][s, : prefix + 1], ref_tok[: prefix + 1], err_msg=f"seq {s} tokens")
+    np.testing.assert_array_equal(gpu["node_parent"][s, : prefix + 1], ref_par[: prefix + 1], err_msg=f"seq {s} parents")
+    np.testing.assert_array_equal(gpu["node_depth"][s, : prefix + 1], ref_dep[: prefix + 1], err_msg=f"seq {s} depths")
+    rep["prefix_nodes"] += prefix
+    if prefix == B and n >= B:
+        m, pos = O.tree_mask(ref_par.astype(np.int64), ref_dep.astype(np.int64), int(gpu["root_pos"][s]))
+        np.testing.assert_array_equal(gpu["mask"][s], m, err_msg=f"seq {s} mask")
+        np.testing.assert_array_equal(gpu["pos_ids"][s], pos, err_msg=f"seq {s} pos")
+        rep["exact_trees"] += 1
+    elif B in decided:
+        rep["set_trees"] += 1

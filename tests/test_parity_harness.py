@@ -81,3 +81,62 @@ def test_harness_rejects_two_prev_rows_swapped_within_a_depth():
         g[k][0, [r, r + 1]] = g[k][0, [r + 1, r]]
     with pytest.raises(AssertionError):
         parity.compare(cfg, g, orc, 1e-4, 1e-3, check_structure=False)
+
+
+# ------------------------------------------------------------------ the bf16 end-to-end contract
+
+
+def _bf16_case(B=16, seed=0):
+    cfg = synth.get_config("tiny_peaked", batch=2, K2=B, B=B)
+    inp = synth.make_inputs(cfg, seed=seed)
+    orc = parity.run_oracle(cfg, inp)
+    orc_e = parity.run_oracle(cfg, inp, emulate_bf16=True)
+    return cfg, inp, orc, orc_e
+
+
+def test_bf16_contract_accepts_the_emulating_oracle():
+    # the emulating oracle's own outputs pass, with every cut decided (its scores are exact
+    # against itself) and the whole tree compared bit for bit
+    cfg, inp, orc, orc_e = _bf16_case()
+    g = fake_gpu(cfg, orc_e, inp["root_pos"].numpy())
+    rep = parity.check_bf16_end_to_end(cfg, g, orc, orc_e)
+    assert rep["excluded_trees"] == 0 and rep["rows_s2"] == 2 * cfg.R
+    assert rep["cuts"] == 2 * cfg.B and rep["cuts_determined"] > 0
+    assert rep["exact_trees"] + rep["set_trees"] <= 2
+    assert rep["max_err_node"] < 1e-5
+
+
+def test_bf16_contract_rejects_a_swapped_node_at_a_decided_cut():
+    # replace the last node of a tree by the best node left out: wherever the cut at B is
+    # decided, the contract must notice
+    cfg, inp, orc, orc_e = _bf16_case()
+    base = fake_gpu(cfg, orc_e, inp["root_pos"].numpy())
+    hit = 0
+    for s in range(cfg.batch):
+        e = orc_e[s]
+        src = O.ChildSource(cfg.mode, cfg.gamma, cfg.M, e.top_ids, e.s1_logp, e.s2_logp)
+        big = O.build_tree_lazy(src, int(e.tree.tok[0]), cfg.B + 1)
+        pops = [p[0] for p in big.pops]
+        if pops[cfg.B - 1] - pops[cfg.B] <= 2 * parity.BF16["node"]:
+            continue          # the cut at B is not decided: nothing to assert there
+        if big.parent[cfg.B + 1] == cfg.B:
+            continue          # the left-out node hangs below the node it would replace
+        g = {k: (v.copy() if isinstance(v, np.ndarray) else v) for k, v in base.items()}
+        for k, src_arr in (("node_tok", big.tok), ("node_parent", big.parent), ("node_depth", big.depth)):
+            g[k][s, cfg.B] = src_arr[cfg.B + 1]
+        g["node_score"][s, cfg.B] = pops[cfg.B]
+        m, pos = O.tree_mask(g["node_parent"][s].astype(np.int64), g["node_depth"][s].astype(np.int64),
+                             int(g["root_pos"][s]))
+        g["mask"][s], g["pos_ids"][s] = m, pos
+        with pytest.raises(AssertionError):
+            parity.check_bf16_end_to_end(cfg, g, orc, orc_e)
+        hit += 1
+    assert hit > 0, "no sequence with a decided cut at B to plant the mistake in"
+
+
+def test_bf16_contract_rejects_stage2_values_beyond_the_bound():
+    cfg, inp, orc, orc_e = _bf16_case()
+    g = fake_gpu(cfg, orc_e, inp["root_pos"].numpy())
+    g["child_logp"][0, 3, 0] += 1.5 * parity.BF16["s2"]
+    with pytest.raises(AssertionError):
+        parity.check_bf16_end_to_end(cfg, g, orc, orc_e)
