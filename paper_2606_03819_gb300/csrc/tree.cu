@@ -650,6 +650,205 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
 }
 
 // ------------------------------------------------------------------------------------------
+// Builder with a sorted queue, for the one-token rule and the marginal modes with B <= 64 and
+// every reachable list entry staged. The same pops, tie rules and results as
+// build_tree_reg_kernel. After t pops only the B - t best live entries can still be popped (each
+// needs every better entry popped first), and at most t + 1 entries are live (a pop replaces its
+// entry by the next sibling and adds at most the node's first child), so at most
+// min(t + 1, B - t) <= 32 entries matter: lane i of one warp holds the i-th best. A pop takes
+// lane 0's entry, tests its token against the stage-1 candidates of its depth with a ballot
+// (the M-ary rule), and places its two successors (next sibling, first child) with two ballots
+// over the remaining keys; every lane then takes its new entry from itself or a neighbour by
+// shuffle. There is no warp-wide max and no divergent branch; a pop costs about 300 ns on
+// GB300, a chain of some hundred dependent single-warp instructions.
+// ------------------------------------------------------------------------------------------
+constexpr int kFastThreads = 512;
+// Shared-memory bytes of build_tree_fast_kernel: nodes, candidates, mask bits and the staged
+// lists (token and log-probability of every entry).
+__host__ __device__ inline size_t fast_tree_smem(int B, int gamma, int M, int rows, int sw, bool with_mask) {
+    const size_t n = static_cast<size_t>(B) + 1;
+    size_t bytes = n * 16 + static_cast<size_t>(gamma) * M * 4;
+    bytes = (bytes + 15) & ~static_cast<size_t>(15);
+    if (with_mask) bytes += (tree_mask_words(static_cast<int>(n)) * 4 + 15) & ~static_cast<size_t>(15);
+    return bytes + static_cast<size_t>(rows) * sw * 8 + 16;
+}
+
+__device__ __forceinline__ bool key_gt(uint32_t ahi, uint32_t alo, uint32_t bhi, uint32_t blo) {
+    return ahi > bhi || (ahi == bhi && alo > blo);
+}
+
+__global__ void __launch_bounds__(kFastThreads) build_tree_fast_kernel(TreeArgs a, int sw) {
+    pdl_trigger();
+    pdl_wait();
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    constexpr unsigned kFull = 0xffffffffu;
+    const int n_out = a.B + 1, s = blockIdx.x, tid = threadIdx.x;
+    const int T = blockDim.x;
+    const bool ar = a.mode == TF_MODE_AR, mary = a.mode != TF_MODE_MARGINAL;
+    const int rows_l = ar ? a.R : a.gamma;
+    const int stride = ar ? a.K2 : a.K1;
+    // every array is carved by a byte offset into smem_raw, so that all accesses stay
+    // shared-memory accesses
+    int* o_tok = reinterpret_cast<int*>(smem_raw);
+    int* o_par = o_tok + n_out;
+    int* o_dep = o_par + n_out;
+    float* o_score = reinterpret_cast<float*>(o_dep + n_out);
+    int* topm = reinterpret_cast<int*>(o_score + n_out);
+    size_t off = (static_cast<size_t>(reinterpret_cast<uint8_t*>(topm + a.gamma * a.M) - smem_raw) + 15) & ~static_cast<size_t>(15);
+    uint32_t* anc = reinterpret_cast<uint32_t*>(smem_raw + off);
+    if (a.mask) off += (tree_mask_words(n_out) * 4 + 15) & ~static_cast<size_t>(15);
+    const int n = rows_l * sw;
+    int* l_tok = reinterpret_cast<int*>(smem_raw + off);
+    float* l_lp = reinterpret_cast<float*>(l_tok + n);
+
+    // ---- the lists and the stage-1 candidates
+    const int32_t* g_ids = ar ? a.child_ids + static_cast<size_t>(s) * a.R * a.K2
+                              : a.top_ids + static_cast<size_t>(s) * a.gamma * a.K1;
+    const float* g_lp = ar ? a.child_logp + static_cast<size_t>(s) * a.R * a.K2
+                           : a.top_logp + static_cast<size_t>(s) * a.gamma * a.K1;
+    const bool vec = sw == stride && (sw & 3) == 0 &&
+                     ((reinterpret_cast<uintptr_t>(g_ids) | reinterpret_cast<uintptr_t>(g_lp)) & 15) == 0;
+    if (vec) {
+        const int n4 = n >> 2;
+        const int4* gi = reinterpret_cast<const int4*>(g_ids);
+        const float4* gl = reinterpret_cast<const float4*>(g_lp);
+        for (int base = tid; base < n4; base += 8 * T) {
+            int4 vi[8];
+            float4 vl[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                if (base + u * T < n4) {
+                    vi[u] = gi[base + u * T];
+                    vl[u] = gl[base + u * T];
+                }
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                if (base + u * T < n4) {
+                    reinterpret_cast<int4*>(l_tok)[base + u * T] = vi[u];
+                    reinterpret_cast<float4*>(l_lp)[base + u * T] = vl[u];
+                }
+        }
+    } else {
+        for (int i = tid; i < n; i += T) {
+            const int r = i / sw;
+            const size_t g = static_cast<size_t>(r) * stride + (i - r * sw);
+            l_tok[i] = g_ids[g];
+            l_lp[i] = g_lp[g];
+        }
+    }
+    for (int i = tid; i < a.gamma * a.M; i += T)
+        topm[i] = a.top_ids[(static_cast<size_t>(s) * a.gamma + i / a.M) * a.K1 + i % a.M];
+    __syncthreads();
+    // ---- the pops (one warp): lane i holds the i-th best live entry, as its key (score, depth,
+    // parent), its list entry (row << 10 | rank) and its parent's score; key 0 marks an empty lane
+    if (tid < 32) {
+        const int lane = tid;
+        const int list_len = a.K2 < sw ? a.K2 : sw;   // staged ranks; a pop never reaches rank sw
+        int flags = 0;
+        const int root = a.root_tok[s];
+        if (root < 0 || root >= a.V) flags |= TF_DEV_BAD_TOKEN;
+        uint32_t khi = 0u, klo = 0u;
+        int rr = 0;
+        float psc = 0.0f;
+        if (lane == 0) {
+            const unsigned long long k0 = queue_key(l_lp[0], 1, 0);
+            khi = static_cast<uint32_t>(k0 >> 32);
+            klo = static_cast<uint32_t>(k0);
+            o_tok[0] = root;
+            o_par[0] = -1;
+            o_dep[0] = 0;
+            o_score[0] = 0.0f;
+        }
+        int count = 1;    // nodes placed
+        while (count < n_out) {
+            // the head: lane 0's entry
+            const uint32_t hhi = __shfl_sync(kFull, khi, 0);
+            if (hhi == 0u) break;                      // queue empty
+            const uint32_t hlo = __shfl_sync(kFull, klo, 0);
+            const int hrr = __shfl_sync(kFull, rr, 0);
+            const float hpsc = __shfl_sync(kFull, psc, 0);
+            // the rest shifted by one: lane i sees entries i + 1 (next) and i - 1 (prev)
+            uint32_t nhi = __shfl_down_sync(kFull, khi, 1), nlo = __shfl_down_sync(kFull, klo, 1);
+            const int nrr = __shfl_down_sync(kFull, rr, 1);
+            const float npsc = __shfl_down_sync(kFull, psc, 1);
+            if (lane == 31) nhi = nlo = 0u;
+            const uint32_t phi = __shfl_up_sync(kFull, khi, 1), plo = __shfl_up_sync(kFull, klo, 1);
+            const int prr = __shfl_up_sync(kFull, rr, 1);
+            const float ppsc = __shfl_up_sync(kFull, psc, 1);
+            // the popped node
+            const int row = hrr >> 10, rank = hrr & 1023, idx = row * sw + rank;
+            const int dep = 127 - static_cast<int>(hlo >> 24);
+            const int par = 0xFFFFFF - static_cast<int>(hlo & 0xFFFFFFu);
+            const float sc = key_float(hhi);
+            const int node = count++;
+            const int tok = l_tok[idx];
+            // its children: none at the depth cap; DDTree: the next depth's marginal row;
+            // otherwise only for a stage-1 candidate m of its depth (Algorithm 1 Part 2), found by
+            // ballots over the depth's candidates (the first equal one counts): stage-2 row
+            // 1 + (dep - 1) M + m, or the next marginal row
+            const int* cand = topm + (dep < a.gamma && mary ? (dep - 1) * a.M : 0);
+            const int c0 = lane < a.M ? cand[lane] : -1, c1 = lane + 32 < a.M ? cand[lane + 32] : -1;
+            const unsigned b0 = __ballot_sync(kFull, lane < a.M && c0 == tok);
+            const unsigned b1 = __ballot_sync(kFull, lane + 32 < a.M && c1 == tok);
+            const int m = b0 ? __ffs(b0) - 1 : b1 ? 32 + __ffs(b1) - 1 : -1;
+            const int crow = dep >= a.gamma ? -1 : !mary ? dep : m < 0 ? -1 : ar ? 1 + (dep - 1) * a.M + m : dep;
+            const bool sib_ok = rank + 1 < list_len;
+            const float slp = l_lp[sib_ok ? idx + 1 : idx];
+            const bool ch_ok = crow >= 0 && node + 1 < n_out;   // nothing is popped after the last node
+            const float clp = l_lp[ch_ok ? crow * sw : 0];
+            if (lane == 0) {
+                if (tok < 0 || tok >= a.V) flags |= TF_DEV_BAD_TOKEN;
+                if (!isfinite(sc)) flags |= TF_DEV_NONFINITE;
+                o_tok[node] = tok;
+                o_par[node] = par;
+                o_dep[node] = dep;
+                o_score[node] = sc;
+            }
+            // its successors, A before B in queue order (0 = none)
+            const unsigned long long sk = sib_ok ? queue_key(hpsc + slp, dep, par) : 0ull;
+            const unsigned long long ckk = ch_ok ? queue_key(sc + clp, dep + 1, node) : 0ull;
+            const bool s_first = sk > ckk;
+            const unsigned long long kA = s_first ? sk : ckk, kB = s_first ? ckk : sk;
+            const uint32_t ahi = static_cast<uint32_t>(kA >> 32), alo = static_cast<uint32_t>(kA);
+            const uint32_t bhi = static_cast<uint32_t>(kB >> 32), blo = static_cast<uint32_t>(kB);
+            const int arr = s_first ? hrr + 1 : crow << 10, brr = s_first ? crow << 10 : hrr + 1;
+            const float apsc = s_first ? hpsc : sc, bpsc = s_first ? sc : hpsc;
+            // their places among the remaining entries (sorted, so the larger keys are a prefix)
+            const int pA = __popc(__ballot_sync(kFull, key_gt(nhi, nlo, ahi, alo)));
+            const int pB = __popc(__ballot_sync(kFull, key_gt(nhi, nlo, bhi, blo)));
+            // new entry i: rest[i] before A, A, rest[i - 1] up to B, B, rest[i - 2] after it
+            const int j = lane;
+            const bool takeA = j == pA, takeB = j == pB + 1;
+            const bool fromN = j < pA, fromO = j > pA && j <= pB;
+            khi = takeA ? ahi : takeB ? bhi : fromN ? nhi : fromO ? khi : phi;
+            klo = takeA ? alo : takeB ? blo : fromN ? nlo : fromO ? klo : plo;
+            rr = takeA ? arr : takeB ? brr : fromN ? nrr : fromO ? rr : prr;
+            psc = takeA ? apsc : takeB ? bpsc : fromN ? npsc : fromO ? psc : ppsc;
+        }
+        flags = static_cast<int>(__reduce_or_sync(kFull, static_cast<unsigned>(flags)));
+        if (count < n_out) flags |= TF_DEV_UNDERFULL;
+        for (int i = count + lane; i < n_out; i += 32) {
+            o_tok[i] = -1;
+            o_par[i] = -1;
+            o_dep[i] = -1;
+            o_score[i] = -INFINITY;
+        }
+        if (lane == 0) a.dev_status[s] = flags;
+    }
+    __syncthreads();
+    for (int i = tid; i < n_out; i += T) {
+        const size_t o = static_cast<size_t>(s) * n_out + i;
+        a.node_tok[o] = o_tok[i];
+        a.node_parent[o] = o_par[i];
+        a.node_depth[o] = o_dep[i];
+        a.node_score[o] = o_score[i];
+    }
+    if (a.mask)
+        mask_rows(n_out, o_par, o_dep, a.root_pos[s], 0, n_out, anc, a.mask + static_cast<size_t>(s) * n_out * n_out,
+                  a.pos_ids + static_cast<size_t>(s) * n_out);
+}
+
+// ------------------------------------------------------------------------------------------
 // The tree-attention mask and position ids (mask_rows) of a drafted tree in global memory: one
 // CTA per sequence and block of kMaskRows rows.
 // ------------------------------------------------------------------------------------------
@@ -912,8 +1111,22 @@ cudaError_t launch_build_tree(const Ctx& ctx, int b, int gamma, int M, int K1, i
         sw = static_cast<int>(room / (static_cast<size_t>(rows_l) * 8)) & ~3;
         if (sw > sw_full) sw = sw_full;
     }
+    // the builder with precomputed successors for the one-token rule and the marginal modes
+    // whenever B + 1 slots fit in four registers per lane and every reachable entry is staged
+    // the sorted-queue builder for the one-token rule and the marginal modes with B <= 64 and
+    // every reachable entry staged
+    if (!a.two_prev && B <= 64) {
+        const size_t fsm = fast_tree_smem(B, gamma, M, rows_l, sw_full, mask != nullptr);
+        if (fsm <= kTreeSmemLimit) {
+            cudaError_t e = cudaFuncSetAttribute(build_tree_fast_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 static_cast<int>(fsm));
+            if (e != cudaSuccess) return e;
+            e = launch_pdl(build_tree_fast_kernel, dim3(b), dim3(kFastThreads), fsm, ctx.stream, a, sw_full);
+            return e != cudaSuccess ? e : cudaGetLastError();
+        }
+    }
     const size_t smem = fixed + tree_smem_lists(rows_l, sw);
-    // the register-queue builder whenever B + 1 slots fit in four registers per lane
+    // otherwise the register-queue builder whenever B + 1 slots fit in four registers per lane
     const bool full = sw == sw_full;
     void (*kern)(TreeArgs, int) =
         B + 1 <= 32    ? (full ? build_tree_reg_kernel<1, true> : build_tree_reg_kernel<1, false>)
