@@ -42,21 +42,15 @@ __device__ unsigned long long block_kth_largest(const unsigned long long* keys, 
     unsigned long long prefix = 0;
     int rem = k;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int n_pad = (n + kThreads - 1) / kThreads * kThreads;
     for (int shift = 56; shift >= 0; shift -= 8) {
         for (int i = tid; i < 256; i += kThreads) hist[i] = 0;
         __syncthreads();
         const unsigned long long hi_mask = shift == 56 ? 0ull : (~0ull << (shift + 8));
-        // warp-aggregated counting: lanes holding the same digit add once (plain atomics would
-        // serialise on the few bins the keys of one row fall into)
-        for (int i = tid; i < n_pad; i += kThreads) {
-            int digit = 256;
-            if (i < n) {
-                const unsigned long long key = keys[i];
-                if ((key & hi_mask) == prefix) digit = static_cast<int>((key >> shift) & 255);
-            }
-            const unsigned peers = __match_any_sync(0xffffffffu, digit);
-            if (digit < 256 && lane == __ffs(peers) - 1) atomicAdd(&hist[digit], __popc(peers));
+        // shared-memory atomics: lanes of a warp on one bin are combined by the hardware (a
+        // warp match to aggregate them first costs far more on GB300)
+        for (int i = tid; i < n; i += kThreads) {
+            const unsigned long long key = keys[i];
+            if ((key & hi_mask) == prefix) atomicAdd(&hist[static_cast<int>((key >> shift) & 255)], 1);
         }
         __syncthreads();
         if (warp == 0) {
@@ -180,15 +174,9 @@ __device__ unsigned long long block_kth_largest_fast(const unsigned long long* k
         const int b = static_cast<int>((key_value(key) - vlo) * scale);
         return b < 0 ? 0 : (b >= kBuckets ? kBuckets - 1 : b);
     };
-    const int n_pad = (n + kThreads - 1) / kThreads * kThreads;
-    for (int i = tid; i < n_pad; i += kThreads) {
-        int b = kBuckets;
-        if (i < n) {
-            const unsigned long long key = keys[i];
-            if (key != 0ull) b = bucket_of(key);
-        }
-        const unsigned peers = __match_any_sync(0xffffffffu, b);
-        if (b < kBuckets && lane == __ffs(peers) - 1) atomicAdd(&B.hist[b], __popc(peers));
+    for (int i = tid; i < n; i += kThreads) {
+        const unsigned long long key = keys[i];
+        if (key != 0ull) atomicAdd(&B.hist[bucket_of(key)], 1);
     }
     __syncthreads();
     if (warp == 0) {
