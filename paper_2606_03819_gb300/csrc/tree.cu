@@ -949,13 +949,15 @@ __device__ __forceinline__ __nv_bfloat16 bf16_round_sum(float r, float t) {
 
 // bf16 rows with d % 8 == 0: 16-byte loads and stores, 8 elements per thread and step. x is the
 // correctly rounded bf16 value of the definition (an element off by one bf16 ulp would perturb
-// every gate/up output and flip many later roundings), computed without per-element fp64 work:
-//  - mean(h^2): every square of a bf16 value is exact in fp32; the sums are compensated
-//    (TwoSum), widened to fp64 only once per thread for the block reduction;
-//  - 1 / sqrt(mean + eps) in fp64 once per row, split into fp32 hi + lo;
+// every gate/up output and flip many later roundings), computed in fp32 only (GB300's fp64 is too
+// slow even for the few scalar steps of a row):
+//  - mean(h^2): every square of a bf16 value is exact in fp32; the sums, and their warp and block
+//    reductions, are compensated (TwoSum pairs);
+//  - 1 / sqrt(mean + eps) as hi + lo: hi = rsqrtf, then one Newton step in double-float
+//    arithmetic (the squares and products formed exactly with FMAs), about 2^-46 relative;
 //  - h * w is exact in fp32 (two 8-bit significands); (h w) * hi is rounded once and its
 //    rounding error recovered with an FMA, so (h w) / sqrt(mean + eps) is known as r + t to
-//    about 2^-47 relative, which decides the bf16 rounding (bf16_round_sum).
+//    about 2^-45 relative, which decides the bf16 rounding (bf16_round_sum).
 template <int NE>
 __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
     const uint4* __restrict__ hidden, const uint4* __restrict__ embed, const uint4* __restrict__ norm_h,
@@ -965,20 +967,24 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
     pdl_trigger();
     constexpr int kMaxPerThread = 4;          // d <= 256 * 8 * 4 = 8192
     constexpr int NS = 1 + NE;                // parts of x: the hidden state, then NE embeddings
-    __shared__ double red[NS][8];
+    __shared__ float red[NS][2][8];
     __shared__ float scale[2 * NS];           // hi, lo of 1 / sqrt(mean + eps) of every part
     const int row = blockIdx.x;
     const int hid = stage2_row_hidden(row, R, gamma, M, NE == 2);
 
     const int dv = d / 8;
-    // the hidden state is a step input (no kernel writes it): read before waiting for the
-    // previous kernel, which produces the candidate tokens
+    // the hidden state and the norm weights are step inputs (no kernel writes them): read before
+    // waiting for the previous kernel, which produces the candidate tokens
     const uint4* h = hidden + static_cast<size_t>(hid) * dv;
-    uint4 v[NS][kMaxPerThread];
+    uint4 v[NS][kMaxPerThread], wh[kMaxPerThread], we[kMaxPerThread];
 #pragma unroll
     for (int i = 0; i < kMaxPerThread; ++i) {
         const int c = threadIdx.x + i * 256;
-        if (c < dv) v[0][i] = h[c];
+        if (c < dv) {
+            v[0][i] = h[c];
+            wh[i] = norm_h[c];
+            we[i] = norm_e[c];
+        }
     }
     pdl_wait();
     int tok[2] = {0, 0};
@@ -996,6 +1002,8 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
             if (c < dv) v[1 + j][i] = e[c];
         }
     }
+    // sums of squares: every square of a bf16 value is exact in fp32; the running sums are
+    // compensated (TwoSum), and the (sum, compensation) pairs are combined the same way
     float sum[NS], comp[NS];
 #pragma unroll
     for (int j = 0; j < NS; ++j) sum[j] = comp[j] = 0.0f;
@@ -1014,25 +1022,49 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
             }
         }
     }
-    double dsum[NS];
-#pragma unroll
-    for (int j = 0; j < NS; ++j) dsum[j] = static_cast<double>(sum[j]) + static_cast<double>(comp[j]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1)
 #pragma unroll
-        for (int j = 0; j < NS; ++j) dsum[j] += __shfl_xor_sync(0xffffffffu, dsum[j], o);
+        for (int j = 0; j < NS; ++j) {
+            const float s2 = __shfl_xor_sync(0xffffffffu, sum[j], o);
+            const float c2 = __shfl_xor_sync(0xffffffffu, comp[j], o);
+            two_sum_acc(sum[j], comp[j], s2);
+            comp[j] += c2;
+        }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0)
 #pragma unroll
-        for (int j = 0; j < NS; ++j) red[j][warp] = dsum[j];
+        for (int j = 0; j < NS; ++j) {
+            red[j][0][warp] = sum[j];
+            red[j][1][warp] = comp[j];
+        }
     __syncthreads();
     if (threadIdx.x < NS) {
-        double a = 0.0;
-        for (int w = 0; w < 8; ++w) a += red[threadIdx.x][w];
-        const double inv = 1.0 / sqrt(a / d + static_cast<double>(eps));
-        const float hi = __double2float_rn(inv);
-        scale[2 * threadIdx.x] = hi;
-        scale[2 * threadIdx.x + 1] = __double2float_rn(inv - static_cast<double>(hi));
+        const int j = threadIdx.x;
+        float S = 0.0f, C = 0.0f;
+        for (int w = 0; w < 8; ++w) {
+            two_sum_acc(S, C, red[j][0][w]);
+            C += red[j][1][w];
+        }
+        // m = (S + C) / d + eps as a double-float (mh, ml); d is scaled exactly when it is a
+        // power of two, otherwise the quotient's rounding error is recovered by an FMA
+        const float fd = static_cast<float>(d);
+        const float q = S / fd;
+        const float qerr = fmaf(-q, fd, S) / fd + C / fd;
+        float mh = q + eps;
+        float ml = (q - (mh - (mh - q))) + (eps - (mh - q)) + qerr;   // TwoSum(q, eps) plus the rest
+        const float t = mh + ml;
+        ml = ml - (t - mh);
+        mh = t;
+        // y = 1 / sqrt(m): y0 = rsqrtf(mh), then one Newton step in double-float arithmetic,
+        // y = y0 + y0 (1 - m y0^2) / 2, with y0^2 and m y0^2 formed by exact FMA products
+        const float y0 = rsqrtf(mh);
+        const float p = y0 * y0, pl = fmaf(y0, y0, -p);          // y0^2 = p + pl exactly
+        const float u = mh * p, ul = fmaf(mh, p, -u);              // mh p = u + ul exactly
+        const float r = ((1.0f - u) - ul) - (mh * pl + ml * p);    // 1 - m y0^2, ~2^-23
+        const float hi = y0, lo = 0.5f * y0 * r;
+        scale[2 * j] = hi;
+        scale[2 * j + 1] = lo;
     }
     __syncthreads();
     uint4* xr = X + static_cast<size_t>(row) * NS * dv;
@@ -1040,19 +1072,18 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
     for (int i = 0; i < kMaxPerThread; ++i) {
         const int c = threadIdx.x + i * 256;
         if (c < dv) {
-            const uint4 wh = norm_h[c], we = norm_e[c];
 #pragma unroll
             for (int j = 0; j < NS; ++j) {
                 const float is = scale[2 * j], is_lo = scale[2 * j + 1];
                 const __nv_bfloat16* b = reinterpret_cast<const __nv_bfloat16*>(&v[j][i]);
-                const __nv_bfloat16* wb = reinterpret_cast<const __nv_bfloat16*>(j == 0 ? &wh : &we);
+                const __nv_bfloat16* wb = reinterpret_cast<const __nv_bfloat16*>(j == 0 ? &wh[i] : &we[i]);
                 uint4 o;
                 __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(&o);
 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
-                    const float p = __bfloat162float(b[k]) * __bfloat162float(wb[k]);
-                    const float r = p * is;
-                    ob[k] = bf16_round_sum(r, fmaf(p, is_lo, fmaf(p, is, -r)));
+                    const float pv = __bfloat162float(b[k]) * __bfloat162float(wb[k]);
+                    const float rv = pv * is;
+                    ob[k] = bf16_round_sum(rv, fmaf(pv, is_lo, fmaf(pv, is, -rv)));
                 }
                 xr[j * dv + c] = o;
             }
