@@ -116,10 +116,16 @@ Layout layout(const Dims& D) {
     L.A = take(rows2 * D.I * D.esize);
     L.hp = take(rows2 * D.d * D.esize);
     L.hres = take(D.two_prev ? rows2 * D.d * D.esize : 0);   // residual row of each stage-2 row
-    // split-K partial sums of the bf16 approximator GEMMs: [k_splits][max(2I, d) / 4][rows][4] fp32
-    L.kpart = D.dtype == TF_BF16 ? take(static_cast<size_t>(kMaxKSplits) * rows2 *
-                                        (2 * static_cast<size_t>(D.I) > static_cast<size_t>(D.d) ? 2 * D.I : D.d) * 4)
-                                 : take(0);
+    // split-K partial sums of the bf16 approximator GEMMs: [k_splits][max(2I, d) / 4][rows][4] fp32,
+    // or the exchange area of their cluster path, whichever is larger
+    if (D.dtype == TF_BF16) {
+        const size_t partial = static_cast<size_t>(kMaxKSplits) * rows2 *
+                               (2 * static_cast<size_t>(D.I) > static_cast<size_t>(D.d) ? 2 * D.I : D.d) * 4;
+        const size_t xg = std::max(splitk_exchange_bytes(D.I, 2), splitk_exchange_bytes(D.d, 1));
+        L.kpart = take(rows2 > 0 ? std::max(partial, xg) : 0);
+    } else {
+        L.kpart = take(0);
+    }
     L.h_hidden = take(rows1 * D.d * D.esize);
     L.h_root = take(static_cast<size_t>(D.b) * D.root_stride * sizeof(int32_t));
     L.h_pos = take(D.b * sizeof(int32_t));

@@ -176,6 +176,9 @@ cudaError_t launch_swiglu_tc(const Ctx&, const void* X, int k_in, const void* w_
                              const void* w_up, const void* w_down, const void* hidden, int n_rows,
                              int d, int I, int R, int M, int gamma, void* A, void* h_prime,
                              float* partial);
+// bytes of the split-K exchange area of the cluster path for a GEMM with n_out_cols output columns
+// made of nb adjacent matrices (the workspace's partial-sum region must hold it)
+size_t splitk_exchange_bytes(int n_out_cols, int nb);
 // split-K reductions of the approximator GEMMs (partial sums in fp32, [k_splits][N / 4][rows][4])
 cudaError_t launch_swiglu_reduce(const Ctx&, const float* partial, int k_splits, int n_rows, int I,
                                  __nv_bfloat16* A);

@@ -576,44 +576,43 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         // ------------------------------------------------------------------ split-K sum
         // The tile's output columns are owned in CL blocks of BN / CL: CTA o adds the CL partial
         // sums of block o in K-range order (the order of the split-K reduction kernels) and
-        // applies the epilogue. Every CTA first writes the blocks it does not own into their
-        // owners' stage rings (idle once all MMAs of the cluster are done), laid out
-        // [16-byte unit][row] so that the 32 lanes (rows) of a warp store 512 contiguous bytes.
+        // applies the epilogue. Every CTA writes the blocks it does not own to the exchange area
+        // in global memory (it stays in L2; through L2 this takes half the time of remote
+        // shared-memory stores), laid out [cluster][owner][sender slot][16-byte unit][row] so that
+        // the 32 lanes (rows) of a warp store and load 512 contiguous bytes; one cluster barrier
+        // (release/acquire at cluster scope) then makes them visible to their owners.
         constexpr int kOwn = BN / CL;                    // output columns per owner
         constexpr int kRowF4 = NB * kOwn / 4;            // 16-byte units per row of a block
-        constexpr int kSlotBytes = MT * kBM * kRowF4 * 16;
+        constexpr int kSlotF4 = MT * kBM * kRowF4;       // 16-byte units of one block
         static_assert(kOwn == 32, "one TMEM load per block and accumulator");
-        static_assert((CL - 1) * kSlotBytes <= STAGES * C::kStageBytes, "the received blocks fit the ring");
         const bool has_unit = cid < n_units;
         const int e = warp - 2;
         const int g = e / (kEpiWarps / 2), q = warp & 3, half = (e % (kEpiWarps / 2)) / 4;
         const int r = g * kBM + q * 32 + lane;           // tile row: TMEM slot g, lane q * 32 + lane
         const uint32_t tb = tmem_base + 256u * g + (static_cast<uint32_t>(q * 32) << 16);
-        const uint32_t ring = ptx::smem_u32(smem);
-        __syncwarp();
-        ptx::tc_fence_before();
-        ptx::cluster_sync();   // all accumulators of the cluster are final; no copy or MMA uses a ring
-        ptx::tc_fence_after();
+        float4* xchg = reinterpret_cast<float4*>(ep.partial);
+        // (the epilogue warps waited for this CTA's accumulators in the loop above)
         if (warp >= 2 && has_unit) {
             // the warp's half of the columns holds the blocks of owners 2 half and 2 half + 1
             for (int o = 2 * half; o < 2 * half + 2; ++o) {
                 if (o == crank) continue;
                 const int slot = crank < o ? crank : crank - 1;
-                const uint32_t dst = ptx::mapa_shared(ring + slot * kSlotBytes + r * 16, o);
+                float4* dst = xchg + (static_cast<size_t>(cid * CL + o) * (CL - 1) + slot) * kSlotF4 + r;
 #pragma unroll
                 for (int nb = 0; nb < NB; ++nb) {
                     uint32_t ra[32];
                     ptx::tmem_ld_32cols(tb + nb * BN + o * kOwn, ra);
 #pragma unroll
                     for (int f = 0; f < 8; ++f)
-                        ptx::st_cluster_f4(dst + (nb * 8 + f) * (MT * kBM * 16), __uint_as_float(ra[4 * f]),
-                                           __uint_as_float(ra[4 * f + 1]), __uint_as_float(ra[4 * f + 2]),
-                                           __uint_as_float(ra[4 * f + 3]));
+                        dst[(nb * 8 + f) * (MT * kBM)] = make_float4(__uint_as_float(ra[4 * f]), __uint_as_float(ra[4 * f + 1]),
+                                                                   __uint_as_float(ra[4 * f + 2]), __uint_as_float(ra[4 * f + 3]));
                 }
             }
         }
         __syncwarp();
-        ptx::cluster_sync();   // every block is in its owner's shared memory
+        ptx::tc_fence_before();
+        ptx::cluster_sync();   // every block is in the exchange area
+        ptx::tc_fence_after();
         if (warp >= 2 && has_unit) {
             // this warp: 16 of the own block's columns, c0 .. c0 + 15 of the tile
             const Unit w = unit_of(cid);
@@ -632,7 +631,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                         for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(ra[j]);
                     } else {
                         const int slot = kx < crank ? kx : kx - 1;
-                        const float4* src = reinterpret_cast<const float4*>(smem + slot * kSlotBytes) + r;
+                        const float4* src = xchg + (static_cast<size_t>(cid * CL + crank) * (CL - 1) + slot) * kSlotF4 + r;
 #pragma unroll
                         for (int f = 0; f < 4; ++f) {
                             const float4 t = src[(nb * 8 + half * 4 + f) * (MT * kBM)];
@@ -781,8 +780,18 @@ cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& t
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+}  // namespace
+
+// Bytes of the split-K exchange area of the cluster path: per output tile (cluster) of 128
+// columns, CL = 4 owners receive 3 blocks of 2 M-tiles x 128 rows x NB x 32 fp32 columns.
+size_t splitk_exchange_bytes(int n_out_cols, int nb) {
+    return static_cast<size_t>(n_out_cols / 128) * 4 * 3 * (2 * 128) * nb * 32 * 4;
+}
+
+namespace {
+
 // Whether n_tiles clusters of the split-K kernel can all be resident at once (each cluster then
-// runs its one tile and the ring can take the partial sums; a second wave would serialise them).
+// runs its one tile; a second wave would serialise them).
 template <int EPI, int MT, int NB, int BN, int STAGES, int CL>
 bool splitk_clusters_fit(const Ctx& ctx, int n_tiles) {
     using C = TileCfg<MT, NB, BN, STAGES>;
