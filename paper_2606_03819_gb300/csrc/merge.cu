@@ -22,7 +22,7 @@
 namespace tf {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 256;   // 512 or more: two CTAs no longer fit an SM, so 241 rows take two waves
 
 __device__ __forceinline__ void lse_combine(float& m, float& s, float m2, float s2) {
     if (m2 > m) {
@@ -145,19 +145,23 @@ __device__ unsigned long long block_kth_largest_fast(const unsigned long long* k
     }
     for (int i = tid; i < kBuckets; i += kThreads) B.hist[i] = 0;
     __syncthreads();
-    if (tid == 0) {
-        float mx = -INFINITY, mn = INFINITY;
-        int c = 0;
-        for (int w = 0; w < kThreads / 32; ++w) {
-            mx = fmaxf(mx, B.wmax[w]);
-            mn = fminf(mn, B.wmin[w]);
-            c += B.wcnt[w];
+    if (warp == 0) {
+        float mx = lane < kThreads / 32 ? B.wmax[lane] : -INFINITY;
+        float mn = lane < kThreads / 32 ? B.wmin[lane] : INFINITY;
+        int c = lane < kThreads / 32 ? B.wcnt[lane] : 0;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+            c += __shfl_xor_sync(0xffffffffu, c, o);
         }
-        B.total = c;
-        B.vmin = mn;
-        const float range = mx - mn;
-        B.scale = (range > 0.0f && isfinite(range)) ? static_cast<float>(kBuckets) / range : 0.0f;
-        B.n_coll = 0;
+        if (lane == 0) {
+            B.total = c;
+            B.vmin = mn;
+            const float range = mx - mn;
+            B.scale = (range > 0.0f && isfinite(range)) ? static_cast<float>(kBuckets) / range : 0.0f;
+            B.n_coll = 0;
+        }
     }
     __syncthreads();
     const int total = B.total;
@@ -383,12 +387,20 @@ __global__ void __launch_bounds__(kThreads) lmhead_merge_kernel(Partials partial
     __syncthreads();
     atomicAdd(&n_valid, my_valid);
     __syncthreads();
-    if (tid == 0) {
-        float M = -INFINITY, Ssum = 0.0f;
-        for (int w = 0; w < kThreads / 32; ++w) lse_combine(M, Ssum, red_m[w], red_s[w]);
-        const float lse = M + logf(Ssum);
-        lse_s = lse;
-        if (!isfinite(lse)) set_status(status, TF_DEV_NONFINITE);
+    if (warp == 0) {
+        float M = lane < kThreads / 32 ? red_m[lane] : -INFINITY;
+        float Ssum = lane < kThreads / 32 ? red_s[lane] : 0.0f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float m2 = __shfl_xor_sync(0xffffffffu, M, o);
+            const float s2 = __shfl_xor_sync(0xffffffffu, Ssum, o);
+            lse_combine(M, Ssum, m2, s2);
+        }
+        if (lane == 0) {
+            const float lse = M + logf(Ssum);
+            lse_s = lse;
+            if (!isfinite(lse)) set_status(status, TF_DEV_NONFINITE);
+        }
     }
 
     // 2. theta0 and the halves at or above it (at most k: the keys are distinct)
