@@ -1142,8 +1142,6 @@ cudaError_t launch_build_tree(const Ctx& ctx, int b, int gamma, int M, int K1, i
         sw = static_cast<int>(room / (static_cast<size_t>(rows_l) * 8)) & ~3;
         if (sw > sw_full) sw = sw_full;
     }
-    // the builder with precomputed successors for the one-token rule and the marginal modes
-    // whenever B + 1 slots fit in four registers per lane and every reachable entry is staged
     // the sorted-queue builder for the one-token rule and the marginal modes with B <= 64 and
     // every reachable entry staged
     if (!a.two_prev && B <= 64) {
