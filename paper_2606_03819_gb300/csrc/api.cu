@@ -39,7 +39,7 @@ struct Dims {
 };
 
 struct Layout {
-    size_t status, halves, chunks, X, A, hp, hres, kpart;
+    size_t status, halves, chunks, X, A, hp, hres, kpart, kpart_bytes;
     size_t h_hidden, h_root, h_pos, top_ids, top_logp, child_ids, child_logp;
     size_t n_tok, n_par, n_dep, n_score, n_mask, n_pos, n_stat;
     size_t total;
@@ -109,7 +109,7 @@ Layout layout(const Dims& D) {
     const size_t rows2 = D.mode == TF_MODE_AR ? static_cast<size_t>(D.b) * D.R : 0;
     const size_t rows = rows1 > rows2 ? rows1 : rows2;
     const size_t nn = static_cast<size_t>(D.b) * (D.B + 1);
-    L.status = take(sizeof(int32_t));
+    L.status = take(sizeof(int32_t) * (1 + kTailSems));   // the status word, then the tail-split counters
     L.halves = take(rows * D.n_tiles * kHalfBytesPerRowBlock);
     L.chunks = take(rows * D.n_tiles * kChunkBytesPerRowBlock);
     L.X = take(rows2 * D.k_in * D.esize);
@@ -122,8 +122,10 @@ Layout layout(const Dims& D) {
         const size_t partial = static_cast<size_t>(kMaxKSplits) * rows2 *
                                (2 * static_cast<size_t>(D.I) > static_cast<size_t>(D.d) ? 2 * D.I : D.d) * 4;
         const size_t xg = std::max(splitk_exchange_bytes(D.I, 2), splitk_exchange_bytes(D.d, 1));
-        L.kpart = take(rows2 > 0 ? std::max(partial, xg) : 0);
+        L.kpart_bytes = rows2 > 0 ? std::max(partial, xg) : 0;
+        L.kpart = take(L.kpart_bytes);
     } else {
+        L.kpart_bytes = 0;
         L.kpart = take(0);
     }
     L.h_hidden = take(rows1 * D.d * D.esize);
@@ -213,7 +215,7 @@ tf_status do_ar_approx(const Ctx& ctx, const Dims& D, const Layout& L, void* ws,
     if (D.approx == TF_APPROX_LINEAR) {
         if (D.dtype == TF_BF16)
             return cuda_status(launch_linear_tc(ctx, X, w->w_lin, hidden, rows, D.d, D.R, D.M, D.gamma, hp,
-                                                at<float>(ws, L.kpart)));
+                                                at<float>(ws, L.kpart), L.kpart_bytes));
         return cuda_status(launch_linear_simt(ctx, X, w->w_lin, hidden, rows, D.d, D.R, D.M, D.gamma, hp));
     }
     // the residual of stage-2 row r is the hidden state of its depth; with two previous tokens the
@@ -222,7 +224,7 @@ tf_status do_ar_approx(const Ctx& ctx, const Dims& D, const Layout& L, void* ws,
     const int rR = D.two_prev ? 1 : D.R, rM = D.two_prev ? 1 : D.M, rG = D.two_prev ? 1 : D.gamma;
     if (D.dtype == TF_BF16)
         return cuda_status(launch_swiglu_tc(ctx, X, D.k_in, w->w_gate, w->w_up, w->w_down, res, rows, D.d, D.I, rR, rM,
-                                            rG, A, hp, at<float>(ws, L.kpart)));
+                                            rG, A, hp, at<float>(ws, L.kpart), L.kpart_bytes));
     return cuda_status(launch_swiglu_simt(ctx, X, D.k_in, w->w_gate, w->w_up, w->w_down, res, rows, D.d, D.I, rR,
                                           rM, rG, A, hp));
 }

@@ -19,6 +19,10 @@ constexpr int kMaxB = 1023;         // largest draft budget
 constexpr int kMaxGamma = 64;
 constexpr int kMergeExpandChunks = 64;     // chunks a merge may recompute exactly
 constexpr int kMaxKSplits = 4;        // split-K factor of the approximator GEMMs (workspace sized for it)
+// Counters of the approximator GEMMs' tail split (K-chunks of the units of a last, partial round),
+// kept in the workspace right after the status word and zeroed by the gather of every call.
+constexpr int kTailSems = 1024;
+constexpr int kMaxTailSplit = 8;       // K-chunks per tail unit
 
 // What the LM-head pass leaves per (row, vocabulary block of 256). Both arrays are indexed
 // [block][part][row], so the 32 lanes of an epilogue warp (32 consecutive rows) store 512
@@ -175,7 +179,7 @@ cudaError_t launch_gather_norm(const Ctx&, int dtype, const void* hidden, const 
 cudaError_t launch_swiglu_tc(const Ctx&, const void* X, int k_in, const void* w_gate,
                              const void* w_up, const void* w_down, const void* hidden, int n_rows,
                              int d, int I, int R, int M, int gamma, void* A, void* h_prime,
-                             float* partial);
+                             float* partial, size_t partial_bytes);
 // bytes of the split-K exchange area of the cluster path for a GEMM with n_out_cols output columns
 // made of nb adjacent matrices (the workspace's partial-sum region must hold it)
 size_t splitk_exchange_bytes(int n_out_cols, int nb);
@@ -192,7 +196,7 @@ cudaError_t launch_swiglu_simt(const Ctx&, const void* X, int k_in, const void* 
 // the "w/ Linear" approximator: h' = h + X W_lin^T, X [n_rows, 2d], W_lin [d, 2d]
 cudaError_t launch_linear_tc(const Ctx&, const void* X, const void* w_lin, const void* hidden,
                              int n_rows, int d, int R, int M, int gamma, void* h_prime,
-                             float* partial);
+                             float* partial, size_t partial_bytes);
 cudaError_t launch_linear_simt(const Ctx&, const void* X, const void* w_lin, const void* hidden,
                                int n_rows, int d, int R, int M, int gamma, void* h_prime);
 // Part 2 and the mask

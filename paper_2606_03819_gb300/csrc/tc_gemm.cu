@@ -62,6 +62,13 @@ struct EpiParams {
     int reset_status;            // LMHEAD: zero *status first (the first kernel of a stage-1 call)
     unsigned long long wait_ns;  // limit of every wait for progress (0: kWaitLimitNs); the waits
                                  // that drain in-flight copies and MMAs always take kWaitLimitNs
+    // GATEUP / DOWN with one CTA per SM: units n_full.. (the last, partial round) run as
+    // tail_split K-chunks each (0: none). A chunk writes its fp32 partial sums to `partial`, laid
+    // out [tail unit][chunk][M-tile][col / 4][128 rows][4]; the chunk that finishes last (counted
+    // in sem[tail unit * MT + M-tile], zero between calls) adds them in chunk order and applies
+    // the epilogue.
+    int n_full, tail_split;
+    int* sem;
 };
 
 // Work unit u -> (N tile, M-tile group, K split); consecutive units share the N tile and K split
@@ -174,6 +181,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     uint64_t* drain = tempty + 2;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    volatile int* last_chunk = abort_flag + 1;   // [2]: this group's chunk was its unit's last
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -191,6 +199,33 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     auto unit_of = [&](int u) {
         if constexpr (kSplitK) return Unit{u / n_mgroups, u % n_mgroups, crank};
         return decode_unit(u, n_mgroups, k_splits);
+    };
+    // Work items: the units, except that with a tail split each unit of the last round becomes
+    // tail_split items over consecutive K-chunks of its range ([kb0, kb1) in K-steps).
+    constexpr bool kTail = CL == 1 && (EPI == EPI_GATEUP || EPI == EPI_DOWN);
+    const int n_split = kTail ? ep.tail_split : 0;
+    const int n_items = n_split ? ep.n_full + (n_units - ep.n_full) * n_split : n_units;
+    struct Item {
+        Unit w;
+        int kb0, kb1, tail, chunk;   // tail unit and chunk index (-1: a whole unit)
+    };
+    auto item_of = [&](int i) {
+        Item it;
+        const int ns = n_split > 0 ? n_split : 1;   // (a constant 1 in kernels without a tail split)
+        if (n_split == 0 || i < ep.n_full) {
+            it.w = unit_of(i);
+            it.kb0 = it.w.kx * nk;
+            it.kb1 = it.kb0 + nk;
+            it.tail = it.chunk = -1;
+        } else {
+            const int r = i - ep.n_full;
+            it.tail = r / ns;
+            it.chunk = r - it.tail * ns;
+            it.w = unit_of(ep.n_full + it.tail);
+            it.kb0 = it.w.kx * nk + nk * it.chunk / ns;
+            it.kb1 = it.w.kx * nk + nk * (it.chunk + 1) / ns;
+        }
+        return it;
     };
     // shared::cluster address of this CTA's barrier `bar` as seen at the same offset in the pair's
     // even CTA (pair mode: the barriers the issuer waits on) or in the odd one
@@ -272,12 +307,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             // The weights are no kernel's output: the first unit's first weight tiles are
             // requested before waiting for the previous kernel (which may be writing X).
             int pre = 0;
-            if (cid < n_units) {
-                const Unit w = unit_of(cid);
-                pre = nk < STAGES ? nk : STAGES;
+            if (cid < n_items) {
+                const Item f = item_of(cid);
+                pre = f.kb1 - f.kb0 < STAGES ? f.kb1 - f.kb0 : STAGES;
                 for (int i = 0; i < pre; ++i) {
                     if (leader) ptx::mbar_arrive_expect_tx(&full[i], kTxBytes);
-                    load_w(smem + i * C::kStageBytes, &full[i], w.kx * nk + i, w.nt);
+                    load_w(smem + i * C::kStageBytes, &full[i], f.kb0 + i, f.w.nt);
                 }
             }
             pdl_wait();
@@ -287,10 +322,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             uint32_t last_parity[STAGES > 0 ? STAGES : 1];
             bool ok = true;
             int it = 0;                               // k-steps issued so far by this CTA
-            for (int u = cid; u < n_units && ok; u += ncl) {
-                const Unit w = unit_of(u);
-                const int nt = w.nt, mt0 = (w.mg * m_cl + m_rank) * MT;
-                for (int kb = w.kx * nk; kb < (w.kx + 1) * nk; ++kb, ++it) {
+            for (int u = cid; u < n_items && ok; u += ncl) {
+                const Item itm = item_of(u);
+                const int nt = itm.w.nt, mt0 = (itm.w.mg * m_cl + m_rank) * MT;
+                for (int kb = itm.kb0; kb < itm.kb1; ++kb, ++it) {
                     if (!ptx::mbar_wait(&empty[stage], phase ^ 1u, abort_flag, wait_ns)) {
                         ok = false;
                         break;
@@ -339,14 +374,16 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             uint32_t use[2] = {0u, 0u};
             bool ok = true;
             int kl = 0;
-            for (int u = cid; u < n_units && ok; u += ncl, ++kl) {
+            for (int u = cid; u < n_items && ok; u += ncl, ++kl) {
                 const int g0 = (MT == 2) ? 0 : (kl & 1);
+                const Item itm = item_of(u);
+                const int nk_u = itm.kb1 - itm.kb0;
                 for (int j = 0; j < MT && ok; ++j)
                     ok = kPair ? ptx::mbar_wait_cluster(&tempty[g0 + j], (use[g0 + j] & 1u) ^ 1u, abort_flag, wait_ns)
                                : ptx::mbar_wait(&tempty[g0 + j], (use[g0 + j] & 1u) ^ 1u, abort_flag, wait_ns);
                 if (!ok) break;
                 ptx::tc_fence_after();
-                for (int kb = 0; kb < nk; ++kb) {     // position inside the unit's K range
+                for (int kb = 0; kb < nk_u; ++kb) {   // position inside the item's K range
                     const bool landed = kPair ? ptx::mbar_wait_cluster(&full[stage], phase, abort_flag, wait_ns)
                                               : ptx::mbar_wait(&full[stage], phase, abort_flag, wait_ns);
                     if (!landed) {
@@ -422,7 +459,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 ptx::mbar_arrive(&tempty[slot]);
             }
         };
-        for (int u = cid; u < n_units; u += ncl, ++kl) {
+        for (int u = cid; u < n_items; u += ncl, ++kl) {
             if (MT == 1 && (kl & 1) != g) continue;
             if (!ptx::mbar_wait(&tfull[g], use & 1u, abort_flag, wait_ns)) {
                 *abort_flag = 1;
@@ -431,12 +468,91 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             }
             ++use;
             ptx::tc_fence_after();
-            const Unit w = unit_of(u);
+            const Item itm = item_of(u);
+            const Unit w = itm.w;
             const int nt = w.nt;
             const int row = ((w.mg * m_cl + m_rank) * MT + (MT == 2 ? g : 0)) * kBM + q * 32 + lane;
             const uint32_t tb = tmem_base + 256u * g + (static_cast<uint32_t>(q * 32) << 16);
 
-            if constexpr (kSplitK) {
+            if (kTail && itm.chunk >= 0) {
+                // ---- a K-chunk of a tail unit: its partial sums to `partial`; the group whose
+                // chunk completes the unit's count adds all chunks in chunk order
+                const int j = MT == 2 ? g : 0;                 // M-tile of the unit in this slot
+                const int r = q * 32 + lane;                   // row within the M-tile
+                constexpr int kUnitF4 = kBM * NB * BN / 4;     // float4s of one (chunk, M-tile)
+                float4* part = reinterpret_cast<float4*>(ep.partial);
+                auto at = [&](int ch, int col) {               // float4 of columns col..col+3, row r
+                    return (static_cast<size_t>((itm.tail * n_split + ch) * MT + j) * kUnitF4) +
+                           static_cast<size_t>(col >> 2) * kBM + r;
+                };
+#pragma unroll 1
+                for (int nb = 0; nb < NB; ++nb) {
+#pragma unroll 1
+                    for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 32) {
+                        uint32_t ra[32];
+                        ptx::tmem_ld_32cols(tb + nb * BN + c, ra);
+#pragma unroll
+                        for (int f = 0; f < 8; ++f)
+                            part[at(itm.chunk, nb * BN + c + 4 * f)] =
+                                make_float4(__uint_as_float(ra[4 * f]), __uint_as_float(ra[4 * f + 1]),
+                                            __uint_as_float(ra[4 * f + 2]), __uint_as_float(ra[4 * f + 3]));
+                    }
+                }
+                release_slot(g);
+                __threadfence();                                // this thread's partial sums, device-wide
+                ptx::named_barrier_sync(1 + g, 32 * kEpiWarps / 2);
+                if (e % (kEpiWarps / 2) == 0 && lane == 0) {
+                    __threadfence();
+                    const int done = atomicAdd(ep.sem + itm.tail * MT + j, 1);
+                    last_chunk[g] = done == n_split - 1 ? 1 : 0;
+                }
+                ptx::named_barrier_sync(1 + g, 32 * kEpiWarps / 2);
+                if (last_chunk[g]) {
+                    __threadfence();                            // every chunk's partial sums
+                    // 8 output columns at a time: this warp's half of the tile
+#pragma unroll 1
+                    for (int c = half * (BN / 2); c < (half + 1) * (BN / 2); c += 8) {
+                        float a0[8], a1[8];
+#pragma unroll
+                        for (int t = 0; t < 8; ++t) a0[t] = a1[t] = 0.0f;
+#pragma unroll 1
+                        for (int ch = 0; ch < n_split; ++ch) {
+                            const float4 p0 = part[at(ch, c)], p1 = part[at(ch, c + 4)];
+                            a0[0] += p0.x; a0[1] += p0.y; a0[2] += p0.z; a0[3] += p0.w;
+                            a0[4] += p1.x; a0[5] += p1.y; a0[6] += p1.z; a0[7] += p1.w;
+                            if constexpr (NB == 2) {
+                                const float4 u0 = part[at(ch, BN + c)], u1 = part[at(ch, BN + c + 4)];
+                                a1[0] += u0.x; a1[1] += u0.y; a1[2] += u0.z; a1[3] += u0.w;
+                                a1[4] += u1.x; a1[5] += u1.y; a1[6] += u1.z; a1[7] += u1.w;
+                            }
+                        }
+                        if (row < n_rows) {
+                            uint32_t o[4];
+                            if constexpr (EPI == EPI_GATEUP) {
+#pragma unroll
+                                for (int t = 0; t < 4; ++t)
+                                    o[t] = pack_bf16x2(silu_f(a0[2 * t]) * a1[2 * t], silu_f(a0[2 * t + 1]) * a1[2 * t + 1]);
+                            } else {
+                                const int sq = row / ep.R, rr = row - sq * ep.R;
+                                const int hid_row = sq * ep.gamma + stage2_hidden_index(rr, ep.M);
+                                const uint4 hv = *reinterpret_cast<const uint4*>(
+                                    ep.hidden + static_cast<size_t>(hid_row) * ep.ld_out + nt * BN + c);
+                                const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w};
+#pragma unroll
+                                for (int t = 0; t < 4; ++t) {
+                                    const __nv_bfloat162 h2 = *reinterpret_cast<const __nv_bfloat162*>(&hw[t]);
+                                    o[t] = pack_bf16x2(__bfloat162float(h2.x) + a0[2 * t], __bfloat162float(h2.y) + a0[2 * t + 1]);
+                                }
+                            }
+                            *reinterpret_cast<uint4*>(ep.out + static_cast<size_t>(row) * ep.ld_out + nt * BN + c) =
+                                make_uint4(o[0], o[1], o[2], o[3]);
+                        }
+                    }
+                    // the count starts from zero for the next call
+                    ptx::named_barrier_sync(1 + g, 32 * kEpiWarps / 2);
+                    if (e % (kEpiWarps / 2) == 0 && lane == 0) ep.sem[itm.tail * MT + j] = 0;
+                }
+            } else if constexpr (kSplitK) {
                 // the accumulators are summed across the cluster below, once every CTA has them
             } else if constexpr (EPI == EPI_LMHEAD) {
                 static_assert(BN == kBlockV, "one LM-head N tile is one vocabulary block");
@@ -753,7 +869,8 @@ int resident_clusters(K kern, int smem, int cl, int num_sms) {
 
 template <int EPI, int MT, int NB, int BN, int STAGES, int CL = 1>
 cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& tw0, const CUtensorMap& tw1,
-                     int n_rows, int K, int n_ntiles, int n_mgroups, const EpiParams& ep_in, int k_splits = 1) {
+                     int n_rows, int K, int n_ntiles, int n_mgroups, const EpiParams& ep_in, int k_splits = 1,
+                     size_t partial_bytes = 0) {
     using C = TileCfg<MT, NB, BN, STAGES, (CL == 2 && EPI != EPI_CGATEUP && EPI != EPI_CDOWN)>;
     auto kern = tc_gemm_kernel<EPI, MT, NB, BN, STAGES, CL>;
     EpiParams ep = ep_in;
@@ -768,7 +885,25 @@ cudaError_t run_gemm(const Ctx& ctx, const CUtensorMap& tx, const CUtensorMap& t
         e = launch_pdl_cluster(kern, dim3(CL * n_ntiles * n_mgroups), dim3(kThreads), C::kSmemBytes, ctx.stream, CL,
                                tx, tw0, tw1, n_rows, K, n_ntiles, n_mgroups, CL, stream_once, ep, ctx.status);
     } else if constexpr (CL == 1) {
-        const int grid = n_units < ctx.num_sms ? n_units : ctx.num_sms;
+        int n_items = n_units;
+        if constexpr (EPI == EPI_GATEUP || EPI == EPI_DOWN) {
+            // Tail split: when the units overflow the SMs by a last round that would leave most of
+            // them idle, each unit of that round runs as up to kMaxTailSplit K-chunks on the idle
+            // SMs, summed by the chunk that finishes last (fp32 partial sums in the workspace).
+            const int tail = n_units % ctx.num_sms;
+            int split = tail > 0 ? ctx.num_sms / tail : 0;
+            split = split < kMaxTailSplit ? split : kMaxTailSplit;
+            split = split < K / kBK ? split : K / kBK;
+            const size_t need = static_cast<size_t>(tail) * split * MT * kBM * NB * BN * sizeof(float);
+            if (k_splits == 1 && n_units > ctx.num_sms && split >= 2 && ctx.status && tail * MT <= kTailSems &&
+                ep.partial && need <= partial_bytes) {
+                ep.n_full = n_units - tail;
+                ep.tail_split = split;
+                ep.sem = ctx.status + 1;
+                n_items = ep.n_full + tail * split;
+            }
+        }
+        const int grid = n_items < ctx.num_sms ? n_items : ctx.num_sms;
         e = launch_pdl(kern, dim3(grid), dim3(kThreads), C::kSmemBytes, ctx.stream, tx, tw0, tw1, n_rows, K,
                        n_ntiles, n_mgroups, k_splits, stream_once, ep, ctx.status);
     } else {
@@ -861,7 +996,8 @@ int choose_k_splits(int base_units, int nk, int num_sms) {
 // the linear approximator (K = 2d, In = x). The residual row of stage-2 row r is the hidden state
 // of its depth; the epilogue adds it in fp32 and rounds once to bf16.
 static cudaError_t run_residual_gemm(const Ctx& ctx, const CUtensorMap& ta, const CUtensorMap& td, int K, const void* hidden,
-                              int n_rows, int d, int R, int M, int gamma, void* h_prime, float* partial) {
+                              int n_rows, int d, int R, int M, int gamma, void* h_prime, float* partial,
+                              size_t partial_bytes) {
     constexpr int BN = 128;
     const int m_tiles = (n_rows + kBM - 1) / kBM;
     const int n_mg = m_tiles == 1 ? 1 : (m_tiles + 1) / 2;
@@ -879,10 +1015,10 @@ static cudaError_t run_residual_gemm(const Ctx& ctx, const CUtensorMap& ta, cons
     ed.n_total = d;
     if (ks2 == 1) {
         if (bn_d == BN)
-            return m_tiles == 1 ? run_gemm<EPI_DOWN, 1, 1, BN, 6>(ctx, ta, td, td, n_rows, K, d / BN, 1, ed)
-                                : run_gemm<EPI_DOWN, 2, 1, BN, 4>(ctx, ta, td, td, n_rows, K, d / BN, n_mg, ed);
-        return m_tiles == 1 ? run_gemm<EPI_DOWN, 1, 1, 64, 8>(ctx, ta, td, td, n_rows, K, d / 64, 1, ed)
-                            : run_gemm<EPI_DOWN, 2, 1, 64, 5>(ctx, ta, td, td, n_rows, K, d / 64, n_mg, ed);
+            return m_tiles == 1 ? run_gemm<EPI_DOWN, 1, 1, BN, 6>(ctx, ta, td, td, n_rows, K, d / BN, 1, ed, 1, partial_bytes)
+                                : run_gemm<EPI_DOWN, 2, 1, BN, 4>(ctx, ta, td, td, n_rows, K, d / BN, n_mg, ed, 1, partial_bytes);
+        return m_tiles == 1 ? run_gemm<EPI_DOWN, 1, 1, 64, 8>(ctx, ta, td, td, n_rows, K, d / 64, 1, ed, 1, partial_bytes)
+                            : run_gemm<EPI_DOWN, 2, 1, 64, 5>(ctx, ta, td, td, n_rows, K, d / 64, n_mg, ed, 1, partial_bytes);
     }
     if (m_tiles == 2 && bn_d == BN && ks2 == 4 && splitk_clusters_fit<EPI_CDOWN, 2, 1, BN, 4, 4>(ctx, d / BN))
         return run_gemm<EPI_CDOWN, 2, 1, BN, 4, 4>(ctx, ta, td, td, n_rows, K, d / BN, 1, ed, 4);
@@ -900,7 +1036,7 @@ static cudaError_t run_residual_gemm(const Ctx& ctx, const CUtensorMap& ta, cons
 
 cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, int k_in, const void* w_gate, const void* w_up,
                              const void* w_down, const void* hidden, int n_rows, int d, int I, int R, int M,
-                             int gamma, void* A, void* h_prime, float* partial) {
+                             int gamma, void* A, void* h_prime, float* partial, size_t partial_bytes) {
     if (n_rows <= 0) return cudaSuccess;
     constexpr int BN = 128;
     const int m_tiles = (n_rows + kBM - 1) / kBM;
@@ -925,11 +1061,11 @@ cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, int k_in, const void
     ep.n_total = I;
     if (ks1 == 1) {
         if (bn_gu == BN)
-            e = m_tiles == 1 ? run_gemm<EPI_GATEUP, 1, 2, BN, 4>(ctx, tx, tg, tu, n_rows, k_in, I / BN, 1, ep)
-                             : run_gemm<EPI_GATEUP, 2, 2, BN, 3>(ctx, tx, tg, tu, n_rows, k_in, I / BN, n_mg, ep);
+            e = m_tiles == 1 ? run_gemm<EPI_GATEUP, 1, 2, BN, 4>(ctx, tx, tg, tu, n_rows, k_in, I / BN, 1, ep, 1, partial_bytes)
+                             : run_gemm<EPI_GATEUP, 2, 2, BN, 3>(ctx, tx, tg, tu, n_rows, k_in, I / BN, n_mg, ep, 1, partial_bytes);
         else
-            e = m_tiles == 1 ? run_gemm<EPI_GATEUP, 1, 2, 64, 6>(ctx, tx, tg, tu, n_rows, k_in, I / 64, 1, ep)
-                             : run_gemm<EPI_GATEUP, 2, 2, 64, 4>(ctx, tx, tg, tu, n_rows, k_in, I / 64, n_mg, ep);
+            e = m_tiles == 1 ? run_gemm<EPI_GATEUP, 1, 2, 64, 6>(ctx, tx, tg, tu, n_rows, k_in, I / 64, 1, ep, 1, partial_bytes)
+                             : run_gemm<EPI_GATEUP, 2, 2, 64, 4>(ctx, tx, tg, tu, n_rows, k_in, I / 64, n_mg, ep, 1, partial_bytes);
         if (e != cudaSuccess) return e;
     } else if (m_tiles == 2 && bn_gu == BN && ks1 == 4 &&
                splitk_clusters_fit<EPI_CGATEUP, 2, 2, BN, 3, 4>(ctx, I / BN)) {
@@ -948,18 +1084,18 @@ cudaError_t launch_swiglu_tc(const Ctx& ctx, const void* X, int k_in, const void
     }
 
     // ---- down + residual: h' = h + A Wd^T
-    return run_residual_gemm(ctx, ta, td, I, hidden, n_rows, d, R, M, gamma, h_prime, partial);
+    return run_residual_gemm(ctx, ta, td, I, hidden, n_rows, d, R, M, gamma, h_prime, partial, partial_bytes);
 }
 
 cudaError_t launch_linear_tc(const Ctx& ctx, const void* X, const void* w_lin, const void* hidden, int n_rows, int d,
-                             int R, int M, int gamma, void* h_prime, float* partial) {
+                             int R, int M, int gamma, void* h_prime, float* partial, size_t partial_bytes) {
     if (n_rows <= 0) return cudaSuccess;
     const int bn = d % 128 == 0 ? 128 : 64;
     CUtensorMap tx, tw;
     cudaError_t e = make_tmap(&tx, X, 2 * d, n_rows, kBK, kBM);
     if (e == cudaSuccess) e = make_tmap(&tw, w_lin, 2 * d, d, kBK, bn);
     if (e != cudaSuccess) return e;
-    return run_residual_gemm(ctx, tx, tw, 2 * d, hidden, n_rows, d, R, M, gamma, h_prime, partial);
+    return run_residual_gemm(ctx, tx, tw, 2 * d, hidden, n_rows, d, R, M, gamma, h_prime, partial, partial_bytes);
 }
 
 }  // namespace tf

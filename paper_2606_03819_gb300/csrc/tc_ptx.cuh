@@ -237,6 +237,11 @@ __device__ __forceinline__ uint32_t cluster_count_x() {
     return r;
 }
 // Every thread of every CTA of the cluster arrives, then waits for all others (release/acquire).
+// Barrier `id` (1..15) of `nthreads` threads of this CTA (a multiple of 32).
+__device__ __forceinline__ void named_barrier_sync(int id, int nthreads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
 __device__ __forceinline__ void cluster_sync() {
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }

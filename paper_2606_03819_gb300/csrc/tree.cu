@@ -61,6 +61,9 @@ __global__ void __launch_bounds__(256) gather_norm_kernel(const T* __restrict__ 
                                                           T* __restrict__ hres, int* status) {
     pdl_trigger();
     pdl_wait();
+    // the approximator GEMMs' tail-split counters (after the status word) start each call at zero
+    if (blockIdx.x == 0 && status)
+        for (int i = threadIdx.x; i < kTailSems; i += blockDim.x) status[1 + i] = 0;
     __shared__ float red[1 + NE][8];
     const int row = blockIdx.x;
     const int hid = stage2_row_hidden(row, R, gamma, M, NE == 2);
@@ -987,6 +990,9 @@ __global__ void __launch_bounds__(256) gather_norm_bf16x8_kernel(
         }
     }
     pdl_wait();
+    // the approximator GEMMs' tail-split counters (after the status word) start each call at zero
+    if (blockIdx.x == 0 && status)
+        for (int i = threadIdx.x; i < kTailSems; i += blockDim.x) status[1 + i] = 0;
     int tok[2] = {0, 0};
     stage2_row_tokens(row, R, gamma, M, K1, NE == 2, root_tok, top_ids, tok);
 #pragma unroll

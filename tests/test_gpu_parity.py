@@ -116,6 +116,32 @@ def test_bf16_two_m_tiles_cluster_split_k():
     check(cfg)
 
 
+def test_bf16_tail_split_of_the_last_round():
+    # 150 sequences x 13 rows = 1950 stage-2 rows (8 pairs of M-tiles) with d = I = 2560: on 152
+    # SMs both approximator GEMMs have 20 x 8 = 160 work units, so the 8 units of the last round
+    # run as 8 K-chunks each, added by the chunk that finishes last. Every stage is checked on
+    # every row, the tree end to end on three sequences, and a second call on the same workspace
+    # (its counters reset by the first) gives the same bits.
+    from paper_2606_03819_gb300 import Dims, Drafter
+    cfg = synth.get_config("tiny_peaked", dtype="bf16", batch=150, d=2560, I=2560, V=2000, wd_std=0.05)
+    inp = synth.make_inputs(cfg)
+    dinp = parity.device_inputs(inp)
+    dr = Drafter(Dims.from_config(cfg), dinp)
+    gpu = parity.run_gpu(cfg, dinp, drafter=dr)
+    assert not (gpu["flags"] & ~16), f"device flags {gpu['flags']}"
+    W = parity.oracle_weights(inp)
+    parity.check_bf16_stagewise(cfg, inp, W, gpu)
+    seqs = [0, 77, 149]
+    sub = {k: (v[seqs] if isinstance(v, np.ndarray) and v.ndim >= 1 and v.shape[0] == cfg.batch else v)
+           for k, v in gpu.items()}
+    orc = parity.run_oracle(cfg, inp, seqs=seqs, W=W)
+    orc_e = parity.run_oracle(cfg, inp, emulate_bf16=True, seqs=seqs, W=W)
+    parity.check_bf16_end_to_end(cfg, sub, orc, orc_e)
+    again = parity.run_gpu(cfg, dinp, drafter=dr)
+    for k in ("A", "hp", "child_ids", "child_logp", "node_tok", "node_parent", "mask"):
+        np.testing.assert_array_equal(gpu[k], again[k], err_msg=k)
+
+
 @pytest.mark.parametrize("mode", ["marginal", "marginal_mary"])
 def test_bf16_marginal_modes(mode):
     check(synth.get_config("tiny_peaked", dtype="bf16", batch=3, V=2000, mode=mode))
