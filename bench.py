@@ -12,7 +12,8 @@ fused LM-head pass): algorithmic bytes per launch (|W_lm| + the activation rows)
 CUDA-event duration, from a second pass of the same steps with events around the two LM-head
 launches. `gpu_launches` is the library's own count of kernels launched in the timed region. `e2e` is the same metric
 through tf_draft_tree_host with the step's inputs and outputs in pinned host memory, copies
-inside the timed region. `cpu_baseline` is the fp64 oracle on the host cores on a bounded sample.
+inside the timed region, on a created stream (the library then replays the step as a CUDA graph
+captured at the first call). `cpu_baseline` is the fp64 oracle on the host cores on a bounded sample.
 `torch_eager` times the same step written with PyTorch library calls (logits materialised,
 Part 2 as a host loop, as in the paper's implementation): a reference point, not a competitor.
 
@@ -559,10 +560,12 @@ def run_gpu(args):
                     dev_status=torch.empty(cfg.batch, dtype=torch.int32))
         outs = {k: pin(v) for k, v in outs.items()}
 
+        e2e_stream = torch.cuda.Stream(dev)
+
         def host_step():
             return Bn.tf_draft_tree_host(dims, d, h_hidden, h_root, h_pos, outs["node_tok"], outs["node_parent"],
                                          outs["node_depth"], outs["node_score"], outs["mask"], outs["pos_ids"],
-                                         outs["dev_status"], dr.ws)
+                                         outs["dev_status"], dr.ws, stream=e2e_stream)
         for _ in range(3):
             host_step()
         barrier(world, dev)

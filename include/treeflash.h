@@ -233,10 +233,19 @@ tf_status tf_build_tree_mask(const tf_dims* dims, const int32_t* root_tok, const
                              float* node_score, uint8_t* mask, int32_t* pos_ids,
                              int32_t* dev_status, tf_stream_t stream);
 
-/* The whole drafting step for callers holding the step's inputs in HOST memory (pinned memory
- * makes the copies asynchronous): copies hidden/root_tok/root_pos to the device, runs stage 1,
- * stage 2 (TF_MODE_AR) and tf_build_tree_mask, copies the tree, mask and status back, and
- * synchronises `stream`.
+/* The whole drafting step for callers holding the step's inputs in HOST memory: copies hidden to
+ * the device, runs stage 1, stage 2 (TF_MODE_AR) and tf_build_tree_mask, brings the tree, mask
+ * and status back, and synchronises `stream`.
+ * With page-locked host buffers (cudaHostAlloc, or torch's pin_memory) that the device can
+ * address, the kernels read root_tok and root_pos and write every output in host memory
+ * directly; other buffers go through the workspace and copies. On a created stream (not the
+ * legacy default stream) with page-locked buffers, the first call with a given set of arguments
+ * (dims, weight, buffer and workspace pointers, device, wait limit) captures the step as a CUDA
+ * graph and later calls replay it: the buffers' contents may change between calls, their
+ * addresses may not without a new capture. The library keeps the last 8 such graphs (the CUDA
+ * driver instantiates them; the library itself allocates no memory); a capture that fails leaves
+ * the step on plain launches. The call must not itself be made inside a stream capture (it
+ * synchronises).
  * Host inputs: hidden [b, gamma, d] dtype, root_tok [b] ([b, 2] with TF_APPROX_SWIGLU_2PREV),
  * root_pos [b]. Host outputs:
  * node_tok, node_parent, node_depth [b, B+1] int32, node_score [b, B+1] float,

@@ -1,11 +1,14 @@
 // C ABI of the TreeFlash drafting path (declared in include/treeflash.h): argument checks,
 // workspace layout and the kernel sequence of every call. No allocation; the only global state
-// is the cached driver entry point used to build TMA descriptors and a launch counter.
+// is the cached driver entry point used to build TMA descriptors, a launch counter and the CUDA
+// graphs of the host-buffer step (tf_draft_tree_host).
 #include <math.h>
 #include <string.h>
 
 #include <algorithm>
 #include <atomic>
+#include <mutex>
+#include <vector>
 
 #include "common.cuh"
 
@@ -256,6 +259,213 @@ tf_status prepare(const tf_dims* dims, void* ws, size_t ws_bytes, tf_stream_t st
     return make_ctx(ws, p->L, stream, &p->ctx);
 }
 
+// ---- the host-buffer step ---------------------------------------------------------------------
+struct HostStep {
+    const tf_dims* dims;
+    const tf_weights* w;
+    const void* hidden;
+    const int32_t* root_tok;
+    const int32_t* root_pos;
+    int32_t *node_tok, *node_parent, *node_depth;
+    float* node_score;
+    uint8_t* mask;
+    int32_t *pos_ids, *dev_status;
+    void* ws;
+    size_t ws_bytes;
+    tf_stream_t stream;
+};
+
+// Device-visible addresses of page-locked host buffers (the same memory), or all null.
+struct Mapped {
+    const int32_t *root_tok, *root_pos;
+    int32_t *node_tok, *node_parent, *node_depth;
+    float* node_score;
+    uint8_t* mask;
+    int32_t *pos_ids, *dev_status;
+    bool ok;
+};
+
+// The address under which the device reaches page-locked host memory `ptr`, or null.
+void* device_view(const void* ptr) {
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, ptr) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return nullptr;
+    }
+    return a.type == cudaMemoryTypeHost ? a.devicePointer : nullptr;
+}
+
+Mapped map_host_buffers(const HostStep& h) {
+    Mapped m{};
+    m.root_tok = static_cast<const int32_t*>(device_view(h.root_tok));
+    m.root_pos = static_cast<const int32_t*>(device_view(h.root_pos));
+    m.node_tok = static_cast<int32_t*>(device_view(h.node_tok));
+    m.node_parent = static_cast<int32_t*>(device_view(h.node_parent));
+    m.node_depth = static_cast<int32_t*>(device_view(h.node_depth));
+    m.node_score = static_cast<float*>(device_view(h.node_score));
+    m.mask = static_cast<uint8_t*>(device_view(h.mask));
+    m.pos_ids = static_cast<int32_t*>(device_view(h.pos_ids));
+    m.dev_status = static_cast<int32_t*>(device_view(h.dev_status));
+    m.ok = m.root_tok && m.root_pos && m.node_tok && m.node_parent && m.node_depth && m.node_score && m.mask &&
+           m.pos_ids && m.dev_status;
+    return m;
+}
+
+// Enqueues the whole host-buffer step on the stream, without synchronising: the hidden states to
+// the workspace, stage 1, stage 2, the tree and its mask (dev_status with the workspace status
+// word folded in by the builder, so no separate read is needed). With page-locked buffers that
+// the device can address (m.ok) the kernels read root_tok / root_pos and write the outputs in
+// host memory directly; otherwise those go through the workspace and copies.
+tf_status enqueue_host_step(const Prepared& p, const HostStep& h, const Mapped& m) {
+    const Dims& D = p.D;
+    const Layout& L = p.L;
+    const Ctx& ctx = p.ctx;
+    cudaStream_t st = ctx.stream;
+    void* ws = h.ws;
+    const size_t nn = static_cast<size_t>(D.b) * (D.B + 1);
+    void* d_hidden = at<void>(ws, L.h_hidden);
+    TF_TRY(cuda_status(cudaMemcpyAsync(d_hidden, h.hidden, static_cast<size_t>(D.b) * D.gamma * D.d * D.esize,
+                                       cudaMemcpyHostToDevice, st)));
+    const int32_t* d_root = m.root_tok;
+    const int32_t* d_pos = m.root_pos;
+    if (!m.ok) {
+        int32_t* r = at<int32_t>(ws, L.h_root);
+        int32_t* q = at<int32_t>(ws, L.h_pos);
+        TF_TRY(cuda_status(cudaMemcpyAsync(r, h.root_tok, static_cast<size_t>(D.b) * D.root_stride * sizeof(int32_t),
+                                           cudaMemcpyHostToDevice, st)));
+        TF_TRY(cuda_status(cudaMemcpyAsync(q, h.root_pos, D.b * sizeof(int32_t), cudaMemcpyHostToDevice, st)));
+        d_root = r;
+        d_pos = q;
+    }
+    int32_t* top_ids = at<int32_t>(ws, L.top_ids);
+    float* top_logp = at<float>(ws, L.top_logp);
+    int32_t* child_ids = at<int32_t>(ws, L.child_ids);
+    float* child_logp = at<float>(ws, L.child_logp);
+    TF_TRY(tf_stage1_marginals(h.dims, h.w, d_hidden, top_ids, top_logp, ws, h.ws_bytes, h.stream));
+    if (D.mode == TF_MODE_AR)
+        TF_TRY(tf_stage2_ar_approx(h.dims, h.w, d_hidden, d_root, top_ids, child_ids, child_logp, ws, h.ws_bytes,
+                                   h.stream));
+    int32_t* o_tok = m.ok ? m.node_tok : at<int32_t>(ws, L.n_tok);
+    int32_t* o_par = m.ok ? m.node_parent : at<int32_t>(ws, L.n_par);
+    int32_t* o_dep = m.ok ? m.node_depth : at<int32_t>(ws, L.n_dep);
+    float* o_score = m.ok ? m.node_score : at<float>(ws, L.n_score);
+    uint8_t* o_mask = m.ok ? m.mask : at<uint8_t>(ws, L.n_mask);
+    int32_t* o_pos = m.ok ? m.pos_ids : at<int32_t>(ws, L.n_pos);
+    int32_t* o_stat = m.ok ? m.dev_status : at<int32_t>(ws, L.n_stat);
+    const bool ar = D.mode == TF_MODE_AR;
+    const bool fused = D.B + 1 <= kFusedMaskMaxNodes;   // the builder CTA writes the mask of its tree
+    TF_TRY(cuda_status(launch_build_tree(ctx, D.b, D.gamma, D.M, D.K1, D.K2, D.B, D.V, D.mode, D.R, D.two_prev, d_root,
+                                         top_ids, top_logp, ar ? child_ids : nullptr, ar ? child_logp : nullptr, o_tok,
+                                         o_par, o_dep, o_score, o_stat, fused ? d_pos : nullptr, fused ? o_mask : nullptr,
+                                         fused ? o_pos : nullptr, ctx.status)));
+    if (!fused) TF_TRY(cuda_status(launch_tree_mask(ctx, D.b, D.B, o_par, o_dep, d_pos, o_mask, o_pos)));
+    if (m.ok) return TF_OK;
+    TF_TRY(cuda_status(cudaMemcpyAsync(h.node_tok, o_tok, nn * 4, cudaMemcpyDeviceToHost, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(h.node_parent, o_par, nn * 4, cudaMemcpyDeviceToHost, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(h.node_depth, o_dep, nn * 4, cudaMemcpyDeviceToHost, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(h.node_score, o_score, nn * 4, cudaMemcpyDeviceToHost, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(h.mask, o_mask, nn * (D.B + 1), cudaMemcpyDeviceToHost, st)));
+    TF_TRY(cuda_status(cudaMemcpyAsync(h.pos_ids, o_pos, nn * 4, cudaMemcpyDeviceToHost, st)));
+    return cuda_status(cudaMemcpyAsync(h.dev_status, o_stat, D.b * 4, cudaMemcpyDeviceToHost, st));
+}
+
+// The host-buffer step as a CUDA graph, captured on the first call with a given set of arguments
+// and replayed afterwards: one graph launch in place of three copies, eight to nine kernel launches
+// and seven copies, and the next step's first kernel no longer waits for the host to issue it.
+// Only for a created stream (the legacy default stream cannot be captured) and page-locked host
+// buffers (copies from pageable memory cannot be captured); otherwise, or when the capture or the
+// instantiation fails, the step runs as plain launches. The key holds everything the captured
+// kernels and copies read at capture time: dims, weight, buffer and workspace pointers, the device
+// and the wait limit of the tensor-core kernels. At most kMaxHostGraphs are kept (oldest evicted).
+struct HostGraph {
+    std::vector<uint64_t> key;
+    cudaGraphExec_t exec;       // nullptr: this step could not be captured, run it as plain launches
+    unsigned long long kernels; // kernel launches in the graph (for the library's launch counter)
+};
+std::mutex g_host_graph_mu;
+std::vector<HostGraph> g_host_graphs;
+constexpr size_t kMaxHostGraphs = 8;
+
+uint32_t float_bits(float f) {
+    uint32_t u;
+    memcpy(&u, &f, sizeof(u));
+    return u;
+}
+
+bool page_locked(const void* ptr) {
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, ptr) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return false;
+    }
+    return a.type == cudaMemoryTypeHost;
+}
+
+tf_status launch_host_graph(const Prepared& p, const HostStep& h, const Mapped& m, bool* replayed) {
+    *replayed = false;
+    cudaStream_t st = p.ctx.stream;
+    if (st == nullptr || st == cudaStreamLegacy || st == cudaStreamPerThread) return TF_OK;
+    cudaStreamCaptureStatus cs;
+    if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return TF_OK;
+    }
+    if (cs != cudaStreamCaptureStatusNone) return TF_OK;
+    const void* host_ptrs[] = {h.hidden, h.root_tok, h.root_pos, h.node_tok, h.node_parent, h.node_depth,
+                               h.node_score, h.mask, h.pos_ids, h.dev_status};
+    for (const void* q : host_ptrs)
+        if (!page_locked(q)) return TF_OK;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return TF_ERR_CUDA;
+    const tf_dims& d = *h.dims;
+    std::vector<uint64_t> key = {
+        static_cast<uint64_t>(d.batch), static_cast<uint64_t>(d.d), static_cast<uint64_t>(d.V), static_cast<uint64_t>(d.I),
+        static_cast<uint64_t>(d.gamma), static_cast<uint64_t>(d.M), static_cast<uint64_t>(d.K2), static_cast<uint64_t>(d.B),
+        static_cast<uint64_t>(float_bits(d.temperature)), static_cast<uint64_t>(float_bits(d.rms_eps)),
+        static_cast<uint64_t>(d.dtype), static_cast<uint64_t>(d.mode), static_cast<uint64_t>(d.approx),
+        static_cast<uint64_t>(dev), wait_limit_ns(), reinterpret_cast<uint64_t>(h.ws), static_cast<uint64_t>(h.ws_bytes)};
+    const void* w_ptrs[] = {h.w->lm_head, h.w->embed, h.w->norm_h, h.w->norm_e, h.w->w_gate, h.w->w_up, h.w->w_down,
+                            h.w->w_lin};
+    for (const void* q : w_ptrs) key.push_back(reinterpret_cast<uint64_t>(q));
+    for (const void* q : host_ptrs) key.push_back(reinterpret_cast<uint64_t>(q));
+
+    std::lock_guard<std::mutex> lock(g_host_graph_mu);
+    HostGraph* hit = nullptr;
+    for (auto& g : g_host_graphs)
+        if (g.key == key) hit = &g;
+    if (!hit) {
+        if (cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+            (void)cudaGetLastError();
+            return TF_OK;
+        }
+        // captured launches run only with the graph: they are counted at each replay instead
+        const unsigned long long c0 = tf::g_kernel_launches.load(std::memory_order_relaxed);
+        const tf_status es = enqueue_host_step(p, h, m);
+        const unsigned long long kernels = tf::g_kernel_launches.load(std::memory_order_relaxed) - c0;
+        tf::g_kernel_launches.fetch_sub(kernels, std::memory_order_relaxed);
+        cudaGraph_t graph = nullptr;
+        const cudaError_t ce = cudaStreamEndCapture(st, &graph);
+        cudaGraphExec_t exec = nullptr;
+        if (es == TF_OK && ce == cudaSuccess && graph &&
+            cudaGraphInstantiate(&exec, graph, 0) != cudaSuccess)
+            exec = nullptr;
+        if (graph) cudaGraphDestroy(graph);
+        (void)cudaGetLastError();
+        if (es != TF_OK && es != TF_ERR_CUDA) return es;   // an argument error: nothing to cache
+        if (g_host_graphs.size() >= kMaxHostGraphs) {
+            if (g_host_graphs.front().exec) cudaGraphExecDestroy(g_host_graphs.front().exec);
+            g_host_graphs.erase(g_host_graphs.begin());
+        }
+        g_host_graphs.push_back(HostGraph{key, exec, kernels});
+        hit = &g_host_graphs.back();
+    }
+    if (!hit->exec) return TF_OK;
+    if (cudaGraphLaunch(hit->exec, st) != cudaSuccess) return TF_ERR_CUDA;
+    tf::g_kernel_launches.fetch_add(hit->kernels, std::memory_order_relaxed);
+    *replayed = true;
+    return TF_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -480,47 +690,20 @@ tf_status tf_draft_tree_host(const tf_dims* dims, const tf_weights* w, const voi
     if (!hidden || !root_tok || !root_pos || !node_tok || !node_parent || !node_depth || !node_score || !mask ||
         !pos_ids || !dev_status)
         return TF_ERR_INVALID_ARG;
-    const Dims& D = p.D;
-    const Layout& L = p.L;
+    const HostStep h{dims, w, hidden, root_tok, root_pos, node_tok, node_parent, node_depth, node_score, mask, pos_ids,
+                     dev_status, ws, ws_bytes, stream};
     cudaStream_t st = p.ctx.stream;
-    const size_t nn = static_cast<size_t>(D.b) * (D.B + 1);
-    void* d_hidden = at<void>(ws, L.h_hidden);
-    int32_t* d_root = at<int32_t>(ws, L.h_root);
-    int32_t* d_pos = at<int32_t>(ws, L.h_pos);
-    TF_TRY(cuda_status(cudaMemcpyAsync(d_hidden, hidden, static_cast<size_t>(D.b) * D.gamma * D.d * D.esize,
-                                       cudaMemcpyHostToDevice, st)));
-    TF_TRY(cuda_status(cudaMemcpyAsync(d_root, root_tok, static_cast<size_t>(D.b) * D.root_stride * sizeof(int32_t),
-                                       cudaMemcpyHostToDevice, st)));
-    TF_TRY(cuda_status(cudaMemcpyAsync(d_pos, root_pos, D.b * sizeof(int32_t), cudaMemcpyHostToDevice, st)));
-    int32_t* top_ids = at<int32_t>(ws, L.top_ids);
-    float* top_logp = at<float>(ws, L.top_logp);
-    int32_t* child_ids = at<int32_t>(ws, L.child_ids);
-    float* child_logp = at<float>(ws, L.child_logp);
-    TF_TRY(tf_stage1_marginals(dims, w, d_hidden, top_ids, top_logp, ws, ws_bytes, stream));
-    if (D.mode == TF_MODE_AR)
-        TF_TRY(tf_stage2_ar_approx(dims, w, d_hidden, d_root, top_ids, child_ids, child_logp, ws, ws_bytes, stream));
-    int32_t* d_tok = at<int32_t>(ws, L.n_tok);
-    int32_t* d_par = at<int32_t>(ws, L.n_par);
-    int32_t* d_dep = at<int32_t>(ws, L.n_dep);
-    float* d_score = at<float>(ws, L.n_score);
-    uint8_t* d_mask = at<uint8_t>(ws, L.n_mask);
-    int32_t* d_posid = at<int32_t>(ws, L.n_pos);
-    int32_t* d_stat = at<int32_t>(ws, L.n_stat);
-    TF_TRY(tf_build_tree_mask(dims, d_root, d_pos, top_ids, top_logp, D.mode == TF_MODE_AR ? child_ids : nullptr,
-                              D.mode == TF_MODE_AR ? child_logp : nullptr, d_tok, d_par, d_dep, d_score, d_mask,
-                              d_posid, d_stat, stream));
-    TF_TRY(cuda_status(cudaMemcpyAsync(node_tok, d_tok, nn * 4, cudaMemcpyDeviceToHost, st)));
-    TF_TRY(cuda_status(cudaMemcpyAsync(node_parent, d_par, nn * 4, cudaMemcpyDeviceToHost, st)));
-    TF_TRY(cuda_status(cudaMemcpyAsync(node_depth, d_dep, nn * 4, cudaMemcpyDeviceToHost, st)));
-    TF_TRY(cuda_status(cudaMemcpyAsync(node_score, d_score, nn * 4, cudaMemcpyDeviceToHost, st)));
-    TF_TRY(cuda_status(cudaMemcpyAsync(mask, d_mask, nn * (D.B + 1), cudaMemcpyDeviceToHost, st)));
-    TF_TRY(cuda_status(cudaMemcpyAsync(pos_ids, d_posid, nn * 4, cudaMemcpyDeviceToHost, st)));
-    TF_TRY(cuda_status(cudaMemcpyAsync(dev_status, d_stat, D.b * 4, cudaMemcpyDeviceToHost, st)));
-    int32_t flags = 0;
-    const tf_status rs = tf_status_read(ws, ws_bytes, &flags, stream);  // synchronises the stream
-    if (rs == TF_ERR_CUDA) return rs;
-    for (int s = 0; s < D.b; ++s) dev_status[s] |= flags;
-    return rs;
+    const Mapped m = map_host_buffers(h);
+    bool replayed = false;
+    TF_TRY(launch_host_graph(p, h, m, &replayed));
+    if (!replayed) TF_TRY(enqueue_host_step(p, h, m));
+    if (cudaStreamSynchronize(st) != cudaSuccess) return TF_ERR_CUDA;
+    // every dev_status entry carries the workspace word in bits 16 and up (folded by the builder)
+    const int32_t flags = dev_status[0] >> 16;
+    for (int s = 0; s < p.D.b; ++s) dev_status[s] &= 0xffff;
+    if (flags & TF_DEV_TIMEOUT) return TF_ERR_TIMEOUT;
+    if (flags & ~TF_DEV_RECOMPUTED) return TF_ERR_DEVICE_STATUS;
+    return TF_OK;
 }
 
 }  // extern "C"

@@ -207,7 +207,7 @@ cudaError_t launch_build_tree(const Ctx&, int b, int gamma, int M, int K1, int K
                               const float* child_logp, int32_t* node_tok, int32_t* node_parent,
                               int32_t* node_depth, float* node_score, int32_t* dev_status,
                               const int32_t* root_pos = nullptr, uint8_t* mask = nullptr,
-                              int32_t* pos_ids = nullptr);
+                              int32_t* pos_ids = nullptr, const int32_t* ws_status = nullptr);
 // the largest tree (B + 1 nodes) whose mask launch_build_tree can write from the builder itself
 constexpr int kFusedMaskMaxNodes = 128;
 cudaError_t launch_accept_walk(const Ctx&, int b, int B, int gamma, const int32_t* node_tok,

@@ -147,7 +147,18 @@ struct TreeArgs {
     const int32_t* root_pos;
     uint8_t* mask;
     int32_t* pos_ids;
+    // optional: the workspace status word, final once the builder runs (every earlier kernel of
+    // the step has finished). Each dev_status[s] then becomes seq_bits | w | w << 16 with w that
+    // word, so that a caller that reads dev_status alone also learns w by itself.
+    const int32_t* ws_status;
 };
+
+// The status word of sequence s: its own bits, and with a.ws_status the folded workspace word.
+__device__ __forceinline__ int32_t sequence_status(const TreeArgs& a, int flags) {
+    if (!a.ws_status) return flags;
+    const int32_t w = *a.ws_status;
+    return flags | w | (w << 16);
+}
 
 // Index m of `tok` among the M <= 64 stage-1 candidates of depth `dep` (the M-ary rule of
 // Algorithm 1 Part 2: the node is expandable iff its token is one of them), or -1; two warp
@@ -508,7 +519,7 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_kernel(TreeArgs a, in
             o_dep[i] = -1;
             o_score[i] = -INFINITY;
         }
-        if (lane == 0) a.dev_status[s] = flags;
+        if (lane == 0) a.dev_status[s] = sequence_status(a, flags);
     }
     __syncthreads();
     write_nodes(a, s, t);
@@ -645,7 +656,7 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
             t.o_dep[i] = -1;
             t.o_score[i] = -INFINITY;
         }
-        if (lane == 0) a.dev_status[s] = flags;
+        if (lane == 0) a.dev_status[s] = sequence_status(a, flags);
     }
     __syncthreads();
     write_nodes(a, s, t);
@@ -836,7 +847,7 @@ __global__ void __launch_bounds__(kFastThreads) build_tree_fast_kernel(TreeArgs 
             o_dep[i] = -1;
             o_score[i] = -INFINITY;
         }
-        if (lane == 0) a.dev_status[s] = flags;
+        if (lane == 0) a.dev_status[s] = sequence_status(a, flags);
     }
     __syncthreads();
     for (int i = tid; i < n_out; i += T) {
@@ -1132,11 +1143,11 @@ cudaError_t launch_build_tree(const Ctx& ctx, int b, int gamma, int M, int K1, i
                               int two_prev, const int32_t* root_tok, const int32_t* top_ids, const float* top_logp,
                               const int32_t* child_ids, const float* child_logp, int32_t* node_tok,
                               int32_t* node_parent, int32_t* node_depth, float* node_score, int32_t* dev_status,
-                              const int32_t* root_pos, uint8_t* mask, int32_t* pos_ids) {
+                              const int32_t* root_pos, uint8_t* mask, int32_t* pos_ids, const int32_t* ws_status) {
     if (mask && B + 1 > kFusedMaskMaxNodes) return cudaErrorInvalidValue;
     TreeArgs a{gamma, M, K1, K2, B, V, mode, R, mode == TF_MODE_AR && two_prev ? 1 : 0, root_tok, top_ids, top_logp,
                child_ids, child_logp, node_tok, node_parent, node_depth, node_score, dev_status, root_pos, mask,
-               pos_ids};
+               pos_ids, ws_status};
     const size_t fixed = tree_smem_fixed(B, gamma, M, mask != nullptr);
     const int rows_l = mode == TF_MODE_AR ? R : gamma;
     const int stride = mode == TF_MODE_AR ? K2 : K1;
