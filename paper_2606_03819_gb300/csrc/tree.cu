@@ -754,7 +754,8 @@ __global__ void __launch_bounds__(kFastThreads) build_tree_fast_kernel(TreeArgs 
         topm[i] = a.top_ids[(static_cast<size_t>(s) * a.gamma + i / a.M) * a.K1 + i % a.M];
     __syncthreads();
     // ---- the pops (one warp): lane i holds the i-th best live entry, as its key (score, depth,
-    // parent), its list entry (row << 10 | rank) and its parent's score; key 0 marks an empty lane
+    // parent) and its list entry (row << 10 | rank); key 0 marks an empty lane. The parent's
+    // score, which a sibling's score needs, is read from the placed nodes (o_score[parent]).
     if (tid < 32) {
         const int lane = tid;
         const int list_len = a.K2 < sw ? a.K2 : sw;   // staged ranks; a pop never reaches rank sw
@@ -763,7 +764,6 @@ __global__ void __launch_bounds__(kFastThreads) build_tree_fast_kernel(TreeArgs 
         if (root < 0 || root >= a.V) flags |= TF_DEV_BAD_TOKEN;
         uint32_t khi = 0u, klo = 0u;
         int rr = 0;
-        float psc = 0.0f;
         if (lane == 0) {
             const unsigned long long k0 = queue_key(l_lp[0], 1, 0);
             khi = static_cast<uint32_t>(k0 >> 32);
@@ -775,20 +775,18 @@ __global__ void __launch_bounds__(kFastThreads) build_tree_fast_kernel(TreeArgs 
         }
         int count = 1;    // nodes placed
         while (count < n_out) {
+            __syncwarp();                              // lane 0's node writes, for o_score below
             // the head: lane 0's entry
             const uint32_t hhi = __shfl_sync(kFull, khi, 0);
             if (hhi == 0u) break;                      // queue empty
             const uint32_t hlo = __shfl_sync(kFull, klo, 0);
             const int hrr = __shfl_sync(kFull, rr, 0);
-            const float hpsc = __shfl_sync(kFull, psc, 0);
             // the rest shifted by one: lane i sees entries i + 1 (next) and i - 1 (prev)
             uint32_t nhi = __shfl_down_sync(kFull, khi, 1), nlo = __shfl_down_sync(kFull, klo, 1);
             const int nrr = __shfl_down_sync(kFull, rr, 1);
-            const float npsc = __shfl_down_sync(kFull, psc, 1);
             if (lane == 31) nhi = nlo = 0u;
             const uint32_t phi = __shfl_up_sync(kFull, khi, 1), plo = __shfl_up_sync(kFull, klo, 1);
             const int prr = __shfl_up_sync(kFull, rr, 1);
-            const float ppsc = __shfl_up_sync(kFull, psc, 1);
             // the popped node
             const int row = hrr >> 10, rank = hrr & 1023, idx = row * sw + rank;
             const int dep = 127 - static_cast<int>(hlo >> 24);
@@ -796,15 +794,20 @@ __global__ void __launch_bounds__(kFastThreads) build_tree_fast_kernel(TreeArgs 
             const float sc = key_float(hhi);
             const int node = count++;
             const int tok = l_tok[idx];
+            const float hpsc = o_score[par];           // the parent's score
             // its children: none at the depth cap; DDTree: the next depth's marginal row;
             // otherwise only for a stage-1 candidate m of its depth (Algorithm 1 Part 2), found by
             // ballots over the depth's candidates (the first equal one counts): stage-2 row
             // 1 + (dep - 1) M + m, or the next marginal row
             const int* cand = topm + (dep < a.gamma && mary ? (dep - 1) * a.M : 0);
-            const int c0 = lane < a.M ? cand[lane] : -1, c1 = lane + 32 < a.M ? cand[lane + 32] : -1;
+            const int c0 = lane < a.M ? cand[lane] : -1;
             const unsigned b0 = __ballot_sync(kFull, lane < a.M && c0 == tok);
-            const unsigned b1 = __ballot_sync(kFull, lane + 32 < a.M && c1 == tok);
-            const int m = b0 ? __ffs(b0) - 1 : b1 ? 32 + __ffs(b1) - 1 : -1;
+            int m = b0 ? __ffs(b0) - 1 : -1;
+            if (a.M > 32) {                            // (the same for every lane)
+                const int c1 = lane + 32 < a.M ? cand[lane + 32] : -1;
+                const unsigned b1 = __ballot_sync(kFull, lane + 32 < a.M && c1 == tok);
+                m = b0 ? m : b1 ? 32 + __ffs(b1) - 1 : -1;
+            }
             const int crow = dep >= a.gamma ? -1 : !mary ? dep : m < 0 ? -1 : ar ? 1 + (dep - 1) * a.M + m : dep;
             const bool sib_ok = rank + 1 < list_len;
             const float slp = l_lp[sib_ok ? idx + 1 : idx];
@@ -826,7 +829,6 @@ __global__ void __launch_bounds__(kFastThreads) build_tree_fast_kernel(TreeArgs 
             const uint32_t ahi = static_cast<uint32_t>(kA >> 32), alo = static_cast<uint32_t>(kA);
             const uint32_t bhi = static_cast<uint32_t>(kB >> 32), blo = static_cast<uint32_t>(kB);
             const int arr = s_first ? hrr + 1 : crow << 10, brr = s_first ? crow << 10 : hrr + 1;
-            const float apsc = s_first ? hpsc : sc, bpsc = s_first ? sc : hpsc;
             // their places among the remaining entries (sorted, so the larger keys are a prefix)
             const int pA = __popc(__ballot_sync(kFull, key_gt(nhi, nlo, ahi, alo)));
             const int pB = __popc(__ballot_sync(kFull, key_gt(nhi, nlo, bhi, blo)));
@@ -837,7 +839,6 @@ __global__ void __launch_bounds__(kFastThreads) build_tree_fast_kernel(TreeArgs 
             khi = takeA ? ahi : takeB ? bhi : fromN ? nhi : fromO ? khi : phi;
             klo = takeA ? alo : takeB ? blo : fromN ? nlo : fromO ? klo : plo;
             rr = takeA ? arr : takeB ? brr : fromN ? nrr : fromO ? rr : prr;
-            psc = takeA ? apsc : takeB ? bpsc : fromN ? npsc : fromO ? psc : ppsc;
         }
         flags = static_cast<int>(__reduce_or_sync(kFull, static_cast<unsigned>(flags)));
         if (count < n_out) flags |= TF_DEV_UNDERFULL;
