@@ -821,13 +821,15 @@ __global__ void __launch_bounds__(kFastThreads) build_tree_fast_kernel(TreeArgs 
                 o_dep[node] = dep;
                 o_score[node] = sc;
             }
-            // its successors, A before B in queue order (0 = none)
-            const unsigned long long sk = sib_ok ? queue_key(hpsc + slp, dep, par) : 0ull;
-            const unsigned long long ckk = ch_ok ? queue_key(sc + clp, dep + 1, node) : 0ull;
-            const bool s_first = sk > ckk;
-            const unsigned long long kA = s_first ? sk : ckk, kB = s_first ? ckk : sk;
-            const uint32_t ahi = static_cast<uint32_t>(kA >> 32), alo = static_cast<uint32_t>(kA);
-            const uint32_t bhi = static_cast<uint32_t>(kB >> 32), blo = static_cast<uint32_t>(kB);
+            // its successors, A before B in queue order (0 = none): the next sibling shares the
+            // head's depth and parent (the low word of its key), the child is one level deeper
+            // with this node as parent
+            const uint32_t shi = sib_ok ? float_key(hpsc + slp) : 0u, slo = sib_ok ? hlo : 0u;
+            const uint32_t chi = ch_ok ? float_key(sc + clp) : 0u;
+            const uint32_t clo = ch_ok ? (static_cast<uint32_t>(126 - dep) << 24) | static_cast<uint32_t>(0xFFFFFF - node) : 0u;
+            const bool s_first = key_gt(shi, slo, chi, clo);
+            const uint32_t ahi = s_first ? shi : chi, alo = s_first ? slo : clo;
+            const uint32_t bhi = s_first ? chi : shi, blo = s_first ? clo : slo;
             const int arr = s_first ? hrr + 1 : crow << 10, brr = s_first ? crow << 10 : hrr + 1;
             // their places among the remaining entries (sorted, so the larger keys are a prefix)
             const int pA = __popc(__ballot_sync(kFull, key_gt(nhi, nlo, ahi, alo)));
