@@ -60,10 +60,6 @@ struct EpiParams {
     int n_cols;                  //          accumulator nb of N tile nt at columns nb * n_total + nt * BN
     int n_total;                 // N of the whole GEMM (n_ntiles * BN)
     int reset_status;            // LMHEAD: zero *status first (the first kernel of a stage-1 call)
-    int row_shift;               // LMHEAD, one CTA per tile: the activation rows occupy tile rows (TMEM
-                                 // lanes) row_shift.. (64 for at most 64 rows, so that the epilogue
-                                 // warps that read them, lanes 64-127, share no SM sub-partition
-                                 // with the producer and MMA warps 0 and 1)
     unsigned long long wait_ns;  // limit of every wait for progress (0: kWaitLimitNs); the waits
                                  // that drain in-flight copies and MMAs always take kWaitLimitNs
     // GATEUP / DOWN with one CTA per SM: units n_full.. (the last, partial round) run as
@@ -274,7 +270,6 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         ptx::tc_fence_after();
     }
     const uint32_t tmem_base = *tmem_slot;
-    const int row_shift = EPI == EPI_LMHEAD && !kPair ? ep.row_shift : 0;
     if (!(warp == 0 && lane == 0)) pdl_wait();   // the producer waits after its weight prefetch
     // a call's status word starts at zero; cleared here, after every earlier kernel has finished,
     // instead of by a separate memset that would end the overlap with the previous kernel
@@ -294,8 +289,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             auto load_x = [&](uint8_t* sp, uint64_t* bar, int j, int kb, int mt) {
                 if constexpr (kPair)
                     ptx::tma_load_2d_pair(sp + j * C::kABytes, &tmap_x, in_leader(bar), kb * kBK, mt * kBM, pol_x);
-                else    // rows above the shift are read out of range: zero fill
-                    ptx::tma_load_2d(sp + j * C::kABytes, &tmap_x, bar, kb * kBK, mt * kBM - row_shift, pol_x);
+                else
+                    ptx::tma_load_2d(sp + j * C::kABytes, &tmap_x, bar, kb * kBK, mt * kBM, pol_x);
             };
             // Weight tiles of one stage; in a pair each CTA stages its half of the rows
             // (tmap_w0's box is BN / 2 rows high).
@@ -476,7 +471,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             const Item itm = item_of(u);
             const Unit w = itm.w;
             const int nt = w.nt;
-            const int row = ((w.mg * m_cl + m_rank) * MT + (MT == 2 ? g : 0)) * kBM + q * 32 + lane - row_shift;
+            const int row = ((w.mg * m_cl + m_rank) * MT + (MT == 2 ? g : 0)) * kBM + q * 32 + lane;
             const uint32_t tb = tmem_base + 256u * g + (static_cast<uint32_t>(q * 32) << 16);
 
             if (kTail && itm.chunk >= 0) {
@@ -565,7 +560,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 constexpr int kHalf = kChunks / 2;
                 const Partials& P = ep.partials;
                 // warps whose 32 rows are all padding skip the accumulators entirely
-                if (row - lane < n_rows && row - lane + 31 >= 0) {
+                if (row - lane < n_rows) {
                     float hm = -INFINITY, hsum = 0.0f, hbv = -INFINITY;
                     int hbid = -1;
                     // half summary; chunks arrive in id order, so strict > keeps the smaller id
@@ -579,7 +574,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                             hsum = hsum * __expf(hm - mn) + c.s * __expf(c.a1 - mn);
                             hm = mn;
                         }
-                        if (row >= 0 && row < n_rows)
+                        if (row < n_rows)
                             P.chunks[P.chunk_at(nt, ci, row)] =
                                 make_float4(c.a1, c.a2, c.a3, __int_as_float(c.i1 | (c.i2 << 8)));
                     };
@@ -612,7 +607,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                             ptx::tmem_wait_ld_regs(rb);
                         }
                     }
-                    if (row >= 0 && row < n_rows)
+                    if (row < n_rows)
                         P.halves[P.half_at(nt, half, row)] = make_float4(hm, hsum, hbv, __int_as_float(hbid));
                 }
                 release_slot(g);
@@ -983,7 +978,6 @@ cudaError_t launch_lmhead_tc(const Ctx& ctx, const void* lm_head, const void* x,
     ep.V = V;
     ep.inv_temp = inv_temp;
     ep.reset_status = reset_status ? 1 : 0;
-    ep.row_shift = n_rows <= 64 ? 64 : 0;
     if (m_tiles == 1) return run_gemm<EPI_LMHEAD, 1, 1, kBlockV, 4>(ctx, tx, tw, tw, n_rows, d, n_tiles, 1, ep);
     return run_gemm<EPI_LMHEAD, 1, 1, kBlockV, 7, 2>(ctx, tx, tw, tw, n_rows, d, n_tiles, (m_tiles + 1) / 2, ep);
 }
