@@ -673,8 +673,9 @@ __global__ void __launch_bounds__(kTreeThreads) build_tree_reg_kernel(TreeArgs a
 // lane 0's entry, tests its token against the stage-1 candidates of its depth with a ballot
 // (the M-ary rule), and places its two successors (next sibling, first child) with two ballots
 // over the remaining keys; every lane then takes its new entry from itself or a neighbour by
-// shuffle. There is no warp-wide max and no divergent branch; a pop costs about 300 ns on
-// GB300, a chain of some hundred dependent single-warp instructions.
+// shuffle. There is no warp-wide max and no divergent branch. The queue carries keys and list
+// entries only (a sibling's parent score is the placed parent's o_score); a pop costs about
+// 250 ns on GB300, a chain of about a hundred dependent single-warp instructions.
 // ------------------------------------------------------------------------------------------
 constexpr int kFastThreads = 512;
 // Shared-memory bytes of build_tree_fast_kernel: nodes, candidates, mask bits and the staged
