@@ -617,7 +617,7 @@ def run_gpu(args):
                           "peak_gbs": peak, "frac": step_bytes / (ms_per_step / 1e3) / 1e9 / peak,
                           "peak_kind": peak_kind, "nominal_gbs": NOMINAL_HBM_GBS,
                           "frac_nominal": step_bytes / (ms_per_step / 1e3) / 1e9 / NOMINAL_HBM_GBS,
-                          "target": "70 % of the HBM roofline, judged against the measured copy rate "
+                          "target": "70 % of the HBM roofline, stated against the measured copy rate "
                                     "(peak_gbs); frac_nominal is the same figure against 8 TB/s"},
         "roofline": roofline,
         "clocks": clocks, "e2e": e2e, "gpu_launches": gpu_launches,

@@ -26,7 +26,7 @@ def declared_functions():
     return sorted(set(re.findall(r"\b(tf_[a-z0-9_]+)\s*\(", src)))
 
 
-def test_header_declares_the_north_star_calls():
+def test_header_declares_the_four_calls_of_the_path():
     names = declared_functions()
     for n in ("tf_stage1_marginals", "tf_stage2_ar_approx", "tf_build_tree", "tf_tree_mask"):
         assert n in names
